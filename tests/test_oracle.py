@@ -1,0 +1,286 @@
+"""Pins of the CPU oracle against things other than itself (CPU only).
+
+Each check targets a plausible mistake: a dropped term (router term of dx,
+bias), a wrong sign (softmax Jacobian), a transposed operand (non-square
+d != F everywhere), a wrong index (gate/up halves, slot order), a wrong
+inequality or tie-break in the pruning rule.
+"""
+import json
+import math
+import os
+
+import numpy as np
+import pytest
+import torch
+
+from oracle import moe_oracle as O
+from paper_2601_14327_gb300 import synth
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+
+
+def _case(T=24, d=40, E=6, k=2, F=24, bias="zipf", seed=3, std=0.2):
+    inp = synth.make_layer_inputs(T, d, E, k, F, bias=bias, seed=seed, weight_std=std)
+    return {n: v.double().numpy() for n, v in inp.items()}
+
+
+# ---------------------------------------------------------------- routing ---
+
+def test_router_logits_brute_force():
+    c = _case(T=7, d=9, E=5, k=2)
+    z = O.router_logits(c["x"], c["w_router"], c["bias"])
+    for t in range(7):
+        for e in range(5):
+            s = math.fsum(c["x"][t, i] * c["w_router"][i, e] for i in range(9)) + c["bias"][e]
+            assert z[t, e] == np.float32(s)
+
+
+def test_route_topk_brute_force_with_ties_and_mask():
+    rng = np.random.default_rng(0)
+    T, E, k = 50, 8, 3
+    # few distinct values -> many exact ties
+    z = rng.integers(-3, 3, size=(T, E)).astype(np.float32)
+    mask = np.array([1, 1, 0, 1, 1, 1, 0, 1], np.uint8)
+    zm = O.apply_mask(z, mask)
+    idx, g = O.route_topk(zm, k)
+    for t in range(T):
+        cand = [(-float(zm[t, e]), e) for e in range(E) if mask[e]]
+        cand.sort()
+        want = [e for (_, e) in cand[:k]]
+        assert list(idx[t]) == want
+        sel = [float(z[t, e]) for e in want]
+        m = max(sel)
+        den = sum(math.exp(s - m) for s in sel)
+        for j in range(k):
+            assert abs(g[t, j] - math.exp(sel[j] - m) / den) < 1e-14
+    assert not np.isin(idx, np.nonzero(mask == 0)[0]).any()
+
+
+def test_gates_k_equals_active_is_plain_softmax():
+    c = _case(T=10, d=16, E=5, k=5)
+    z = O.router_logits(c["x"], c["w_router"], c["bias"])
+    idx, g = O.route_topk(z, 5)
+    ref = torch.softmax(torch.from_numpy(z.astype(np.float64)), dim=1).numpy()
+    got = np.zeros_like(ref)
+    np.put_along_axis(got, idx.astype(np.int64), g, axis=1)
+    np.testing.assert_allclose(got, ref, rtol=0, atol=1e-14)
+    np.testing.assert_allclose(g.sum(1), 1.0, atol=1e-14)
+
+
+def test_route_rejects_k_above_active():
+    z = O.apply_mask(np.zeros((2, 4), np.float32), np.array([1, 0, 0, 1], np.uint8))
+    with pytest.raises(ValueError):
+        O.route_topk(z, 3)
+
+
+def test_counts_invariants():
+    c = _case(T=200, d=16, E=12, k=3)
+    mask = np.ones(12, np.uint8)
+    mask[[1, 5, 7]] = 0
+    z = O.router_logits(c["x"], c["w_router"], c["bias"], mask)
+    idx, _ = O.route_topk(z, 3)
+    cnt = O.expert_counts(idx, 12)
+    assert cnt.sum() == 200 * 3
+    assert (cnt[[1, 5, 7]] == 0).all()
+    for e in range(12):
+        assert cnt[e] == sum(1 for t in range(200) for j in range(3) if idx[t, j] == e)
+
+
+# ------------------------------------------------------------ permutation ---
+
+@pytest.mark.parametrize("pad", [1, 4, 128])
+def test_permutation_brute_force_and_round_trip(pad):
+    c = _case(T=37, d=8, E=5, k=2)
+    idx, g = O.route_topk(O.router_logits(c["x"], c["w_router"], c["bias"]), 2)
+    off, cnt, row = O.permutation(idx, 5, pad)
+    assert (off[1:] - off[:-1] >= cnt).all() and (off % pad == 0).all()
+    for e in range(5):
+        pairs = sorted((t, j) for t in range(37) for j in range(2) if idx[t, j] == e)
+        for r, (t, j) in enumerate(pairs):
+            assert row[t, j] == off[e] + r
+    # round trip: gather rows into the grouped layout, combine back with gates
+    # that sum to one -> the identity
+    xrep = np.repeat(c["x"][:, None, :], 2, axis=1)
+    xperm = O.to_permuted(xrep, row, int(off[-1]))
+    assert (xperm[row.reshape(-1)] == xrep.reshape(-1, 8)).all()
+    back = np.einsum("tj,tjd->td", g, xperm[row])
+    np.testing.assert_allclose(back, c["x"], rtol=0, atol=1e-14)
+    # unit weight per slot: the gather is exactly the inverse
+    assert (xperm[row[:, 1]] == c["x"]).all()
+
+
+# ------------------------------------------------------------- expert FFN ---
+
+def test_single_expert_is_dense_swiglu_mlp():
+    c = _case(T=9, d=12, E=1, k=1, F=20)
+    out = O.moe_layer(c["x"], c["w_router"], c["bias"], None, 1, c["w_gate_up"], c["w_down"])
+    x = torch.from_numpy(c["x"])
+    wg = torch.from_numpy(c["w_gate_up"][0, :20])
+    wu = torch.from_numpy(c["w_gate_up"][0, 20:])
+    wd = torch.from_numpy(c["w_down"][0])
+    ref = (torch.nn.functional.silu(x @ wg.T) * (x @ wu.T)) @ wd.T
+    np.testing.assert_allclose(out["y"], ref.numpy(), rtol=1e-12, atol=1e-13)
+    assert (out["gates"] == 1.0).all()
+
+
+def _torch_layer(c, idx, k):
+    """Same layer through torch fp64 autograd with the routing held fixed."""
+    x = torch.tensor(c["x"], requires_grad=True)
+    wr = torch.tensor(c["w_router"], requires_grad=True)
+    b = torch.tensor(c["bias"])
+    wgu = torch.tensor(c["w_gate_up"], requires_grad=True)
+    wd = torch.tensor(c["w_down"], requires_grad=True)
+    F = wgu.shape[1] // 2
+    z = x @ wr + b
+    # the router's logits are fp32 values: round them, let the gradient through
+    z = z + (z.detach().float().double() - z.detach())
+    ix = torch.from_numpy(idx.astype(np.int64))
+    g = torch.softmax(torch.gather(z, 1, ix), dim=1)
+    y = torch.zeros_like(x)
+    for j in range(k):
+        e = ix[:, j]
+        a = torch.einsum("td,tfd->tf", x, wgu[e, :F])
+        bb = torch.einsum("td,tfd->tf", x, wgu[e, F:])
+        o = torch.einsum("tf,tdf->td", torch.nn.functional.silu(a) * bb, wd[e])
+        y = y + g[:, j:j + 1] * o
+    loss = (y * torch.tensor(c["dy"])).sum()
+    loss.backward()
+    return y.detach().numpy(), x.grad.numpy(), wr.grad.numpy(), wgu.grad.numpy(), wd.grad.numpy()
+
+
+@pytest.mark.parametrize("E,k", [(6, 2), (5, 5), (7, 1)])
+def test_forward_backward_against_torch_autograd(E, k):
+    c = _case(T=30, d=20, E=E, k=k, F=12)
+    out = O.moe_layer(c["x"], c["w_router"], c["bias"], None, k, c["w_gate_up"], c["w_down"],
+                      dy=c["dy"])
+    y, dx, dwr, dwgu, dwd = _torch_layer(c, out["topk_idx"], k)
+    np.testing.assert_allclose(out["y"], y, rtol=1e-11, atol=1e-12)
+    np.testing.assert_allclose(out["dx"], dx, rtol=1e-10, atol=1e-12)
+    np.testing.assert_allclose(out["dw_router"], dwr, rtol=1e-10, atol=1e-12)
+    np.testing.assert_allclose(out["dw_gate_up"], dwgu, rtol=1e-10, atol=1e-12)
+    np.testing.assert_allclose(out["dw_down"], dwd, rtol=1e-10, atol=1e-12)
+
+
+def test_backward_finite_differences():
+    """Central differences of L = <dy, y> with the routing held fixed."""
+    c = _case(T=12, d=10, E=4, k=2, F=8, seed=11)
+    base = O.moe_layer(c["x"], c["w_router"], c["bias"], None, 2, c["w_gate_up"], c["w_down"],
+                       dy=c["dy"])
+    idx = base["topk_idx"]
+
+    def loss(cc):
+        # fixed routing, fp64 logits so that the difference quotient is smooth
+        z = np.asarray(cc["x"]) @ cc["w_router"] + cc["bias"]
+        sel = np.take_along_axis(z, idx.astype(np.int64), axis=1)
+        ex = np.exp(sel - sel.max(1, keepdims=True))
+        g = ex / ex.sum(1, keepdims=True)
+        y = O.moe_forward(cc["x"], idx, g, cc["w_gate_up"], cc["w_down"])["y"]
+        return float((y * cc["dy"]).sum())
+
+    rng = np.random.default_rng(5)
+    h = 1e-6
+    for name, grad in [("x", "dx"), ("w_router", "dw_router"), ("w_gate_up", "dw_gate_up"),
+                       ("w_down", "dw_down")]:
+        for _ in range(6):
+            pos = tuple(int(rng.integers(0, s)) for s in c[name].shape)
+            if name == "w_gate_up":
+                e = pos[0]
+                if not (idx == e).any():
+                    continue
+            cp = {n: v.copy() for n, v in c.items()}
+            cm = {n: v.copy() for n, v in c.items()}
+            cp[name][pos] += h
+            cm[name][pos] -= h
+            num = (loss(cp) - loss(cm)) / (2 * h)
+            ana = base[grad][pos]
+            assert abs(num - ana) <= 1e-6 * max(1.0, abs(ana)), (name, pos, num, ana)
+
+
+def test_zero_count_expert_has_zero_weight_grads():
+    c = _case(T=40, d=16, E=6, k=2, F=8)
+    mask = np.array([1, 1, 0, 1, 1, 1], np.uint8)
+    out = O.moe_layer(c["x"], c["w_router"], c["bias"], mask, 2, c["w_gate_up"], c["w_down"],
+                      dy=c["dy"])
+    assert out["counts"][2] == 0
+    assert (out["dw_gate_up"][2] == 0).all() and (out["dw_down"][2] == 0).all()
+    assert (out["dw_router"][:, 2] == 0).all()
+
+
+def test_per_element_evaluators_match_grouped_oracle():
+    c = _case(T=25, d=18, E=5, k=3, F=10)
+    out = O.moe_layer(c["x"], c["w_router"], c["bias"], None, 3, c["w_gate_up"], c["w_down"],
+                      dy=c["dy"])
+    for t in [0, 7, 24]:
+        y, _ = O.token_forward(c["x"][t], out["topk_idx"][t], out["gates"][t],
+                               c["w_gate_up"], c["w_down"])
+        np.testing.assert_allclose(y, out["y"][t], rtol=1e-12, atol=1e-13)
+        dx, dg, dz = O.token_backward(c["dy"][t], c["x"][t], out["topk_idx"][t], out["gates"][t],
+                                      c["w_router"], c["w_gate_up"], c["w_down"])
+        np.testing.assert_allclose(dx, out["dx"][t], rtol=1e-11, atol=1e-12)
+        np.testing.assert_allclose(dz, out["d_logits"][t], rtol=1e-11, atol=1e-13)
+    e = int(np.argmax(out["counts"]))
+    t, j = np.nonzero(out["topk_idx"] == e)
+    dwd, dwg, dwu = O.expert_weight_grad_columns(e, [0, 3, 9], c["x"][t], c["dy"][t],
+                                                 out["gates"][t, j], c["w_gate_up"], c["w_down"])
+    np.testing.assert_allclose(dwd, out["dw_down"][e][:, [0, 3, 9]].T, rtol=1e-11, atol=1e-12)
+    np.testing.assert_allclose(dwg, out["dw_gate_up"][e][[0, 3, 9]], rtol=1e-11, atol=1e-12)
+    np.testing.assert_allclose(dwu, out["dw_gate_up"][e][[10, 13, 19]], rtol=1e-11, atol=1e-12)
+
+
+def test_three_matrix_expert_matches_table_a1_parameter_counts():
+    """Table A1: 1515B model (103 layers, 64 experts, hidden 4608, FFN 16384) and
+    20B model (48 layers, 64 experts, hidden 1024, FFN 2048, 19.91B in Table 4).
+    Expert parameters with the oracle's three matrices (gate, up, down) land
+    just under the totals; two matrices would miss them by a third."""
+    def expert_params(L, E, d, F, mats):
+        return L * E * mats * d * F
+    big3 = expert_params(103, 64, 4608, 16384, 3)
+    small3 = expert_params(48, 64, 1024, 2048, 3)
+    assert 0.95 < big3 / 1515e9 < 1.0 and 0.95 < small3 / 19.91e9 < 1.0
+    assert expert_params(103, 64, 4608, 16384, 2) / 1515e9 < 0.7
+
+
+# ----------------------------------------------------------- LAEP pruning ---
+
+def _golden():
+    with open(os.path.join(GOLDEN, "laep_prune_cases.json")) as f:
+        return json.load(f)
+
+
+@pytest.mark.parametrize("case", _golden()["alpha_beta"], ids=lambda c: c["name"])
+def test_prune_alpha_beta_golden(case):
+    mask, n = O.prune_mask_alpha_beta(case["counts"], case["S"], case["k"], case["alpha"],
+                                      case["beta"])
+    assert list(mask) == case["mask"] and n == case["n_pruned"]
+
+
+@pytest.mark.parametrize("case", _golden()["lowest"], ids=lambda c: c["name"])
+def test_prune_lowest_golden(case):
+    mask, n = O.prune_mask_lowest(case["counts"], case["P"], case["k"])
+    assert list(mask) == case["mask"] and n == case["n_pruned"]
+
+
+def test_prune_alpha_beta_brute_force_prefix():
+    """Position r of the ascending order is pruned iff the load sum of positions
+    0..r is below S*k*beta and its load is below S*k*alpha/E (both conditions
+    only get harder along the order, so the pruned set is a prefix)."""
+    rng = np.random.default_rng(1)
+    for _ in range(300):
+        E = int(rng.integers(2, 12))
+        k = int(rng.integers(1, E + 1))
+        S = int(rng.integers(1, 50))
+        counts = rng.multinomial(S * k, rng.dirichlet(np.full(E, 0.3)))
+        alpha, beta = float(rng.uniform(0, 2)), float(rng.uniform(0, 0.6))
+        mask, n = O.prune_mask_alpha_beta(counts, S, k, alpha, beta)
+        order = sorted(range(E), key=lambda e: (counts[e], e))
+        want = np.ones(E, np.uint8)
+        pruned = 0
+        for r, e in enumerate(order):
+            prefix = sum(int(counts[q]) for q in order[:r + 1])
+            ok = prefix < S * k * beta and counts[e] < S * k * alpha / E
+            if ok and pruned < E - k:
+                want[e] = 0
+                pruned += 1
+        assert (mask == want).all() and n == pruned
+        kept = [order.index(e) for e in range(E) if mask[e] == 0]
+        assert sorted(kept) == list(range(len(kept)))  # a prefix of the order

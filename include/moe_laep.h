@@ -1,0 +1,242 @@
+/*
+ * moe_laep.h - C ABI of the GB300 (sm_103a) MoE expert-layer hot path that
+ * Layer-Adaptive Expert Pruning (LAEP; Yuan3.0 Ultra report, arXiv 2601.14327)
+ * accelerates during pre-training.
+ *
+ * One MoE layer step on one GPU:
+ *   moe_route              router logits, top-k, gates, per-expert histogram
+ *   moe_load_stats         per-expert histogram of an existing routing
+ *   laep_prune_mask        LAEP pruning decision (host)
+ *   moe_permute            contiguous per-expert groups of token rows
+ *   moe_grouped_ffn_fwd    grouped SwiGLU expert FFN (tcgen05 / TMEM / TMA)
+ *   moe_unpermute_combine  gate-weighted combine back to token order
+ * and the backward companions moe_unpermute_combine_bwd, moe_grouped_ffn_bwd,
+ * moe_route_bwd, moe_permute_bwd.
+ *
+ * Conventions (all entry points):
+ *  - Pointers are DEVICE pointers owned by the caller unless marked "host".
+ *    The library allocates no memory; scratch comes from the caller's `ws`
+ *    (size from moe_workspace_size) or from explicit scratch arguments.
+ *  - bf16 tensors are passed as uint16_t (IEEE bfloat16 bit patterns).
+ *  - Every device call is asynchronous on `stream` (NULL = legacy default
+ *    stream) and returns a status: MOE_OK, or a negative MOE_ERR_* when the
+ *    host-side argument check failed (nothing was launched) or a launch
+ *    failed. moe_last_error_string() describes the last failure of the
+ *    calling thread.
+ *  - Problems the kernels detect on the device (an expert id out of range,
+ *    fewer than k live experts, a histogram that disagrees with the routing,
+ *    a bounded wait that expired) are recorded in a device error word, read
+ *    with moe_device_error(). Kernels never trap.
+ *  - Row-major layouts. Shapes use T tokens, d = d_model, E experts (pruned
+ *    ones included), k experts per token, F = d_ff, A = T*k assignments and
+ *    R = moe_perm_rows_max(T,k,E) rows in the grouped (permuted) layout.
+ *  - Grouped layout: group e holds the assignments routed to expert e in
+ *    (token, slot) order; it starts at group_offsets[e], a multiple of 128,
+ *    and its rows past group_counts[e] up to group_offsets[e+1] are zero
+ *    padding. group_offsets[E] is the number of rows in use (<= R).
+ */
+#ifndef MOE_LAEP_H
+#define MOE_LAEP_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Same type as cudaStream_t. */
+typedef struct CUstream_st *moe_stream_t;
+
+enum {
+  MOE_OK = 0,
+  MOE_ERR_ARG = -1,          /* invalid argument: null pointer, size or alignment */
+  MOE_ERR_UNSUPPORTED = -2,  /* valid but outside the supported shapes */
+  MOE_ERR_CUDA = -3,         /* a CUDA runtime/driver call failed */
+  MOE_ERR_INVARIANT = -4,    /* a device-side consistency check failed */
+  MOE_ERR_TIMEOUT = -5,      /* a bounded device-side wait expired */
+  MOE_ERR_WORKSPACE = -6     /* workspace too small */
+};
+
+/* Codes stored in the device error word (first error wins). */
+enum {
+  MOE_DEV_OK = 0,
+  MOE_DEV_BAD_EXPERT = 1,    /* topk_idx entry outside [0, E) */
+  MOE_DEV_TOO_FEW_LIVE = 2,  /* a token saw fewer than k live experts */
+  MOE_DEV_COUNT_MISMATCH = 3,/* counts disagree with the routing */
+  MOE_DEV_WAIT_TIMEOUT = 4,  /* a pipeline wait in a GEMM kernel gave up */
+  MOE_DEV_ROWS_OVERFLOW = 5  /* grouped layout would exceed R rows */
+};
+
+/* Library version (major*10000 + minor*100 + patch). */
+int moe_version(void);
+
+/* Text of the last error of the calling thread ("" if none). */
+const char *moe_last_error_string(void);
+
+/* Reads the device error word into *code (MOE_DEV_*), clearing it when
+ * `clear` is nonzero. Synchronizes the current device first. Returns MOE_OK
+ * or MOE_ERR_CUDA. */
+int moe_device_error(int *code, int clear);
+
+/* Rows to allocate for every grouped-layout buffer: T*k + 128*E. */
+int64_t moe_perm_rows_max(int T, int k, int E);
+
+/* Bytes of scratch `ws` every device entry point below may use for a layer of
+ * this shape (one buffer serves all calls of a step issued on one stream). */
+size_t moe_workspace_size(int T, int d, int E, int k, int F);
+
+/*
+ * moe_route - router of the MoE layer: which experts each token goes to.
+ * Sec. 3.2 defines the routing indicator E[i,j,l] (token j of layer l sent to
+ * expert i) and Sec. 4 / Table 5 require pruned experts to receive no token;
+ * the router itself is an fp32 linear layer with a fixed bias.
+ *   z[t,e] = sum_i x[t,i] * w_router[i,e] + bias[e]     (fp32 FFMA)
+ *   z[t,e] = -inf where active_mask[e] == 0
+ *   topk_idx[t,0..k-1] = the k largest z (descending, ties to lower index)
+ *   topk_gate[t,j]     = softmax over the k selected z (fp32)
+ *   counts[e]          = #{(t,j) : topk_idx[t,j] == e}   (overwritten)
+ * x [T,d] bf16; w_router [d,E] fp32; bias [E] fp32 or NULL; active_mask [E]
+ * uint8 or NULL (all live); logits_in [T,E] fp32 or NULL: when given it
+ * replaces x*w_router+bias (x, w_router, bias are then not read; the mask is
+ * still applied); logits_out [T,E] fp32 or NULL receives the masked z;
+ * topk_idx [T,k] int32; topk_gate [T,k] fp32; counts [E] int32 or NULL.
+ * Limits: 1 <= E <= 256, 1 <= k <= min(E, 8), d % 8 == 0, T >= 0.
+ * A token with fewer than k live experts sets MOE_DEV_TOO_FEW_LIVE.
+ */
+int moe_route(const uint16_t *x, const float *w_router, const float *bias,
+              const uint8_t *active_mask, int T, int d, int E, int k,
+              const float *logits_in, float *logits_out, int32_t *topk_idx,
+              float *topk_gate, int32_t *counts, moe_stream_t stream);
+
+/*
+ * moe_load_stats - per-expert token number of one routing: the ETN statistic
+ * of Algorithm 1 Step 1 (and the left-hand side of Eq. 1).
+ *   counts[e] (+)= #{(t,j) : topk_idx[t,j] == e}
+ * topk_idx [T,k] int32; counts [E] int32, overwritten when accumulate == 0,
+ * added to otherwise (recording over iterations). Out-of-range ids are
+ * skipped and set MOE_DEV_BAD_EXPERT.
+ */
+int moe_load_stats(const int32_t *topk_idx, int T, int k, int E, int32_t *counts,
+                   int accumulate, moe_stream_t stream);
+
+/*
+ * laep_prune_mask - LAEP expert-pruning decision for one layer (HOST call).
+ * Sec. 3.2 Eq. 1-2 and Algorithm 1 (one histogram): experts are visited in
+ * ascending load order (ties: lower index first); with a running load sum,
+ * an expert is pruned when the sum is < S*k*beta and its own load is
+ * < S*k*alpha/E (E = experts before pruning). With prune_count >= 0 the rule
+ * is instead "prune the prune_count least-loaded experts" (the largest=False
+ * top-K of Eq. 2). At least k experts are always kept.
+ * counts_host [E] int32 (host); S = tokens of the layer; active_mask_host [E]
+ * uint8 (host, out: 1 keep, 0 pruned); n_pruned (host, out, may be NULL).
+ */
+int laep_prune_mask(const int32_t *counts_host, int E, int64_t S, int k, double alpha,
+                    double beta, int prune_count, uint8_t *active_mask_host, int *n_pruned);
+
+/*
+ * moe_permute - dispatch: token rows into contiguous per-expert groups
+ * (the data movement of expert-parallel dispatch, Sec. 3.3, on one GPU).
+ * Stable counting sort of the A assignments by (expert, token, slot), then
+ * x_perm[row_of_assignment[t*k+j], :] = x[t, :]; padding rows are zeroed.
+ * x [T,d] bf16; topk_idx [T,k] int32; counts [E] int32 or NULL: when given it
+ * is checked against the routing (MOE_DEV_COUNT_MISMATCH); rows_cap = rows
+ * allocated in x_perm (>= moe_perm_rows_max); outputs group_offsets [E+1]
+ * int32, group_counts [E] int32, row_of_assignment [T,k] int32,
+ * x_perm [rows_cap, d] bf16. Limits: d % 8 == 0, E <= 256.
+ */
+int moe_permute(const uint16_t *x, const int32_t *topk_idx, const int32_t *counts, int T,
+                int d, int E, int k, int64_t rows_cap, int32_t *group_offsets,
+                int32_t *group_counts, int32_t *row_of_assignment, uint16_t *x_perm,
+                void *ws, size_t ws_bytes, moe_stream_t stream);
+
+/*
+ * moe_grouped_ffn_fwd - the experts' SwiGLU FFN over the grouped layout.
+ * Table A1 fixes three matrices per expert (gate, up, down); for each group
+ * e with rows X_e:
+ *   [A_e | B_e] = X_e * W_gate_up[e]^T;  H_e = silu(A_e) * B_e;
+ *   O_e = H_e * W_down[e]^T
+ * bf16 operands, fp32 accumulation in tensor memory, bf16 results.
+ * x_perm [rows_cap,d]; group_offsets [E+1]; w_gate_up [E,2F,d] bf16 (rows
+ * 0..F-1 gate, F..2F-1 up); w_down [E,d,F] bf16; outputs ab_saved
+ * [rows_cap,2F] bf16 (A in columns 0..F-1, B in F..2F-1; kept for the
+ * backward), h [rows_cap,F] bf16, out_perm [rows_cap,d] bf16. Only rows below
+ * group_offsets[E] are written. Groups of 0 rows cost nothing.
+ * Limits: d % 128 == 0, F % 128 == 0, all pointers 16-byte aligned.
+ */
+int moe_grouped_ffn_fwd(const uint16_t *x_perm, const int32_t *group_offsets, int E, int d,
+                        int F, int64_t rows_cap, const uint16_t *w_gate_up,
+                        const uint16_t *w_down, uint16_t *ab_saved, uint16_t *h,
+                        uint16_t *out_perm, void *ws, size_t ws_bytes, moe_stream_t stream);
+
+/*
+ * moe_unpermute_combine - gate-weighted combine back to token order:
+ *   y[t,:] = sum_j topk_gate[t,j] * out_perm[row_of_assignment[t,j], :]
+ * summed in fp32, rounded once to bf16. out_perm [rows_cap,d] bf16;
+ * row_of_assignment [T,k]; topk_gate [T,k] fp32; y [T,d] bf16. d % 8 == 0.
+ */
+int moe_unpermute_combine(const uint16_t *out_perm, const int32_t *row_of_assignment,
+                          const float *topk_gate, int T, int d, int k, uint16_t *y,
+                          moe_stream_t stream);
+
+/*
+ * moe_unpermute_combine_bwd - backward of the combine:
+ *   d_out_perm[row(t,j), :] = topk_gate[t,j] * dy[t, :]   (bf16)
+ *   d_gate[t,j] = <dy[t,:], out_perm[row(t,j),:]>         (fp32)
+ * and zeroes the padding rows of d_out_perm (group_offsets/group_counts from
+ * moe_permute). dy [T,d] bf16; d_out_perm [rows_cap,d] bf16; d_gate [T,k].
+ */
+int moe_unpermute_combine_bwd(const uint16_t *dy, const uint16_t *out_perm,
+                              const int32_t *row_of_assignment, const float *topk_gate,
+                              const int32_t *group_offsets, const int32_t *group_counts,
+                              int T, int d, int E, int k, uint16_t *d_out_perm,
+                              float *d_gate, moe_stream_t stream);
+
+/*
+ * moe_grouped_ffn_bwd - backward of moe_grouped_ffn_fwd (dgrad and wgrad):
+ *   dH_e = dO_e * W_down[e];  dA_e = dH_e * B_e * silu'(A_e);
+ *   dB_e = dH_e * silu(A_e);  dX_e = [dA_e | dB_e] * W_gate_up[e]
+ *   dW_down[e] = dO_e^T * H_e;  dW_gate_up[e] = [dA_e | dB_e]^T * X_e
+ * Experts whose group is empty get exactly zero weight gradients.
+ * d_out_perm [rows_cap,d] (padding rows zero); x_perm, ab_saved, h from the
+ * forward; d_ab [rows_cap,2F] bf16 caller scratch (receives [dA|dB]);
+ * outputs dx_perm [rows_cap,d] bf16, dw_gate_up [E,2F,d] bf16,
+ * dw_down [E,d,F] bf16 (fp32 accumulation). Limits as in the forward.
+ */
+int moe_grouped_ffn_bwd(const uint16_t *d_out_perm, const uint16_t *x_perm,
+                        const uint16_t *ab_saved, const uint16_t *h,
+                        const int32_t *group_offsets, int E, int d, int F, int64_t rows_cap,
+                        const uint16_t *w_gate_up, const uint16_t *w_down, uint16_t *d_ab,
+                        uint16_t *dx_perm, uint16_t *dw_gate_up, uint16_t *dw_down, void *ws,
+                        size_t ws_bytes, moe_stream_t stream);
+
+/*
+ * moe_route_bwd - backward of the router's softmax over the selected experts:
+ *   d_logits[t,j] = g[t,j] * (d_gate[t,j] - sum_i g[t,i] * d_gate[t,i])
+ *   dw_router[:, e] = sum over assignments (t,j) to e of d_logits[t,j] * x[t,:]
+ * (the bias is fixed, unselected and pruned experts get zero). x_perm is the
+ * grouped copy of x from moe_permute. d_logits [T,k] fp32 (out);
+ * dw_router [d,E] fp32 (out, overwritten).
+ */
+int moe_route_bwd(const uint16_t *x_perm, const int32_t *topk_idx, const float *topk_gate,
+                  const float *d_gate, const int32_t *row_of_assignment,
+                  const int32_t *group_offsets, const int32_t *group_counts, int T, int d,
+                  int E, int k, int64_t rows_cap, float *d_logits, float *dw_router, void *ws,
+                  size_t ws_bytes, moe_stream_t stream);
+
+/*
+ * moe_permute_bwd - gradient of the layer input:
+ *   dx[t,:] = sum_j dx_perm[row(t,j), :] + sum_j d_logits[t,j] * w_router[:, e_j]
+ * summed in fp32, one bf16 rounding. d_logits and w_router may both be NULL
+ * (no router term). dx [T,d] bf16 (out).
+ */
+int moe_permute_bwd(const uint16_t *dx_perm, const int32_t *row_of_assignment,
+                    const int32_t *topk_idx, const float *d_logits, const float *w_router,
+                    int T, int d, int E, int k, uint16_t *dx, void *ws, size_t ws_bytes,
+                    moe_stream_t stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* MOE_LAEP_H */

@@ -1,0 +1,133 @@
+// Host-side entry points: errors, sizes, and the LAEP pruning decision.
+#include <stdarg.h>
+#include <stdio.h>
+
+#include <algorithm>
+#include <numeric>
+#include <vector>
+
+#include "common.cuh"
+
+namespace moe {
+
+static thread_local char g_err_text[512] = "";
+
+int set_error(int code, const char *fmt, ...) {
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(g_err_text, sizeof(g_err_text), fmt, ap);
+  va_end(ap);
+  return code;
+}
+
+int cuda_status(cudaError_t e, const char *what) {
+  if (e == cudaSuccess) return MOE_OK;
+  return set_error(MOE_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+int launch_status(const char *what) { return cuda_status(cudaGetLastError(), what); }
+
+int num_sms() {
+  static int cached[64] = {0};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 148;
+  if (!cached[dev]) {
+    int n = 0;
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0)
+      n = 148;
+    cached[dev] = n;
+  }
+  return cached[dev];
+}
+
+static size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
+
+WsLayout ws_layout(int T, int d, int E, int k, int F) {
+  (void)F;
+  WsLayout w{};
+  const int64_t A = int64_t(T) * k;
+  const int64_t nblk = std::max<int64_t>(1, (A + kPermChunk - 1) / kPermChunk);
+  const int64_t rows = moe_perm_rows_max(T, k, E);
+  size_t off = 0;
+  w.perm_hist = off;
+  off += align256(size_t(E) * nblk * 4);
+  w.dz_perm = off;
+  off += align256(size_t(rows) * 4);
+  w.rb_partial = off;
+  off += align256(size_t(rows / kGroupPad) * d * 4);
+  w.w_router_t = off;
+  off += align256(size_t(E) * d * 4);
+  w.total = off;
+  return w;
+}
+
+}  // namespace moe
+
+extern "C" {
+
+int moe_version(void) { return 100; }
+
+const char *moe_last_error_string(void) { return moe::g_err_text; }
+
+int64_t moe_perm_rows_max(int T, int k, int E) {
+  if (T < 0 || k < 0 || E < 0) return 0;
+  return int64_t(T) * k + int64_t(moe::kGroupPad) * E;
+}
+
+size_t moe_workspace_size(int T, int d, int E, int k, int F) {
+  if (T < 0 || d <= 0 || E <= 0 || k <= 0) return 0;
+  return moe::ws_layout(T, d, E, k, F).total;
+}
+
+int moe_device_error(int *code, int clear) {
+  if (!code) return moe::set_error(MOE_ERR_ARG, "moe_device_error: null code");
+  int st = moe::cuda_status(cudaDeviceSynchronize(), "moe_device_error: synchronize");
+  if (st) return st;
+  int c0 = 0, c1 = 0, c2 = 0;
+  if ((st = moe::route_dev_error(clear, &c0))) return st;
+  if ((st = moe::permute_dev_error(clear, &c1))) return st;
+  if ((st = moe::gemm_dev_error(clear, &c2))) return st;
+  *code = c0 ? c0 : (c1 ? c1 : c2);
+  return MOE_OK;
+}
+
+// LAEP pruning decision (Sec. 3.2 Eq. 1-2, Algorithm 1 with one histogram).
+int laep_prune_mask(const int32_t *counts_host, int E, int64_t S, int k, double alpha,
+                    double beta, int prune_count, uint8_t *active_mask_host, int *n_pruned) {
+  if (!counts_host || !active_mask_host)
+    return moe::set_error(MOE_ERR_ARG, "laep_prune_mask: null pointer");
+  if (E <= 0 || k <= 0 || k > E || S < 0)
+    return moe::set_error(MOE_ERR_ARG, "laep_prune_mask: bad sizes E=%d k=%d S=%lld", E, k,
+                          (long long)S);
+  for (int e = 0; e < E; ++e)
+    if (counts_host[e] < 0) return moe::set_error(MOE_ERR_ARG, "laep_prune_mask: negative count");
+  // Ascending load order; equal loads keep index order (lower index first).
+  std::vector<int> order(E);
+  std::iota(order.begin(), order.end(), 0);
+  std::stable_sort(order.begin(), order.end(),
+                   [&](int a, int b) { return counts_host[a] < counts_host[b]; });
+  for (int e = 0; e < E; ++e) active_mask_host[e] = 1;
+  const int max_prune = E - k;  // routing needs k live experts
+  int pruned = 0;
+  if (prune_count >= 0) {
+    pruned = std::min(prune_count, max_prune);
+    for (int r = 0; r < pruned; ++r) active_mask_host[order[r]] = 0;
+  } else {
+    // Thresholds of Algorithm 1: cumulative < S*topK*beta, individual < S*topK*alpha/E.
+    const double beta_thr = double(S) * double(k) * beta;
+    const double alpha_thr = double(S) * double(k) * alpha / double(E);
+    int64_t running = 0;
+    for (int r = 0; r < E; ++r) {
+      const int e = order[r];
+      running += counts_host[e];
+      if (double(running) < beta_thr && double(counts_host[e]) < alpha_thr && pruned < max_prune) {
+        active_mask_host[e] = 0;
+        ++pruned;
+      }
+    }
+  }
+  if (n_pruned) *n_pruned = pruned;
+  return MOE_OK;
+}
+
+}  // extern "C"

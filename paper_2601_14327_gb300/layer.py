@@ -1,0 +1,109 @@
+"""One MoE expert layer step through the C ABI.
+
+PyTorch only allocates device memory and provides the stream; every step of
+the layer runs in the library's kernels (see _lib.py for the entry points).
+"""
+from __future__ import annotations
+
+import dataclasses
+from typing import Optional
+
+import torch
+
+from . import _lib as L
+
+
+@dataclasses.dataclass
+class LayerShape:
+    T: int
+    d: int
+    E: int
+    k: int
+    F: int
+
+    @property
+    def rows_cap(self) -> int:
+        return L.moe_perm_rows_max(self.T, self.k, self.E)
+
+
+class MoELayerBuffers:
+    """Device buffers of one layer step (activations, grouped layout, grads)."""
+
+    def __init__(self, shape: LayerShape, device="cuda", backward: bool = True):
+        s = shape
+        self.shape = s
+        R = s.rows_cap
+        dev = torch.device(device)
+        bf16, f32, i32 = torch.bfloat16, torch.float32, torch.int32
+        self.ws_bytes = max(L.moe_workspace_size(s.T, s.d, s.E, s.k, s.F), 256)
+        self.ws = torch.empty(self.ws_bytes, dtype=torch.uint8, device=dev)
+        self.logits = torch.empty(s.T, s.E, dtype=f32, device=dev)
+        self.topk_idx = torch.empty(s.T, s.k, dtype=i32, device=dev)
+        self.topk_gate = torch.empty(s.T, s.k, dtype=f32, device=dev)
+        self.counts = torch.empty(s.E, dtype=i32, device=dev)
+        self.group_offsets = torch.empty(s.E + 1, dtype=i32, device=dev)
+        self.group_counts = torch.empty(s.E, dtype=i32, device=dev)
+        self.row_of_assignment = torch.empty(s.T, s.k, dtype=i32, device=dev)
+        self.x_perm = torch.empty(R, s.d, dtype=bf16, device=dev)
+        self.ab = torch.empty(R, 2 * s.F, dtype=bf16, device=dev)
+        self.h = torch.empty(R, s.F, dtype=bf16, device=dev)
+        self.out_perm = torch.empty(R, s.d, dtype=bf16, device=dev)
+        self.y = torch.empty(s.T, s.d, dtype=bf16, device=dev)
+        if backward:
+            self.d_out_perm = torch.empty(R, s.d, dtype=bf16, device=dev)
+            self.d_gate = torch.empty(s.T, s.k, dtype=f32, device=dev)
+            self.d_ab = torch.empty(R, 2 * s.F, dtype=bf16, device=dev)
+            self.dx_perm = torch.empty(R, s.d, dtype=bf16, device=dev)
+            self.dw_gate_up = torch.empty(s.E, 2 * s.F, s.d, dtype=bf16, device=dev)
+            self.dw_down = torch.empty(s.E, s.d, s.F, dtype=bf16, device=dev)
+            self.d_logits = torch.empty(s.T, s.k, dtype=f32, device=dev)
+            self.dw_router = torch.empty(s.d, s.E, dtype=f32, device=dev)
+            self.dx = torch.empty(s.T, s.d, dtype=bf16, device=dev)
+
+
+def route(b: MoELayerBuffers, x, w_router, bias, active_mask=None, logits_in=None,
+          keep_logits: bool = False, stream=None):
+    s = b.shape
+    L.moe_route(x, w_router, bias, active_mask, s.T, s.d, s.E, s.k, logits_in,
+                b.logits if keep_logits else None, b.topk_idx, b.topk_gate, b.counts, stream)
+
+
+def forward(b: MoELayerBuffers, x, w_router, bias, w_gate_up, w_down, active_mask=None,
+            logits_in=None, keep_logits: bool = False, stream=None):
+    """route -> permute -> grouped SwiGLU FFN -> combine. Returns b.y."""
+    s = b.shape
+    R = s.rows_cap
+    route(b, x, w_router, bias, active_mask, logits_in, keep_logits, stream)
+    L.moe_permute(x, b.topk_idx, b.counts, s.T, s.d, s.E, s.k, R, b.group_offsets,
+                  b.group_counts, b.row_of_assignment, b.x_perm, b.ws, b.ws_bytes, stream)
+    L.moe_grouped_ffn_fwd(b.x_perm, b.group_offsets, s.E, s.d, s.F, R, w_gate_up, w_down, b.ab,
+                          b.h, b.out_perm, b.ws, b.ws_bytes, stream)
+    L.moe_unpermute_combine(b.out_perm, b.row_of_assignment, b.topk_gate, s.T, s.d, s.k, b.y,
+                            stream)
+    return b.y
+
+
+def backward(b: MoELayerBuffers, dy, w_router, w_gate_up, w_down, stream=None):
+    """combine bwd -> grouped FFN bwd -> router bwd -> permute bwd.
+    Returns (dx, dw_gate_up, dw_down, dw_router)."""
+    s = b.shape
+    R = s.rows_cap
+    L.moe_unpermute_combine_bwd(dy, b.out_perm, b.row_of_assignment, b.topk_gate,
+                                b.group_offsets, b.group_counts, s.T, s.d, s.E, s.k,
+                                b.d_out_perm, b.d_gate, stream)
+    L.moe_grouped_ffn_bwd(b.d_out_perm, b.x_perm, b.ab, b.h, b.group_offsets, s.E, s.d, s.F, R,
+                          w_gate_up, w_down, b.d_ab, b.dx_perm, b.dw_gate_up, b.dw_down, b.ws,
+                          b.ws_bytes, stream)
+    L.moe_route_bwd(b.x_perm, b.topk_idx, b.topk_gate, b.d_gate, b.row_of_assignment,
+                    b.group_offsets, b.group_counts, s.T, s.d, s.E, s.k, R, b.d_logits,
+                    b.dw_router, b.ws, b.ws_bytes, stream)
+    L.moe_permute_bwd(b.dx_perm, b.row_of_assignment, b.topk_idx, b.d_logits, w_router, s.T,
+                      s.d, s.E, s.k, b.dx, b.ws, b.ws_bytes, stream)
+    return b.dx, b.dw_gate_up, b.dw_down, b.dw_router
+
+
+def prune_from_counts(counts_host, S: int, k: int, *, prune_count: int = -1,
+                      alpha: float = 0.0, beta: float = 0.0):
+    """LAEP decision on a host histogram; returns (mask uint8 tensor on CPU, n_pruned)."""
+    mask, n = L.laep_prune_mask([int(c) for c in counts_host], S, k, alpha, beta, prune_count)
+    return torch.tensor(mask, dtype=torch.uint8), n

@@ -1,0 +1,92 @@
+"""C ABI checks that need no GPU: the library builds, loads and exports every
+declared entry point; the host-side LAEP decision matches the oracle; argument
+validation fails cleanly before any launch."""
+import json
+import os
+import subprocess
+
+import numpy as np
+import pytest
+
+from oracle import moe_oracle as O
+from paper_2601_14327_gb300 import _lib as L
+from paper_2601_14327_gb300 import build as B
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+
+
+@pytest.fixture(scope="module")
+def lib():
+    B.build()
+    return L.load()
+
+
+def test_library_exports_every_declared_symbol(lib):
+    declared = L.header_functions()
+    assert len(declared) >= 15
+    out = subprocess.run(["nm", "-D", "--defined-only", B.LIB], capture_output=True, text=True,
+                         check=True).stdout
+    exported = {line.split()[-1] for line in out.splitlines() if line.strip()}
+    missing = [f for f in declared if f not in exported]
+    assert not missing, missing
+    for f in declared:
+        assert hasattr(lib, f)
+
+
+def test_sizes(lib):
+    assert L.moe_version() == 100
+    assert L.moe_perm_rows_max(100, 8, 64) == 800 + 128 * 64
+    ws = L.moe_workspace_size(16384, 4096, 64, 8, 2048)
+    R = 16384 * 8 + 128 * 64
+    assert ws >= R * 4 + (R // 128) * 4096 * 4 + 64 * 4096 * 4
+
+
+def test_laep_prune_mask_golden(lib):
+    g = json.load(open(os.path.join(GOLDEN, "laep_prune_cases.json")))
+    for c in g["alpha_beta"]:
+        mask, n = L.laep_prune_mask(c["counts"], c["S"], c["k"], c["alpha"], c["beta"], -1)
+        assert mask == c["mask"] and n == c["n_pruned"], c["name"]
+    for c in g["lowest"]:
+        mask, n = L.laep_prune_mask(c["counts"], 1, c["k"], 0, 0, c["P"])
+        assert mask == c["mask"] and n == c["n_pruned"], c["name"]
+
+
+def test_laep_prune_mask_matches_oracle_random(lib):
+    rng = np.random.default_rng(7)
+    for _ in range(400):
+        E = int(rng.integers(1, 257))
+        k = int(rng.integers(1, min(E, 8) + 1))
+        S = int(rng.integers(0, 5000))
+        counts = rng.multinomial(S * k, rng.dirichlet(np.full(E, 0.2))) if S else np.zeros(E, int)
+        alpha, beta = float(rng.uniform(0, 2)), float(rng.uniform(0, 0.5))
+        m, n = L.laep_prune_mask(counts, S, k, alpha, beta, -1)
+        om, on = O.prune_mask_alpha_beta(counts, S, k, alpha, beta)
+        assert m == list(om) and n == on
+        P = int(rng.integers(0, E + 1))
+        m, n = L.laep_prune_mask(counts, S, k, 0, 0, P)
+        om, on = O.prune_mask_lowest(counts, P, k)
+        assert m == list(om) and n == on
+
+
+def test_argument_validation_without_launch(lib):
+    # E too large, k too large, d not a multiple of 128: rejected on the host
+    with pytest.raises(L.MoEError) as e:
+        L.moe_route(None, None, None, None, 10, 64, 300, 2, 1, None, 1, 1, None, stream=0)
+    assert e.value.status == -2
+    with pytest.raises(L.MoEError) as e:
+        L.moe_route(None, None, None, None, 10, 64, 16, 9, 1, None, 1, 1, None, stream=0)
+    assert e.value.status == -2
+    with pytest.raises(L.MoEError) as e:
+        L.moe_grouped_ffn_fwd(16, 16, 8, 100, 256, 4096, 16, 16, 16, 16, 16, 16, 0, stream=0)
+    assert e.value.status == -2
+    with pytest.raises(L.MoEError) as e:
+        L.moe_grouped_ffn_fwd(None, 16, 8, 256, 256, 4096, 16, 16, 16, 16, 16, 16, 0, stream=0)
+    assert e.value.status == -1
+    with pytest.raises(L.MoEError) as e:  # rows_cap below T*k + 128*E
+        L.moe_permute(16, 16, None, 100, 64, 8, 2, 100, 16, 16, 16, 16, 16, 1 << 20, stream=0)
+    assert e.value.status == -1
+    with pytest.raises(L.MoEError) as e:  # workspace too small
+        L.moe_permute(16, 16, None, 100, 64, 8, 2, 2000, 16, 16, 16, 16, 16, 8, stream=0)
+    assert e.value.status == -6
+    with pytest.raises(L.MoEError):
+        L.laep_prune_mask([1, 2, 3], 2, 4)  # k > E

@@ -1,0 +1,242 @@
+"""CUDA path vs the CPU oracle, element by element, through the C ABI.
+
+Integer/index results (routing, counts, grouped layout) must be bit-exact
+when both sides route from the same fp32 logits; floating results must meet
+max|gpu - oracle| / max|oracle| <= 2e-2 (bf16 data, fp32 accumulation).
+"""
+import numpy as np
+import pytest
+import torch
+
+from oracle import moe_oracle as O
+from paper_2601_14327_gb300 import _lib as L
+from paper_2601_14327_gb300 import layer
+
+from gpu_helpers import (assert_close, case_inputs, oracle_inputs, rel_err, run_gpu_layer, to_np,
+                         topk_margin)
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(autouse=True)
+def _clean_device_error():
+    L.moe_device_error(clear=True)
+    yield
+    assert L.moe_device_error(clear=True) == 0
+
+
+def _route_only(T, E, k, z, mask=None):
+    dev = "cuda"
+    zt = torch.from_numpy(np.ascontiguousarray(z, np.float32)).to(dev)
+    m = None if mask is None else torch.as_tensor(mask, dtype=torch.uint8).to(dev)
+    idx = torch.empty(T, k, dtype=torch.int32, device=dev)
+    g = torch.empty(T, k, dtype=torch.float32, device=dev)
+    cnt = torch.empty(E, dtype=torch.int32, device=dev)
+    lo = torch.empty(T, E, dtype=torch.float32, device=dev)
+    L.moe_route(None, None, None, m, T, 8, E, k, zt, lo, idx, g, cnt)
+    torch.cuda.synchronize()
+    return idx.cpu().numpy(), g.cpu().numpy(), cnt.cpu().numpy(), lo.cpu().numpy()
+
+
+@pytest.mark.parametrize("T,E,k,n_masked", [(1000, 64, 6, 10), (777, 16, 2, 0), (513, 128, 8, 7),
+                                            (300, 171, 8, 20), (257, 256, 8, 85), (100, 8, 8, 0)])
+def test_route_bit_exact_from_shared_logits(T, E, k, n_masked):
+    rng = np.random.default_rng(T + E)
+    z = rng.standard_normal((T, E)).astype(np.float32)
+    mask = np.ones(E, np.uint8)
+    mask[rng.permutation(E)[:n_masked]] = 0
+    idx, g, cnt, lo = _route_only(T, E, k, z, mask)
+    zm = O.apply_mask(z, mask)
+    oidx, og = O.route_topk(zm, k)
+    assert (idx == oidx).all()
+    np.testing.assert_allclose(g, og, rtol=0, atol=2e-6)
+    assert (cnt == O.expert_counts(oidx, E)).all()
+    assert (lo == zm).all()
+
+
+def test_route_ties_go_to_lower_index():
+    T, E, k = 400, 32, 5
+    rng = np.random.default_rng(3)
+    z = rng.integers(-2, 2, size=(T, E)).astype(np.float32)  # many exact ties
+    idx, g, cnt, _ = _route_only(T, E, k, z)
+    oidx, og = O.route_topk(z, k)
+    assert (idx == oidx).all()
+    np.testing.assert_allclose(g, og, rtol=0, atol=2e-6)
+
+
+@pytest.mark.parametrize("T,d,E", [(777, 512, 64), (300, 1024, 171), (129, 256, 256)])
+def test_route_logits_fp32(T, d, E):
+    inp = case_inputs(T, d, E, 2, 128, seed=5)
+    o = oracle_inputs(inp)
+    dev = "cuda"
+    b = layer.MoELayerBuffers(layer.LayerShape(T, d, E, 2, 128), dev, backward=False)
+    layer.route(b, inp["x"].to(dev), inp["w_router"].to(dev), inp["bias"].to(dev), keep_logits=True)
+    torch.cuda.synchronize()
+    z = b.logits.cpu().numpy().astype(np.float64)
+    ref = O.router_logits(o["x"], o["w_router"], o["bias"]).astype(np.float64)
+    scale = np.abs(o["x"]) @ np.abs(o["w_router"]) + np.abs(o["bias"])[None, :]
+    assert (np.abs(z - ref) <= 1e-5 * scale + 1e-30).all()
+    # routing from the GPU logits: tokens with a clear top-k margin match exactly
+    idx = b.topk_idx.cpu().numpy()
+    oidx, _ = O.route_topk(ref.astype(np.float32), 2)
+    clear = topk_margin(ref, 2) > 1e-4
+    assert (idx[clear] == oidx[clear]).all()
+
+
+def test_load_stats_bit_exact_and_accumulate():
+    T, k, E = 5000, 8, 200
+    rng = np.random.default_rng(1)
+    idx = rng.integers(0, E, size=(T, k)).astype(np.int32)
+    ti = torch.from_numpy(idx).cuda()
+    cnt = torch.empty(E, dtype=torch.int32, device="cuda")
+    L.moe_load_stats(ti, T, k, E, cnt, accumulate=False)
+    L.moe_load_stats(ti, T, k, E, cnt, accumulate=True)
+    torch.cuda.synchronize()
+    assert (cnt.cpu().numpy() == 2 * np.bincount(idx.reshape(-1), minlength=E)).all()
+
+
+def test_load_stats_flags_bad_expert():
+    idx = torch.tensor([[0, 1], [2, 9]], dtype=torch.int32, device="cuda")
+    cnt = torch.empty(4, dtype=torch.int32, device="cuda")
+    L.moe_load_stats(idx, 2, 2, 4, cnt)
+    assert L.moe_device_error(clear=True) == 1  # MOE_DEV_BAD_EXPERT
+    assert cnt.cpu().tolist() == [1, 1, 1, 0]
+
+
+def test_route_flags_too_few_live_experts():
+    z = np.zeros((4, 6), np.float32)
+    mask = np.array([1, 0, 0, 0, 0, 1], np.uint8)
+    _route_only(4, 6, 3, z, mask)
+    assert L.moe_device_error(clear=True) == 2  # MOE_DEV_TOO_FEW_LIVE
+
+
+def _permute(inp, idx, E, k, counts=None):
+    T, d = inp["x"].shape
+    R = L.moe_perm_rows_max(T, k, E)
+    dev = "cuda"
+    ws_bytes = L.moe_workspace_size(T, d, E, k, 128)
+    ws = torch.empty(max(ws_bytes, 256), dtype=torch.uint8, device=dev)
+    goff = torch.empty(E + 1, dtype=torch.int32, device=dev)
+    gcnt = torch.empty(E, dtype=torch.int32, device=dev)
+    row = torch.empty(T, k, dtype=torch.int32, device=dev)
+    xp = torch.full((R, d), float("nan"), dtype=torch.bfloat16, device=dev)
+    ct = None if counts is None else torch.as_tensor(counts, dtype=torch.int32).to(dev)
+    L.moe_permute(inp["x"].to(dev), torch.from_numpy(np.ascontiguousarray(idx, np.int32)).to(dev), ct,
+                  T, d, E, k, R, goff, gcnt, row, xp, ws, ws.numel())
+    torch.cuda.synchronize()
+    return goff.cpu().numpy(), gcnt.cpu().numpy(), row.cpu().numpy(), xp.cpu()
+
+
+@pytest.mark.parametrize("T,d,E,k,bias", [(3000, 256, 64, 6, "zipf"), (4097, 128, 16, 2, "none"),
+                                          (1000, 512, 128, 8, "loguniform")])
+def test_permute_bit_exact(T, d, E, k, bias):
+    inp = case_inputs(T, d, E, k, 128, bias=bias, seed=9)
+    o = oracle_inputs(inp)
+    oidx, _ = O.route_topk(O.router_logits(o["x"], o["w_router"], o["bias"]), k)
+    goff, gcnt, row, xp = _permute(inp, oidx, E, k, counts=O.expert_counts(oidx, E))
+    ooff, ocnt, orow = O.permutation(oidx, E, 128)
+    assert (goff == ooff).all() and (gcnt == ocnt).all() and (row == orow).all()
+    x = inp["x"]
+    assert torch.equal(xp[torch.from_numpy(orow.reshape(-1))], x.repeat_interleave(k, dim=0))
+    for e in range(E):
+        pad = xp[ooff[e] + ocnt[e]:ooff[e + 1]]
+        assert (pad.float() == 0).all()
+
+
+def test_permute_all_tokens_one_expert_and_empty():
+    T, d, E, k = 700, 128, 8, 1
+    inp = case_inputs(T, d, E, k, 128, seed=2)
+    idx = np.full((T, 1), 5, np.int32)
+    goff, gcnt, row, xp = _permute(inp, idx, E, k)
+    ooff, ocnt, orow = O.permutation(idx, E, 128)
+    assert (goff == ooff).all() and (gcnt == ocnt).all() and (row == orow).all()
+    # no tokens at all
+    inp0 = case_inputs(1, d, E, k, 128, seed=2)
+    inp0["x"] = inp0["x"][:0]
+    goff, gcnt, row, xp = _permute(inp0, np.zeros((0, 1), np.int32), E, k)
+    assert (goff == 0).all() and (gcnt == 0).all()
+
+
+def test_permute_flags_count_mismatch():
+    T, d, E, k = 300, 128, 8, 2
+    inp = case_inputs(T, d, E, k, 128, seed=4)
+    rng = np.random.default_rng(0)
+    idx = rng.integers(0, E, size=(T, k)).astype(np.int32)
+    bad = np.bincount(idx.reshape(-1), minlength=E)
+    bad[0] += 1
+    _permute(inp, idx, E, k, counts=bad)
+    assert L.moe_device_error(clear=True) == 3  # MOE_DEV_COUNT_MISMATCH
+
+
+LAYER_CASES = [
+    # T, d, E, k, F, bias, n_masked
+    (512, 256, 16, 2, 512, "none", 0),        # the tiny workload
+    (1500, 384, 12, 4, 640, "zipf", 3),       # ragged groups, BN=128 paths, empty groups
+    (700, 512, 8, 8, 256, "zipf", 0),         # k = number of experts
+    (2100, 256, 32, 2, 384, "loguniform", 0), # volatile load, several empty experts
+]
+
+
+@pytest.mark.parametrize("T,d,E,k,F,bias,n_masked", LAYER_CASES)
+def test_layer_fwd_bwd_against_oracle(T, d, E, k, F, bias, n_masked):
+    inp = case_inputs(T, d, E, k, F, bias=bias, seed=T)
+    o = oracle_inputs(inp)
+    mask = None
+    if n_masked:
+        mask = np.ones(E, np.uint8)
+        mask[np.random.default_rng(1).permutation(E)[:n_masked]] = 0
+    z = O.router_logits(o["x"], o["w_router"], o["bias"])  # shared fp32 logits
+    ref = O.moe_layer(o["x"], o["w_router"], o["bias"], mask, k, o["w_gate_up"], o["w_down"],
+                      dy=o["dy"], logits32=z)
+    b = run_gpu_layer(inp, E, k, mask=mask, logits_in=z)
+    # integer parts: bit-exact
+    assert (b.topk_idx.cpu().numpy() == ref["topk_idx"]).all()
+    assert (b.counts.cpu().numpy() == ref["counts"]).all()
+    assert (b.group_offsets.cpu().numpy() == ref["group_offsets"]).all()
+    assert (b.group_counts.cpu().numpy() == ref["group_counts"]).all()
+    row = b.row_of_assignment.cpu().numpy()
+    assert (row == ref["row_of_assignment"]).all()
+    # floating parts, per assignment through the grouped layout
+    flat = row.reshape(-1)
+    nrows = lambda a: a.reshape(T * k, -1)
+    np.testing.assert_allclose(b.topk_gate.cpu().numpy(), ref["gates"], rtol=0, atol=2e-6)
+    assert_close("a", to_np(b.ab)[flat][:, :F], nrows(ref["a"]))
+    assert_close("b", to_np(b.ab)[flat][:, F:], nrows(ref["b"]))
+    assert_close("h", to_np(b.h)[flat], nrows(ref["h"]))
+    assert_close("o", to_np(b.out_perm)[flat], nrows(ref["o"]))
+    assert_close("y", to_np(b.y), ref["y"])
+    assert_close("d_gate", b.d_gate.cpu().numpy(), ref["d_gate"])
+    assert_close("dA", to_np(b.d_ab)[flat][:, :F], nrows(ref["dA"]))
+    assert_close("dB", to_np(b.d_ab)[flat][:, F:], nrows(ref["dB"]))
+    assert_close("dX", to_np(b.dx_perm)[flat], nrows(ref["dX"]))
+    assert_close("dw_down", to_np(b.dw_down), ref["dw_down"])
+    assert_close("dw_gate_up", to_np(b.dw_gate_up), ref["dw_gate_up"])
+    assert_close("d_logits", b.d_logits.cpu().numpy(), ref["d_logits"])
+    assert_close("dw_router", b.dw_router.cpu().numpy(), ref["dw_router"])
+    assert_close("dx", to_np(b.dx), ref["dx"])
+    # experts without tokens get exactly zero weight gradients
+    empty = np.nonzero(ref["counts"] == 0)[0]
+    for e in empty:
+        assert (to_np(b.dw_down[e]) == 0).all() and (to_np(b.dw_gate_up[e]) == 0).all()
+        assert (b.dw_router[:, e].cpu().numpy() == 0).all()
+
+
+def test_tiny_workload_end_to_end_gpu_logits():
+    """The tiny workload with the router computed on the GPU (no shared logits)."""
+    T, d, E, k, F = 512, 256, 16, 2, 512
+    inp = case_inputs(T, d, E, k, F, bias="none", seed=1000)
+    o = oracle_inputs(inp)
+    ref = O.moe_layer(o["x"], o["w_router"], o["bias"], None, k, o["w_gate_up"], o["w_down"],
+                      dy=o["dy"])
+    b = run_gpu_layer(inp, E, k)
+    idx = b.topk_idx.cpu().numpy()
+    clear = topk_margin(ref["logits"], k) > 1e-4
+    assert clear.mean() > 0.99
+    assert (idx[clear] == ref["topk_idx"][clear]).all()
+    y = to_np(b.y)
+    assert rel_err(y[clear], ref["y"][clear]) <= 2e-2
+    assert rel_err(to_np(b.dx)[clear], ref["dx"][clear]) <= 2e-2
+    if clear.all():
+        assert_close("dw_gate_up", to_np(b.dw_gate_up), ref["dw_gate_up"])
+        assert_close("dw_down", to_np(b.dw_down), ref["dw_down"])
+        assert_close("dw_router", b.dw_router.cpu().numpy(), ref["dw_router"])

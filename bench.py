@@ -1,0 +1,424 @@
+#!/usr/bin/env python
+"""Benchmark of one MoE expert-layer training step (forward + backward) on GB300.
+
+A step is one pass of the whole hot path over one batch: route (fp32 logits,
+top-k over the experts LAEP kept, gates, histogram) -> permute -> grouped
+SwiGLU FFN forward -> combine -> combine backward -> grouped FFN backward
+(dgrad + wgrad) -> router backward -> permute backward. The LAEP pruning
+decision itself runs once before the timed steps, as in the paper (one prune
+once the loads are stable), on the histogram of a first routing pass.
+
+Default workload: T=16384 tokens, d_model=4096, 64 experts of which the 16
+least-loaded are pruned (48 live), top-8, d_ff=2048, Zipf(1.2) gate bias,
+bf16 data with an fp32 router, seeded synthetic inputs.
+
+Prints ONE JSON line (rank 0). `--impl reference` times the CPU oracle on a
+bounded token sample of the same workload instead.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+NCPU = os.cpu_count() or 1
+for _v in ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS"):
+    os.environ.setdefault(_v, str(NCPU))
+
+import numpy as np  # noqa: E402
+import torch  # noqa: E402
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+from paper_2601_14327_gb300 import _lib as L  # noqa: E402
+from paper_2601_14327_gb300 import layer, synth  # noqa: E402
+
+METRIC = "MoE layer fwd+bwd tokens/s; grouped-GEMM TFLOPS as % of GB300 bf16 peak"
+GEMMS = ["gemm_gate_up", "gemm_down", "gemm_dgrad_down", "gemm_dgrad_gate_up",
+         "gemm_wgrad_down", "gemm_wgrad_gate_up"]
+
+
+def measured_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as f:
+            p = json.load(f)
+        return {"hbm_gbs": p["hbm_gbs"], "bf16_tflops": p["bf16_tflops"],
+                "bf16_tflops_sustained": p.get("bf16_tflops_sustained", p["bf16_tflops"]),
+                "source": "measured"}
+    return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0,
+            "source": "fallback"}
+
+
+# --------------------------------------------------------------------- clocks
+
+class ClockSampler:
+    """nvidia-smi samples during the timed region (median SM clock under load)."""
+
+    Q = ("clocks.sm,clocks.max.sm,utilization.gpu,power.draw,clocks_event_reasons.hw_slowdown,"
+         "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+         "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+        self.lines = []
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.Q}",
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.thread = threading.Thread(target=self._read, daemon=True)
+            self.thread.start()
+        except OSError:
+            self.proc = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.thread.join(timeout=2)
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        sm, mx, reasons, loaded = [], None, set(), []
+        for ln in self.lines:
+            f = [x.strip() for x in ln.split(",")]
+            if len(f) < 8:
+                continue
+            try:
+                s, m, u = float(f[0]), float(f[1]), float(f[2])
+            except ValueError:
+                continue
+            sm.append(s)
+            mx = m
+            if u >= 50:
+                loaded.append(s)
+            for n, v in zip(names, f[4:8]):
+                if v.lower() in ("active", "1"):
+                    reasons.add(n)
+        use = loaded or sm
+        return {"sm_mhz": statistics.median(use) if use else None, "sm_max_mhz": mx,
+                "reasons": sorted(reasons), "samples": len(sm), "samples_under_load": len(loaded)}
+
+
+# ------------------------------------------------------------------- workload
+
+class Workload:
+    """Inputs, the one-time LAEP prune, and the buffers of one layer step."""
+
+    def __init__(self, cfg_id: int, device: str, compact_override=None, tokens=None,
+                 experts=None, no_prune=False):
+        c = synth.CONFIGS[cfg_id]
+        if tokens or experts or no_prune:  # a smaller case of the same kernels (profiling)
+            import dataclasses
+            c = dataclasses.replace(c, name=c.name + f"_small_T{tokens or c.T}_E{experts or c.E}",
+                                    T=tokens or c.T, E=experts or c.E,
+                                    prune_lowest=0 if no_prune else c.prune_lowest)
+        self.cfg = c
+        self.cfg_id = cfg_id
+        self.device = device
+        inp = synth.make_layer_inputs(c.T, c.d, c.E, c.k, c.F, bias=c.bias, zipf_s=c.zipf_s,
+                                      seed=synth.seed_for(cfg_id), device=device)
+        self.inp = inp
+        T, d, E, k, F = c.T, c.d, c.E, c.k, c.F
+        self.mask = None
+        self.n_pruned = 0
+        compact = c.compact if compact_override is None else compact_override
+        if c.prune_lowest:
+            # first routing pass over all experts -> histogram -> LAEP decision
+            b0 = layer.MoELayerBuffers(layer.LayerShape(T, d, E, k, F), device, backward=False)
+            layer.route(b0, inp["x"], inp["w_router"], inp["bias"])
+            counts = b0.counts.cpu().tolist()
+            del b0
+            mask, self.n_pruned = layer.prune_from_counts(counts, T, k,
+                                                          prune_count=c.prune_lowest)
+            if compact:
+                keep = torch.nonzero(mask).flatten().to(device)
+                inp["w_router"] = inp["w_router"].index_select(1, keep).contiguous()
+                inp["bias"] = inp["bias"].index_select(0, keep).contiguous()
+                inp["w_gate_up"] = inp["w_gate_up"].index_select(0, keep).contiguous()
+                inp["w_down"] = inp["w_down"].index_select(0, keep).contiguous()
+                E = int(keep.numel())
+            else:
+                self.mask = mask.to(device)
+        self.shape = layer.LayerShape(T, d, E, k, F)
+        self.E_live = E - (self.n_pruned if self.mask is not None else 0)
+        self.bufs = layer.MoELayerBuffers(self.shape, device, backward=True)
+
+    def step(self, x=None, dy=None):
+        i, b = self.inp, self.bufs
+        layer.forward(b, i["x"] if x is None else x, i["w_router"], i["bias"], i["w_gate_up"],
+                      i["w_down"], self.mask)
+        layer.backward(b, i["dy"] if dy is None else dy, i["w_router"], i["w_gate_up"],
+                       i["w_down"])
+
+    def gemm_flops(self):
+        """Algorithmic FLOPs per GEMM kernel launch (real assignments only)."""
+        s = self.shape
+        A = s.T * s.k
+        two = 2.0 * A * s.d * s.F
+        return {"gemm_gate_up": 2 * two, "gemm_down": two, "gemm_dgrad_down": two,
+                "gemm_dgrad_gate_up": 2 * two, "gemm_wgrad_down": two,
+                "gemm_wgrad_gate_up": 2 * two}
+
+
+# ------------------------------------------------------------------ the arms
+
+def dist_setup(n_gpus):
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    else:
+        torch.cuda.set_device(0)
+    return world, rank, local
+
+
+def barrier(world):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def max_over_ranks(x, world):
+    if world > 1:
+        import torch.distributed as dist
+        t = torch.tensor([x], dtype=torch.float64, device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        return float(t.item())
+    return x
+
+
+def oracle_sample(wl_inputs_host, mask_host, k, n_tok):
+    """Runs the CPU oracle over the first n_tok tokens; returns (seconds, threads)."""
+    from oracle import moe_oracle as O
+    h = wl_inputs_host
+    t0 = time.perf_counter()
+    O.moe_layer(h["x"][:n_tok], h["w_router"], h["bias"], mask_host, k, h["w_gate_up"],
+                h["w_down"], dy=h["dy"][:n_tok])
+    return time.perf_counter() - t0
+
+
+def host_inputs(inp, n_tok):
+    """float32 host copies of the inputs the oracle reads (bf16 values are exact)."""
+    out = {}
+    for n in ("x", "dy"):
+        out[n] = inp[n][:n_tok].float().cpu().numpy()
+    for n in ("w_router", "bias"):
+        out[n] = inp[n].float().cpu().numpy()
+    for n in ("w_gate_up", "w_down"):
+        out[n] = inp[n].float().cpu().numpy()
+    return out
+
+
+def run_ours(args):
+    world, rank, local = dist_setup(args.gpus)
+    L.load()
+    peaks = measured_peaks()
+    wl = Workload(args.config, "cuda", tokens=args.tokens, experts=args.experts,
+                  no_prune=args.no_prune)
+    s = wl.shape
+    torch.cuda.synchronize()
+    for _ in range(args.warmup):
+        wl.step()
+    torch.cuda.synchronize()
+    assert L.moe_device_error(clear=True) == 0, "device error during warm-up"
+
+    stream = torch.cuda.current_stream()
+    clocks = ClockSampler(local)
+    L.moe_timing_enable(True)
+    L.moe_timing_read(reset=True)
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    barrier(world)
+    torch.cuda.synchronize()
+    clocks.start()
+    time.sleep(0.3)  # let the sampler start
+    ev0.record(stream)
+    for _ in range(args.steps):
+        wl.step()
+    ev1.record(stream)
+    torch.cuda.synchronize()
+    barrier(world)
+    clk = clocks.stop()
+    L.moe_timing_enable(False)
+    per_kernel = L.moe_timing_read(reset=True)
+    ms_total = ev0.elapsed_time(ev1)
+    ms_total = max_over_ranks(ms_total, world)
+    ms_step = ms_total / args.steps
+    tokens_per_s = world * s.T * args.steps / (ms_total / 1e3)
+    launches = sum(n for n, _ in per_kernel.values())
+    assert L.moe_device_error(clear=True) == 0, "device error during the timed steps"
+
+    # dominant kernel and its roofline
+    gemm_ms = {n: per_kernel[n][1] / per_kernel[n][0] for n in GEMMS if n in per_kernel}
+    flops = wl.gemm_flops()
+    dom = max(gemm_ms, key=lambda n: per_kernel[n][1])
+    dom_tflops = flops[dom] / (gemm_ms[dom] / 1e3) / 1e12
+    all_gemm_ms = sum(per_kernel[n][1] for n in gemm_ms) / args.steps
+    all_gemm_tflops = sum(flops.values()) / (all_gemm_ms / 1e3) / 1e12
+    peak = peaks["bf16_tflops_sustained"]
+    kernel_table = {n: {"launches": c, "ms_per_step": round(ms / args.steps, 4),
+                        "share": round(ms / sum(v[1] for v in per_kernel.values()), 4)}
+                    for n, (c, ms) in per_kernel.items()}
+
+    # end to end through the public API: pinned host inputs in, results out
+    e2e = None
+    if not args.no_e2e:
+        x_h = wl.inp["x"].cpu().pin_memory()
+        dy_h = wl.inp["dy"].cpu().pin_memory()
+        y_h = torch.empty_like(x_h).pin_memory()
+        dx_h = torch.empty_like(x_h).pin_memory()
+        x_d = torch.empty_like(wl.inp["x"])
+        dy_d = torch.empty_like(wl.inp["dy"])
+
+        def e2e_step():
+            x_d.copy_(x_h, non_blocking=True)
+            dy_d.copy_(dy_h, non_blocking=True)
+            wl.step(x_d, dy_d)
+            y_h.copy_(wl.bufs.y, non_blocking=True)
+            dx_h.copy_(wl.bufs.dx, non_blocking=True)
+
+        for _ in range(2):
+            e2e_step()
+        barrier(world)
+        torch.cuda.synchronize()
+        ev0.record(stream)
+        for _ in range(args.steps):
+            e2e_step()
+        ev1.record(stream)
+        torch.cuda.synchronize()
+        barrier(world)
+        e_ms = max_over_ranks(ev0.elapsed_time(ev1), world)
+        nbytes = x_h.numel() * 2
+        e2e = {"value": round(world * s.T * args.steps / (e_ms / 1e3), 1), "unit": "tokens/s",
+               "h2d_bytes_per_step": 2 * nbytes, "d2h_bytes_per_step": 2 * nbytes}
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        n_tok = args.cpu_tokens
+        hin = host_inputs(wl.inp, n_tok)
+        mask_h = None if wl.mask is None else wl.mask.cpu().numpy()
+        secs = oracle_sample(hin, mask_h, s.k, n_tok)
+        cpu = {"value": round(n_tok / secs, 3), "unit": "tokens/s",
+               "cores": int(os.environ.get("OPENBLAS_NUM_THREADS", NCPU)), "kind": "oracle",
+               "sample": f"first {n_tok} of {s.T} tokens of the same layer step (all {s.E} experts, "
+                         f"same mask and weights), fp64 numpy oracle, {secs:.1f} s wall"}
+
+    c = wl.cfg
+    out = {
+        "metric": METRIC, "value": round(tokens_per_s, 1), "unit": "tokens/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_step, 4),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic (seeded; random-init expert weights)",
+        "config": {"workload": c.name, "T": s.T, "d_model": s.d, "experts": c.E,
+                   "experts_live": wl.E_live, "top_k": s.k, "d_ff": s.F, "gate_bias": c.bias,
+                   "pruned": wl.n_pruned, "l2": "working set far above L2 (x 134 MB, expert "
+                   "weights GBs); no flush", "parallelism": "replicas" if world > 1 else "1 GPU"},
+        "grouped_gemm": {"tflops": round(all_gemm_tflops, 1),
+                         "frac_of_peak": round(all_gemm_tflops / peak, 4),
+                         "peak_tflops": peak, "peak": f"bf16 sustained, {peaks['source']}",
+                         "ms_per_step": round(all_gemm_ms, 4)},
+        "roofline": {"kernel": dom, "bound": "tensor", "achieved": round(dom_tflops, 1),
+                     "peak": peak, "unit": "TFLOP/s", "frac": round(dom_tflops / peak, 4),
+                     "traffic": None, "peak_source": f"bf16 sustained ({peaks['source']})"},
+        "kernels": kernel_table,
+        "gpu_launches": launches,
+        "clocks": clk,
+        "e2e": e2e,
+        "cpu_baseline": cpu,
+    }
+    if rank == 0:
+        print(json.dumps(out), flush=True)
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+def run_reference(args):
+    """The CPU oracle on the host cores: each step a bounded token sample."""
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    c = synth.CONFIGS[args.config]
+    n_tok = args.ref_tokens
+    dev = "cuda" if torch.cuda.is_available() else "cpu"
+    inp = synth.make_config_inputs(args.config, device=dev)
+    mask_h = None
+    E = c.E
+    if c.prune_lowest:
+        from oracle import moe_oracle as O
+        xr = inp["x"].float().cpu().numpy()
+        z = O.router_logits(xr, inp["w_router"].cpu().numpy(), inp["bias"].cpu().numpy())
+        idx, _ = O.route_topk(z, c.k)
+        mask_h, _ = O.prune_mask_lowest(O.expert_counts(idx, E), c.prune_lowest, c.k)
+        del xr, z
+    hin = host_inputs(inp, n_tok)
+    del inp
+    for _ in range(args.warmup):
+        oracle_sample(hin, mask_h, c.k, n_tok)
+    secs = 0.0
+    for _ in range(args.steps):
+        secs += oracle_sample(hin, mask_h, c.k, n_tok)
+    v = n_tok * args.steps / secs
+    cores = int(os.environ.get("OPENBLAS_NUM_THREADS", NCPU))
+    sample = (f"first {n_tok} of {c.T} tokens per step, full layer fwd+bwd over all {E} experts "
+              f"(16 least-loaded masked when the workload prunes), fp64 numpy oracle")
+    print(json.dumps({
+        "impl": "reference", "metric": METRIC, "value": round(v, 3), "unit": "tokens/s",
+        "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": round(secs / args.steps * 1e3, 1), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": c.name, "T": c.T, "d_model": c.d, "experts": c.E, "top_k": c.k,
+                   "d_ff": c.F},
+        "cpu_baseline": {"value": round(v, 3), "unit": "tokens/s", "cores": cores,
+                         "kind": "oracle", "sample": sample},
+        "e2e": {"value": round(v, 3), "unit": "tokens/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0}}), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=30)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--config", type=int, default=2, choices=sorted(synth.CONFIGS))
+    ap.add_argument("--cpu-tokens", type=int, default=1024)
+    ap.add_argument("--ref-tokens", type=int, default=64)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    # smaller cases of the same kernels, for profiler captures
+    ap.add_argument("--tokens", type=int, default=None)
+    ap.add_argument("--experts", type=int, default=None)
+    ap.add_argument("--no-prune", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3 and args.impl == "ours":
+        args.warmup = 3
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ours(args)
+
+
+if __name__ == "__main__":
+    main()

@@ -79,6 +79,15 @@ const char *moe_last_error_string(void);
  * or MOE_ERR_CUDA. */
 int moe_device_error(int *code, int clear);
 
+/* Kernel timing (instrumentation; not part of the paper's method). While
+ * enabled, every kernel the library launches is bracketed by two CUDA events
+ * recorded on its stream. moe_timing_read() waits for those events and
+ * writes one line per kernel name, "name launches total_ms\n", in first-seen
+ * order into buf (NUL-terminated); reset != 0 then forgets the records.
+ * Host calls; they return MOE_OK, MOE_ERR_ARG or MOE_ERR_CUDA. */
+int moe_timing_enable(int enable);
+int moe_timing_read(char *buf, size_t buf_len, int reset);
+
 /* Rows to allocate for every grouped-layout buffer: T*k + 128*E. */
 int64_t moe_perm_rows_max(int T, int k, int E);
 

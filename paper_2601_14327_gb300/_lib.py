@@ -39,6 +39,8 @@ _SIGS = {
     "moe_version": (I, []),
     "moe_last_error_string": (ctypes.c_char_p, []),
     "moe_device_error": (I, [P, I]),
+    "moe_timing_enable": (I, [I]),
+    "moe_timing_read": (I, [ctypes.c_char_p, SZ, I]),
     "moe_perm_rows_max": (I64, [I, I, I]),
     "moe_workspace_size": (SZ, [I, I, I, I, I]),
     "moe_route": (I, [P, P, P, P, I, I, I, I, P, P, P, P, P, P]),
@@ -121,6 +123,21 @@ def moe_device_error(clear=True):
     code = ctypes.c_int(0)
     _check("moe_device_error", load().moe_device_error(ctypes.byref(code), int(clear)))
     return code.value
+
+
+def moe_timing_enable(enable=True):
+    _check("moe_timing_enable", load().moe_timing_enable(int(enable)))
+
+
+def moe_timing_read(reset=True):
+    """{kernel name: (launches, total_ms)} recorded since the last reset."""
+    buf = ctypes.create_string_buffer(1 << 16)
+    _check("moe_timing_read", load().moe_timing_read(buf, len(buf), int(reset)))
+    out = {}
+    for line in buf.value.decode().splitlines():
+        name, n, ms = line.split()
+        out[name] = (int(n), float(ms))
+    return out
 
 
 def moe_route(x, w_router, bias, active_mask, T, d, E, k, logits_in, logits_out, topk_idx,

@@ -3,7 +3,10 @@
 #include <stdio.h>
 
 #include <algorithm>
+#include <map>
+#include <mutex>
 #include <numeric>
+#include <string>
 #include <vector>
 
 #include "common.cuh"
@@ -38,6 +41,59 @@ int num_sms() {
     cached[dev] = n;
   }
   return cached[dev];
+}
+
+// ---- kernel timing registry ----
+namespace {
+struct TimingRec {
+  const char *name;
+  cudaEvent_t a, b;
+};
+struct Timing {
+  std::mutex mu;
+  bool enabled = false;
+  std::vector<cudaEvent_t> pool;
+  std::vector<TimingRec> recs;
+};
+Timing &timing() {
+  static Timing t;
+  return t;
+}
+cudaEvent_t take_event(Timing &t) {
+  if (!t.pool.empty()) {
+    cudaEvent_t e = t.pool.back();
+    t.pool.pop_back();
+    return e;
+  }
+  cudaEvent_t e = nullptr;
+  if (cudaEventCreate(&e) != cudaSuccess) return nullptr;
+  return e;
+}
+}  // namespace
+
+cudaEvent_t timing_begin(cudaStream_t s) {
+  Timing &t = timing();
+  if (!t.enabled) return nullptr;
+  std::lock_guard<std::mutex> g(t.mu);
+  cudaEvent_t e = take_event(t);
+  if (e && cudaEventRecord(e, s) != cudaSuccess) {
+    t.pool.push_back(e);
+    return nullptr;
+  }
+  return e;
+}
+
+void timing_end(const char *name, cudaEvent_t begin, cudaStream_t s) {
+  if (!begin) return;
+  Timing &t = timing();
+  std::lock_guard<std::mutex> g(t.mu);
+  cudaEvent_t e = take_event(t);
+  if (!e || cudaEventRecord(e, s) != cudaSuccess) {
+    t.pool.push_back(begin);
+    if (e) t.pool.push_back(e);
+    return;
+  }
+  t.recs.push_back({name, begin, e});
 }
 
 static size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
@@ -88,6 +144,52 @@ int moe_device_error(int *code, int clear) {
   if ((st = moe::permute_dev_error(clear, &c1))) return st;
   if ((st = moe::gemm_dev_error(clear, &c2))) return st;
   *code = c0 ? c0 : (c1 ? c1 : c2);
+  return MOE_OK;
+}
+
+int moe_timing_enable(int enable) {
+  moe::Timing &t = moe::timing();
+  std::lock_guard<std::mutex> g(t.mu);
+  t.enabled = enable != 0;
+  return MOE_OK;
+}
+
+int moe_timing_read(char *buf, size_t buf_len, int reset) {
+  if (!buf || buf_len == 0) return moe::set_error(MOE_ERR_ARG, "moe_timing_read: null buffer");
+  moe::Timing &t = moe::timing();
+  std::lock_guard<std::mutex> g(t.mu);
+  struct Acc {
+    long long n = 0;
+    double ms = 0;
+  };
+  std::map<std::string, Acc> acc;
+  std::vector<std::string> order;
+  for (const auto &r : t.recs) {
+    if (cudaEventSynchronize(r.b) != cudaSuccess)
+      return moe::set_error(MOE_ERR_CUDA, "moe_timing_read: event synchronize");
+    float ms = 0.f;
+    if (cudaEventElapsedTime(&ms, r.a, r.b) != cudaSuccess)
+      return moe::set_error(MOE_ERR_CUDA, "moe_timing_read: elapsed time");
+    if (!acc.count(r.name)) order.push_back(r.name);
+    acc[r.name].n += 1;
+    acc[r.name].ms += ms;
+  }
+  size_t off = 0;
+  buf[0] = 0;
+  for (const auto &name : order) {
+    const int w = snprintf(buf + off, buf_len - off, "%s %lld %.6f\n", name.c_str(), acc[name].n,
+                           acc[name].ms);
+    if (w < 0 || size_t(w) >= buf_len - off)
+      return moe::set_error(MOE_ERR_ARG, "moe_timing_read: buffer too small");
+    off += size_t(w);
+  }
+  if (reset) {
+    for (const auto &r : t.recs) {
+      t.pool.push_back(r.a);
+      t.pool.push_back(r.b);
+    }
+    t.recs.clear();
+  }
   return MOE_OK;
 }
 

@@ -36,12 +36,27 @@ WsLayout ws_layout(int T, int d, int E, int k, int F);
 constexpr int kPermChunk = 4096;  // assignments per block in the permutation
 constexpr int kGroupPad = 128;    // rows per group are padded to this
 
+// Kernel timing registry (moe_timing_enable / moe_timing_read). When enabled,
+// every kernel launch of the library is bracketed by CUDA events recorded on
+// the launching stream; otherwise these calls cost a flag test.
+cudaEvent_t timing_begin(cudaStream_t s);
+void timing_end(const char *name, cudaEvent_t begin, cudaStream_t s);
+
 // Device error words of each translation unit.
 int route_dev_error(int clear, int *code);
 int permute_dev_error(int clear, int *code);
 int gemm_dev_error(int clear, int *code);
 
 }  // namespace moe
+
+// Launches a kernel (the variadic part is the launch statement) under the
+// timing registry, then checks the launch.
+#define MOE_LAUNCH(name, stream, ...)                        \
+  do {                                                       \
+    cudaEvent_t moe_ev_ = moe::timing_begin(stream);         \
+    __VA_ARGS__;                                             \
+    moe::timing_end(name, moe_ev_, stream);                  \
+  } while (0)
 
 // -------------------------------------------------------------- device side
 #define MOE_DEV_ERR_DECL static __device__ int g_dev_err;

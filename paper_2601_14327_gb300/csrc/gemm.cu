@@ -38,6 +38,10 @@ enum Mode : int {
   kWgradGateUp = 5
 };
 
+const char *const kGemmName[] = {"gemm_gate_up",       "gemm_down",
+                                 "gemm_dgrad_down",    "gemm_dgrad_gate_up",
+                                 "gemm_wgrad_down",    "gemm_wgrad_gate_up"};
+
 constexpr int BM = 128;   // tile rows (TMEM lanes)
 constexpr int BK = 64;    // k-block: 64 bf16 = one 128-byte swizzle row
 constexpr int UMMA_K = 16;
@@ -461,7 +465,7 @@ int launch(const CUtensorMap &a, const CUtensorMap &b, const GemmParams &p, cuda
     if (e != cudaSuccess) return moe::cuda_status(e, what);
     attr = true;
   }
-  grouped_gemm_kernel<MODE, BN><<<moe::num_sms(), kThreads, Sh::SMEM, s>>>(a, b, p);
+  MOE_LAUNCH(kGemmName[MODE], s, grouped_gemm_kernel<MODE, BN><<<moe::num_sms(), kThreads, Sh::SMEM, s>>>(a, b, p));
   return moe::launch_status(what);
 }
 

@@ -356,19 +356,19 @@ int moe_permute(const uint16_t *x, const int32_t *topk_idx, const int32_t *count
   const int64_t A = int64_t(T) * k;
   const int nblk = int(std::max<int64_t>(1, (A + kChunk - 1) / kChunk));
   int32_t *hist = reinterpret_cast<int32_t *>(static_cast<char *>(ws) + L.perm_hist);
-  perm_hist_kernel<<<nblk, kThreads, 0, s>>>(topk_idx, A, E, nblk, hist);
+  MOE_LAUNCH("perm_hist", s, perm_hist_kernel<<<nblk, kThreads, 0, s>>>(topk_idx, A, E, nblk, hist));
   if (int st = moe::launch_status("moe_permute: hist")) return st;
-  perm_scan_kernel<<<1, 1024, 0, s>>>(hist, E, nblk, counts, rows_cap, group_offsets, group_counts);
+  MOE_LAUNCH("perm_scan", s, perm_scan_kernel<<<1, 1024, 0, s>>>(hist, E, nblk, counts, rows_cap, group_offsets, group_counts));
   if (int st = moe::launch_status("moe_permute: scan")) return st;
   if (A > 0) {
-    perm_rank_kernel<<<nblk, kThreads, 0, s>>>(topk_idx, A, E, nblk, hist, group_offsets, rows_cap,
-                                               row_of_assignment);
+    MOE_LAUNCH("perm_rank", s, perm_rank_kernel<<<nblk, kThreads, 0, s>>>(topk_idx, A, E, nblk, hist, group_offsets, rows_cap,
+                                               row_of_assignment));
     if (int st = moe::launch_status("moe_permute: rank")) return st;
-    perm_gather_kernel<<<warp_grid(T), kThreads, 0, s>>>(x, row_of_assignment, T, d, k, rows_cap,
-                                                         x_perm);
+    MOE_LAUNCH("perm_gather", s, perm_gather_kernel<<<warp_grid(T), kThreads, 0, s>>>(x, row_of_assignment, T, d, k, rows_cap,
+                                                         x_perm));
     if (int st = moe::launch_status("moe_permute: gather")) return st;
   }
-  pad_zero_kernel<<<E, kThreads, 0, s>>>(group_offsets, group_counts, E, d, rows_cap, x_perm);
+  MOE_LAUNCH("pad_zero", s, pad_zero_kernel<<<E, kThreads, 0, s>>>(group_offsets, group_counts, E, d, rows_cap, x_perm));
   return moe::launch_status("moe_permute: pad");
 }
 
@@ -382,7 +382,7 @@ int moe_unpermute_combine(const uint16_t *out_perm, const int32_t *row_of_assign
     return moe::set_error(MOE_ERR_ARG, "moe_unpermute_combine: null pointer");
   if (!moe::aligned16(out_perm) || !moe::aligned16(y))
     return moe::set_error(MOE_ERR_ARG, "moe_unpermute_combine: alignment");
-  combine_kernel<<<warp_grid(T), kThreads, 0, s>>>(out_perm, row_of_assignment, topk_gate, T, d, k, y);
+  MOE_LAUNCH("combine", s, combine_kernel<<<warp_grid(T), kThreads, 0, s>>>(out_perm, row_of_assignment, topk_gate, T, d, k, y));
   return moe::launch_status("moe_unpermute_combine: launch");
 }
 
@@ -401,11 +401,11 @@ int moe_unpermute_combine_bwd(const uint16_t *dy, const uint16_t *out_perm,
     return moe::set_error(MOE_ERR_ARG, "moe_unpermute_combine_bwd: alignment");
   const int64_t rows_cap = moe_perm_rows_max(T, k, E);
   if (T > 0) {
-    combine_bwd_kernel<<<warp_grid(T), kThreads, 0, s>>>(dy, out_perm, row_of_assignment, topk_gate,
-                                                         T, d, k, rows_cap, d_out_perm, d_gate);
+    MOE_LAUNCH("combine_bwd", s, combine_bwd_kernel<<<warp_grid(T), kThreads, 0, s>>>(dy, out_perm, row_of_assignment, topk_gate,
+                                                         T, d, k, rows_cap, d_out_perm, d_gate));
     if (int st = moe::launch_status("moe_unpermute_combine_bwd: launch")) return st;
   }
-  pad_zero_kernel<<<E, kThreads, 0, s>>>(group_offsets, group_counts, E, d, rows_cap, d_out_perm);
+  MOE_LAUNCH("pad_zero", s, pad_zero_kernel<<<E, kThreads, 0, s>>>(group_offsets, group_counts, E, d, rows_cap, d_out_perm));
   return moe::launch_status("moe_unpermute_combine_bwd: pad");
 }
 
@@ -429,12 +429,13 @@ int moe_permute_bwd(const uint16_t *dx_perm, const int32_t *row_of_assignment,
     if (!moe::aligned16(ws)) return moe::set_error(MOE_ERR_ARG, "moe_permute_bwd: ws alignment");
     w_t = reinterpret_cast<float *>(static_cast<char *>(ws) + L.w_router_t);
     dim3 grid((d + 31) / 32, (E + 31) / 32), block(32, 8);
-    transpose_router_kernel<<<grid, block, 0, s>>>(w_router, d, E, w_t);
+    MOE_LAUNCH("transpose_router", s, transpose_router_kernel<<<grid, block, 0, s>>>(w_router, d, E, w_t));
     if (int st = moe::launch_status("moe_permute_bwd: transpose")) return st;
   }
-  permute_bwd_kernel<<<warp_grid(T), kThreads, 0, s>>>(dx_perm, row_of_assignment, topk_idx,
-                                                       d_logits, w_t, T, d, E, k, dx);
+  MOE_LAUNCH("permute_bwd", s, permute_bwd_kernel<<<warp_grid(T), kThreads, 0, s>>>(dx_perm, row_of_assignment, topk_idx,
+                                                       d_logits, w_t, T, d, E, k, dx));
   return moe::launch_status("moe_permute_bwd: launch");
 }
 
 }  // extern "C"
+

@@ -286,8 +286,8 @@ int launch_route(const uint16_t *x, const float *w, const float *b, const uint8_
     attr_set = true;
   }
   const int grid = (T + S::BM - 1) / S::BM;
-  route_kernel<NE><<<grid, kRouteThreads, S::kSmem, s>>>(x, w, b, mask, T, d, E, k, lin, lout,
-                                                        idx, gate, counts);
+  MOE_LAUNCH("route", s, route_kernel<NE><<<grid, kRouteThreads, S::kSmem, s>>>(x, w, b, mask, T, d, E, k, lin, lout,
+                                                        idx, gate, counts));
   return moe::launch_status("moe_route: launch");
 }
 
@@ -311,7 +311,7 @@ int moe_route(const uint16_t *x, const float *w_router, const float *bias,
   if (!logits_in && (!x || !w_router)) return moe::set_error(MOE_ERR_ARG, "moe_route: null x/w_router");
   if (x && !moe::aligned16(x)) return moe::set_error(MOE_ERR_ARG, "moe_route: x not 16-byte aligned");
   if (counts) {
-    zero_i32_kernel<<<1, 256, 0, s>>>(counts, E);
+    MOE_LAUNCH("zero_counts", s, zero_i32_kernel<<<1, 256, 0, s>>>(counts, E));
     if (int st = moe::launch_status("moe_route: zero counts")) return st;
   }
   if (T == 0) return MOE_OK;
@@ -327,13 +327,13 @@ int moe_load_stats(const int32_t *topk_idx, int T, int k, int E, int32_t *counts
   if (E < 1 || E > 256 || k < 1 || T < 0) return moe::set_error(MOE_ERR_ARG, "moe_load_stats: sizes");
   if (!counts || (T > 0 && !topk_idx)) return moe::set_error(MOE_ERR_ARG, "moe_load_stats: null");
   if (!accumulate) {
-    zero_i32_kernel<<<1, 256, 0, s>>>(counts, E);
+    MOE_LAUNCH("zero_counts", s, zero_i32_kernel<<<1, 256, 0, s>>>(counts, E));
     if (int st = moe::launch_status("moe_load_stats: zero")) return st;
   }
   const int64_t A = int64_t(T) * k;
   if (A == 0) return MOE_OK;
   const int grid = int(std::min<int64_t>((A + 255) / 256, int64_t(moe::num_sms()) * 4));
-  load_stats_kernel<<<grid, 256, 0, s>>>(topk_idx, A, E, counts);
+  MOE_LAUNCH("load_stats", s, load_stats_kernel<<<grid, 256, 0, s>>>(topk_idx, A, E, counts));
   return moe::launch_status("moe_load_stats: launch");
 }
 
@@ -358,16 +358,16 @@ int moe_route_bwd(const uint16_t *x_perm, const int32_t *topk_idx, const float *
   float *dz_perm = reinterpret_cast<float *>(static_cast<char *>(ws) + L.dz_perm);
   float *partial = reinterpret_cast<float *>(static_cast<char *>(ws) + L.rb_partial);
   if (T > 0) {
-    route_bwd_dz_kernel<<<(T + 255) / 256, 256, 0, s>>>(topk_gate, d_gate, row_of_assignment, T, k,
-                                                        rows_cap, d_logits, dz_perm);
+    MOE_LAUNCH("route_bwd_dz", s, route_bwd_dz_kernel<<<(T + 255) / 256, 256, 0, s>>>(topk_gate, d_gate, row_of_assignment, T, k,
+                                                        rows_cap, d_logits, dz_perm));
     if (int st = moe::launch_status("moe_route_bwd: dz")) return st;
     const int tiles = int(rows_cap / moe::kGroupPad);
-    route_bwd_partial_kernel<<<tiles, 256, 0, s>>>(x_perm, dz_perm, group_offsets, group_counts, E,
-                                                   d, partial);
+    MOE_LAUNCH("route_bwd_partial", s, route_bwd_partial_kernel<<<tiles, 256, 0, s>>>(x_perm, dz_perm, group_offsets, group_counts, E,
+                                                   d, partial));
     if (int st = moe::launch_status("moe_route_bwd: partial")) return st;
   }
   dim3 grid((d + 255) / 256, E);
-  route_bwd_reduce_kernel<<<grid, 256, 0, s>>>(partial, group_offsets, E, d, dw_router);
+  MOE_LAUNCH("route_bwd_reduce", s, route_bwd_reduce_kernel<<<grid, 256, 0, s>>>(partial, group_offsets, E, d, dw_router));
   return moe::launch_status("moe_route_bwd: reduce");
 }
 

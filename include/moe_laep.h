@@ -160,6 +160,32 @@ int moe_permute(const uint16_t *x, const int32_t *topk_idx, const int32_t *count
                 void *ws, size_t ws_bytes, moe_stream_t stream);
 
 /*
+ * moe_permute_noalloc - moe_permute for callers that cannot allocate device
+ * memory. The paper has no counterpart; this is a deployment variant.
+ * Some callers may not call cudaMalloc or hand out a workspace, e.g. code
+ * running inside an engine whose device memory is planned before it runs
+ * (an inference plugin's enqueue) or while a stream is being captured into a
+ * CUDA graph. This entry point computes exactly what moe_permute computes
+ * (same arguments minus ws/ws_bytes, same results) but keeps its per-block
+ * histograms in a fixed 256 KiB array compiled into the library (65536
+ * int32 entries) instead of a workspace; it allocates nothing.
+ * Limit: E * ceil(T*k / 4096) <= 65536 (e.g. 256 experts with at most
+ * 1,048,576 assignments); larger problems return MOE_ERR_UNSUPPORTED before
+ * anything is launched.
+ * The first call on a device looks up the array's device address (once per
+ * device, with that device current); make that first call before any stream
+ * capture. Every GPU that loads the library holds the array until the
+ * process exits. All calls share the one array and it keeps the last call's
+ * contents (nothing in it needs to start at zero): calls whose kernels may
+ * overlap on the GPU (other streams, other host threads) race on it and must
+ * be serialized by the caller.
+ */
+int moe_permute_noalloc(const uint16_t *x, const int32_t *topk_idx, const int32_t *counts, int T,
+                        int d, int E, int k, int64_t rows_cap, int32_t *group_offsets,
+                        int32_t *group_counts, int32_t *row_of_assignment, uint16_t *x_perm,
+                        moe_stream_t stream);
+
+/*
  * moe_grouped_ffn_fwd - the experts' SwiGLU FFN over the grouped layout.
  * Table A1 fixes three matrices per expert (gate, up, down); for each group
  * e with rows X_e:

@@ -47,6 +47,7 @@ _SIGS = {
     "moe_load_stats": (I, [P, I, I, I, P, I, P]),
     "laep_prune_mask": (I, [P, I, I64, I, D, D, I, P, P]),
     "moe_permute": (I, [P, P, P, I, I, I, I, I64, P, P, P, P, P, SZ, P]),
+    "moe_permute_noalloc": (I, [P, P, P, I, I, I, I, I64, P, P, P, P, P]),
     "moe_grouped_ffn_fwd": (I, [P, P, I, I, I, I64, P, P, P, P, P, P, SZ, P]),
     "moe_unpermute_combine": (I, [P, P, P, I, I, I, P, P]),
     "moe_unpermute_combine_bwd": (I, [P, P, P, P, P, P, I, I, I, I, P, P, P]),
@@ -170,6 +171,13 @@ def moe_permute(x, topk_idx, counts, T, d, E, k, rows_cap, group_offsets, group_
         _ptr(x), _ptr(topk_idx), _ptr(counts), T, d, E, k, rows_cap, _ptr(group_offsets),
         _ptr(group_counts), _ptr(row_of_assignment), _ptr(x_perm), _ptr(ws), ws_bytes,
         _stream(stream)))
+
+
+def moe_permute_noalloc(x, topk_idx, counts, T, d, E, k, rows_cap, group_offsets, group_counts,
+                        row_of_assignment, x_perm, stream=None):
+    _check("moe_permute_noalloc", load().moe_permute_noalloc(
+        _ptr(x), _ptr(topk_idx), _ptr(counts), T, d, E, k, rows_cap, _ptr(group_offsets),
+        _ptr(group_counts), _ptr(row_of_assignment), _ptr(x_perm), _stream(stream)))
 
 
 def moe_grouped_ffn_fwd(x_perm, group_offsets, E, d, F, rows_cap, w_gate_up, w_down, ab_saved,

@@ -4,6 +4,8 @@
 // (order inside a group: token, then slot), so the grouped layout is
 // deterministic and bit-exact. Groups start at multiples of 128 rows so that
 // every 128-row GEMM tile belongs to one expert; padding rows are zero.
+#include <mutex>
+
 #include "common.cuh"
 
 MOE_DEV_ERR_DECL
@@ -439,3 +441,88 @@ int moe_permute_bwd(const uint16_t *dx_perm, const int32_t *row_of_assignment,
 
 }  // extern "C"
 
+// ---------------------------------------------------------------------------
+// moe_permute_noalloc: moe_permute for callers that cannot allocate device
+// memory (no cudaMalloc and no caller workspace), e.g. code running inside an
+// engine whose device memory is planned before execution (an inference
+// plugin's enqueue, a stream being captured into a CUDA graph). The
+// per-block histograms live in a fixed array compiled into the library
+// instead of the caller's workspace.
+//
+// The array holds kNoAllocScratchInts int32 entries (256 KiB). A call needs
+// E * ceil(T*k / 4096) of them, so 256 experts fit with up to 1,048,576
+// assignments (T*k). Every GPU that loads the library keeps the array until
+// the process exits. All calls share it: calls whose kernels overlap on the
+// GPU (different streams, or different host threads) race on it and must be
+// serialized by the caller. Nothing in it has to start at zero: every entry a
+// call reads was written earlier in the same call.
+constexpr int kNoAllocScratchInts = 65536;
+static __device__ __align__(256) int32_t g_perm_noalloc_scratch[kNoAllocScratchInts];
+
+namespace {
+// Device address of the array on the current device, looked up once per
+// device (host code cannot use the array's name as a device pointer).
+int noalloc_scratch(int32_t **out) {
+  static std::mutex mu;
+  static int32_t *addr[128] = {nullptr};
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return moe::cuda_status(e, "moe_permute_noalloc: cudaGetDevice");
+  if (dev < 0 || dev >= 128) return moe::set_error(MOE_ERR_UNSUPPORTED, "moe_permute_noalloc: device %d", dev);
+  std::lock_guard<std::mutex> g(mu);
+  if (addr[dev] == nullptr) {
+    void *p = nullptr;
+    e = cudaGetSymbolAddress(&p, g_perm_noalloc_scratch);
+    if (e != cudaSuccess) return moe::cuda_status(e, "moe_permute_noalloc: cudaGetSymbolAddress");
+    addr[dev] = static_cast<int32_t *>(p);
+  }
+  *out = addr[dev];
+  return MOE_OK;
+}
+}  // namespace
+
+extern "C" int moe_permute_noalloc(const uint16_t *x, const int32_t *topk_idx,
+                                   const int32_t *counts, int T, int d, int E, int k,
+                                   int64_t rows_cap, int32_t *group_offsets,
+                                   int32_t *group_counts, int32_t *row_of_assignment,
+                                   uint16_t *x_perm, moe_stream_t stream) {
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if (E < 1 || E > 256 || k < 1 || k > 8 || T < 0 || d <= 0 || d % 8)
+    return moe::set_error(MOE_ERR_ARG, "moe_permute_noalloc: sizes T=%d d=%d E=%d k=%d", T, d, E, k);
+  const int64_t A = int64_t(T) * k;
+  const int64_t nblk64 = std::max<int64_t>(1, (A + kChunk - 1) / kChunk);
+  if (int64_t(E) * nblk64 > kNoAllocScratchInts)
+    return moe::set_error(MOE_ERR_UNSUPPORTED,
+                          "moe_permute_noalloc: E * ceil(T*k/%d) = %lld exceeds the built-in "
+                          "scratch of %d entries (use moe_permute with a workspace)",
+                          kChunk, (long long)(int64_t(E) * nblk64), kNoAllocScratchInts);
+  if (!group_offsets || !group_counts || (T > 0 && (!x || !topk_idx || !row_of_assignment || !x_perm)))
+    return moe::set_error(MOE_ERR_ARG, "moe_permute_noalloc: null pointer");
+  if (rows_cap < moe_perm_rows_max(T, k, E))
+    return moe::set_error(MOE_ERR_ARG, "moe_permute_noalloc: rows_cap %lld < %lld",
+                          (long long)rows_cap, (long long)moe_perm_rows_max(T, k, E));
+  if (rows_cap >= (int64_t(1) << 31))
+    return moe::set_error(MOE_ERR_UNSUPPORTED, "moe_permute_noalloc: rows_cap >= 2^31");
+  if ((x && !moe::aligned16(x)) || (x_perm && !moe::aligned16(x_perm)))
+    return moe::set_error(MOE_ERR_ARG, "moe_permute_noalloc: x/x_perm not 16-byte aligned");
+  int32_t *hist = nullptr;
+  if (int st = noalloc_scratch(&hist)) return st;
+  const int nblk = int(nblk64);
+  MOE_LAUNCH("perm_hist", s, perm_hist_kernel<<<nblk, kThreads, 0, s>>>(topk_idx, A, E, nblk, hist));
+  if (int st = moe::launch_status("moe_permute_noalloc: hist")) return st;
+  MOE_LAUNCH("perm_scan", s, perm_scan_kernel<<<1, 1024, 0, s>>>(hist, E, nblk, counts, rows_cap,
+                                                                  group_offsets, group_counts));
+  if (int st = moe::launch_status("moe_permute_noalloc: scan")) return st;
+  if (A > 0) {
+    MOE_LAUNCH("perm_rank", s, perm_rank_kernel<<<nblk, kThreads, 0, s>>>(
+                                   topk_idx, A, E, nblk, hist, group_offsets, rows_cap,
+                                   row_of_assignment));
+    if (int st = moe::launch_status("moe_permute_noalloc: rank")) return st;
+    MOE_LAUNCH("perm_gather", s, perm_gather_kernel<<<warp_grid(T), kThreads, 0, s>>>(
+                                     x, row_of_assignment, T, d, k, rows_cap, x_perm));
+    if (int st = moe::launch_status("moe_permute_noalloc: gather")) return st;
+  }
+  MOE_LAUNCH("pad_zero", s, pad_zero_kernel<<<E, kThreads, 0, s>>>(group_offsets, group_counts, E,
+                                                                    d, rows_cap, x_perm));
+  return moe::launch_status("moe_permute_noalloc: pad");
+}

@@ -138,6 +138,8 @@ class Workload:
         self.inp = inp
         T, d, E, k, F = c.T, c.d, c.E, c.k, c.F
         self.mask = None
+        self.keep = None
+        self.counts0 = None
         self.n_pruned = 0
         compact = c.compact if compact_override is None else compact_override
         if c.prune_lowest:
@@ -145,11 +147,13 @@ class Workload:
             b0 = layer.MoELayerBuffers(layer.LayerShape(T, d, E, k, F), device, backward=False)
             layer.route(b0, inp["x"], inp["w_router"], inp["bias"])
             counts = b0.counts.cpu().tolist()
+            self.counts0 = counts
             del b0
             mask, self.n_pruned = layer.prune_from_counts(counts, T, k,
                                                           prune_count=c.prune_lowest)
             if compact:
                 keep = torch.nonzero(mask).flatten().to(device)
+                self.keep = keep.cpu().numpy()
                 inp["w_router"] = inp["w_router"].index_select(1, keep).contiguous()
                 inp["bias"] = inp["bias"].index_select(0, keep).contiguous()
                 inp["w_gate_up"] = inp["w_gate_up"].index_select(0, keep).contiguous()

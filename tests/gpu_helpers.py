@@ -60,8 +60,9 @@ def run_gpu_layer(inp, E, k, mask=None, logits_in=None, backward=True):
 
 
 def topk_margin(z32, k):
-    """Gap between the k-th and (k+1)-th largest logit per token (inf if no k+1-th)."""
-    z = np.sort(np.asarray(z32, np.float64), axis=1)[:, ::-1]
+    """Smallest gap among the k+1 largest logits per token: above the rounding of
+    the logits, the ordered top-k is unique (inf gaps past the last expert)."""
+    z = np.sort(np.asarray(z32, np.float64), axis=1)[:, ::-1][:, :k + 1]
     if z.shape[1] <= k:
-        return np.full(z.shape[0], np.inf)
-    return z[:, k - 1] - z[:, k]
+        z = np.concatenate([z, np.full((z.shape[0], 1), -np.inf)], axis=1)
+    return (z[:, :-1] - z[:, 1:]).min(axis=1)

@@ -45,6 +45,24 @@ GEMMS = ["gemm_gate_up", "gemm_down", "gemm_dgrad_down", "gemm_dgrad_gate_up",
          "gemm_wgrad_down", "gemm_wgrad_gate_up"]
 
 
+def committed_traffic(kernel):
+    """DRAM bytes per launch of `kernel` from the committed ncu capture, or None when
+    the kernel sources changed since the counters were taken (or no capture exists)."""
+    import hashlib
+    path = os.path.join(ROOT, "profiles", "dram_traffic_laep_pruned_fwdbwd_T16384.json")
+    if not os.path.exists(path):
+        return None
+    with open(path) as f:
+        rec = json.load(f)
+    h = hashlib.sha256()
+    for src in rec["sources"]:
+        with open(os.path.join(ROOT, src), "rb") as f:
+            h.update(f.read())
+    if h.hexdigest() != rec["sources_sha256"]:
+        return None
+    return rec["dram_bytes_per_launch"].get(kernel)
+
+
 def measured_peaks():
     path = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(path):
@@ -234,6 +252,93 @@ def host_inputs(inp, n_tok):
     return out
 
 
+def timed_steps(wl, steps, world, local):
+    """K timed steps between barrier+synchronize; returns (max-over-ranks ms, per-kernel
+    CUDA-event table, clock samples)."""
+    stream = torch.cuda.current_stream()
+    clocks = ClockSampler(local)
+    L.moe_timing_enable(True)
+    L.moe_timing_read(reset=True)
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    barrier(world)
+    torch.cuda.synchronize()
+    clocks.start()
+    time.sleep(0.3)  # let the sampler start
+    ev0.record(stream)
+    for _ in range(steps):
+        wl.step()
+    ev1.record(stream)
+    torch.cuda.synchronize()
+    barrier(world)
+    clk = clocks.stop()
+    L.moe_timing_enable(False)
+    per_kernel = L.moe_timing_read(reset=True)
+    assert L.moe_device_error(clear=True) == 0, "device error during the timed steps"
+    return max_over_ranks(ev0.elapsed_time(ev1), world), per_kernel, clk
+
+
+def kernel_report(wl, per_kernel, steps, peaks):
+    """Per-kernel live CUDA-event times with achieved rates against the roofline."""
+    s = wl.shape
+    A = s.T * s.k
+    flops = wl.gemm_flops()
+    hbm = {  # algorithmic bytes per launch of the HBM-bound kernels
+        "perm_gather": 2 * s.T * s.d + 2 * A * s.d,
+        "combine": 2 * A * s.d + 2 * s.T * s.d,
+        "combine_bwd": 2 * s.T * s.d + 4 * A * s.d,
+        "permute_bwd": 2 * A * s.d + 2 * s.T * s.d,
+        "route_bwd_partial": 2 * A * s.d,
+    }
+    tot = sum(v[1] for v in per_kernel.values())
+    out = {}
+    for n, (c, ms) in per_kernel.items():
+        e = {"launches": c, "ms_per_step": round(ms / steps, 4), "share": round(ms / tot, 4)}
+        per_launch_s = ms / c / 1e3
+        if n in flops:
+            tf = flops[n] / per_launch_s / 1e12
+            e.update(tflops=round(tf, 1), frac=round(tf / peaks["bf16_tflops_sustained"], 4))
+        elif n in hbm:
+            gbs = hbm[n] / per_launch_s / 1e9
+            e.update(gbs=round(gbs, 1), frac=round(gbs / peaks["hbm_gbs"], 4))
+        elif n == "route":
+            tf = 2.0 * s.T * s.d * s.E / per_launch_s / 1e12
+            e.update(fp32_tflops=round(tf, 2))
+        out[n] = e
+    return out
+
+
+PARAMS_NOTE = ("paper context (Table 5, 824 AI chips, BF16, expert parallelism): LAEP lifts "
+               "pre-training from 62.14 to 92.60 TFLOPS per chip (+49%) and cuts parameters "
+               "1515B -> 1010B (-33.3%); on one GPU with fixed top-k the FLOPs are unchanged, so "
+               "only weight bytes, dW writes and ragged tiles differ")
+
+
+def laep_comparison(args, world, local, pruned_tps, wl_pruned):
+    """Same workload without pruning (all experts live), timed the same way."""
+    steps = max(3, min(args.steps, 10))
+    pruned_params = 3 * wl_pruned.shape.E * wl_pruned.shape.d * wl_pruned.shape.F
+    c = wl_pruned.cfg
+    # free the pruned workload's activations while the unpruned one runs
+    saved = wl_pruned.bufs
+    wl_pruned.bufs = None
+    torch.cuda.empty_cache()
+    wl_u = Workload(args.config, "cuda", no_prune=True)
+    for _ in range(args.warmup):
+        wl_u.step()
+    ms_u, _, _ = timed_steps(wl_u, steps, world, local)
+    tps_u = world * wl_u.shape.T * steps / (ms_u / 1e3)
+    unpruned_params = 3 * wl_u.shape.E * wl_u.shape.d * wl_u.shape.F
+    del wl_u
+    torch.cuda.empty_cache()
+    wl_pruned.bufs = saved
+    return {"experts_unpruned": c.E, "experts_pruned": wl_pruned.shape.E,
+            "unpruned_tokens_per_s": round(tps_u, 1), "pruned_tokens_per_s": round(pruned_tps, 1),
+            "speedup": round(pruned_tps / tps_u, 4),
+            "expert_params_unpruned": unpruned_params, "expert_params_pruned": pruned_params,
+            "expert_param_reduction": round(1 - pruned_params / unpruned_params, 4),
+            "unpruned_steps": steps, "context": PARAMS_NOTE}
+
+
 def run_ours(args):
     world, rank, local = dist_setup(args.gpus)
     L.load()
@@ -248,29 +353,10 @@ def run_ours(args):
     assert L.moe_device_error(clear=True) == 0, "device error during warm-up"
 
     stream = torch.cuda.current_stream()
-    clocks = ClockSampler(local)
-    L.moe_timing_enable(True)
-    L.moe_timing_read(reset=True)
-    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    barrier(world)
-    torch.cuda.synchronize()
-    clocks.start()
-    time.sleep(0.3)  # let the sampler start
-    ev0.record(stream)
-    for _ in range(args.steps):
-        wl.step()
-    ev1.record(stream)
-    torch.cuda.synchronize()
-    barrier(world)
-    clk = clocks.stop()
-    L.moe_timing_enable(False)
-    per_kernel = L.moe_timing_read(reset=True)
-    ms_total = ev0.elapsed_time(ev1)
-    ms_total = max_over_ranks(ms_total, world)
+    ms_total, per_kernel, clk = timed_steps(wl, args.steps, world, local)
     ms_step = ms_total / args.steps
     tokens_per_s = world * s.T * args.steps / (ms_total / 1e3)
     launches = sum(n for n, _ in per_kernel.values())
-    assert L.moe_device_error(clear=True) == 0, "device error during the timed steps"
 
     # dominant kernel and its roofline
     gemm_ms = {n: per_kernel[n][1] / per_kernel[n][0] for n in GEMMS if n in per_kernel}
@@ -280,9 +366,10 @@ def run_ours(args):
     all_gemm_ms = sum(per_kernel[n][1] for n in gemm_ms) / args.steps
     all_gemm_tflops = sum(flops.values()) / (all_gemm_ms / 1e3) / 1e12
     peak = peaks["bf16_tflops_sustained"]
-    kernel_table = {n: {"launches": c, "ms_per_step": round(ms / args.steps, 4),
-                        "share": round(ms / sum(v[1] for v in per_kernel.values()), 4)}
-                    for n, (c, ms) in per_kernel.items()}
+    kernel_table = kernel_report(wl, per_kernel, args.steps, peaks)
+    laep = None
+    if wl.cfg.compact and args.tokens is None and args.experts is None and not args.no_prune:
+        laep = laep_comparison(args, world, local, tokens_per_s, wl)
 
     # end to end through the public API: pinned host inputs in, results out
     e2e = None
@@ -303,6 +390,7 @@ def run_ours(args):
 
         for _ in range(2):
             e2e_step()
+        ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         barrier(world)
         torch.cuda.synchronize()
         ev0.record(stream)
@@ -343,8 +431,11 @@ def run_ours(args):
                          "ms_per_step": round(all_gemm_ms, 4)},
         "roofline": {"kernel": dom, "bound": "tensor", "achieved": round(dom_tflops, 1),
                      "peak": peak, "unit": "TFLOP/s", "frac": round(dom_tflops / peak, 4),
-                     "traffic": None, "peak_source": f"bf16 sustained ({peaks['source']})"},
+                     "traffic": (committed_traffic(dom) if wl.cfg_id == 2 and args.tokens is None
+                                 and args.experts is None and not args.no_prune else None),
+                     "peak_source": f"bf16 sustained ({peaks['source']})"},
         "kernels": kernel_table,
+        "laep": laep,
         "gpu_launches": launches,
         "clocks": clk,
         "e2e": e2e,

@@ -21,6 +21,7 @@
 //   kWgradDown   dW_down[e] = dO_e^T H_e  (A and B MN-major; K = group rows)
 //   kWgradGateUp dW_gu[e] = [dA|dB]_e^T X_e
 #include <cuda.h>
+#include <stdlib.h>
 
 #include "common.cuh"
 #include "tc_ptx.cuh"
@@ -98,6 +99,91 @@ __device__ __forceinline__ void store_row_bf16(uint16_t *dst, const uint32_t (&r
 }
 
 __device__ __forceinline__ float silu_f(float a) { return a / (1.f + __expf(-a)); }
+
+// Epilogue of one accumulator tile for the 32 rows this warp owns: reads the fp32
+// accumulator from tensor memory at `tb` (lane base and column base included) and
+// writes the mode's outputs. `row` = row of this thread in the grouped layout
+// (activation modes), `out_row` = row in the expert's weight-gradient matrix.
+template <int MODE, int BN>
+__device__ __forceinline__ void epilogue_tile(const GemmParams &p, uint32_t tb, size_t row,
+                                              int out_row, int e, int nt) {
+  using Tr = Traits<MODE>;
+  if (MODE == kGateUp) {
+    const int F = p.F;
+    uint16_t *hrow = p.out + row * F + nt * 128;
+    uint16_t *arow = p.out2 + row * 2 * F + nt * 128;
+    uint16_t *brow = arow + F;
+#pragma unroll 1
+    for (int c = 0; c < 128; c += 32) {
+      uint32_t ra[32], rb[32];
+      tc::tmem_ld_32x32b_x32(tb + c, ra);
+      tc::tmem_ld_32x32b_x32(tb + 128 + c, rb);
+      tc::tmem_ld_wait();
+#pragma unroll
+      for (int v = 0; v < 4; ++v) {
+        float fa[8], fb[8], fh[8];
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+          fa[i] = __uint_as_float(ra[v * 8 + i]);
+          fb[i] = __uint_as_float(rb[v * 8 + i]);
+          fh[i] = silu_f(fa[i]) * fb[i];
+        }
+        stg_v4(hrow + c + v * 8, pack8(fh));
+        stg_v4(arow + c + v * 8, pack8(fa));
+        stg_v4(brow + c + v * 8, pack8(fb));
+      }
+    }
+  } else if (MODE == kDgradDown) {
+    const int F = p.F;
+    const int f0 = nt * BN;
+    const uint16_t *arow = p.aux + row * 2 * F + f0;
+    const uint16_t *brow = arow + F;
+    uint16_t *darow = p.out + row * 2 * F + f0;
+    uint16_t *dbrow = darow + F;
+#pragma unroll 1
+    for (int c = 0; c < BN; c += 32) {
+      uint4 va[4], vb[4];
+#pragma unroll
+      for (int v = 0; v < 4; ++v) {
+        va[v] = ldg_nc_v4(arow + c + v * 8);
+        vb[v] = ldg_nc_v4(brow + c + v * 8);
+      }
+      uint32_t r[32];
+      tc::tmem_ld_32x32b_x32(tb + c, r);
+      tc::tmem_ld_wait();
+#pragma unroll
+      for (int v = 0; v < 4; ++v) {
+        float fa[8], fb[8], da[8], db[8];
+        unpack8(va[v], fa);
+        unpack8(vb[v], fb);
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+          const float dh = __uint_as_float(r[v * 8 + i]);
+          const float sg = 1.f / (1.f + __expf(-fa[i]));
+          da[i] = dh * fb[i] * (sg * (1.f + fa[i] * (1.f - sg)));
+          db[i] = dh * fa[i] * sg;
+        }
+        stg_v4(darow + c + v * 8, pack8(da));
+        stg_v4(dbrow + c + v * 8, pack8(db));
+      }
+    }
+  } else {
+    uint16_t *orow;
+    if (Tr::WGRAD) {
+      const int M_out = p.m_tiles_w * BM, N_out = p.n_tiles * BN;
+      orow = p.out + (size_t(e) * M_out + out_row) * N_out + nt * BN;
+    } else {
+      orow = p.out + row * p.d + nt * BN;
+    }
+#pragma unroll 1
+    for (int c = 0; c < BN; c += 32) {
+      uint32_t r[32];
+      tc::tmem_ld_32x32b_x32(tb + c, r);
+      tc::tmem_ld_wait();
+      store_row_bf16(orow + c, r);
+    }
+  }
+}
 
 template <int MODE, int BN>
 __global__ void __launch_bounds__(kThreads, 1)
@@ -317,84 +403,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       tc::fence_after_sync();
       const uint32_t tb = tmem_base + (uint32_t(q * 32) << 16) + a * BN;
 
-      if (MODE == kGateUp) {
-        const int F = p.F;
-        const size_t row = size_t(t.goff) + t.mt * BM + r_in_tile;
-        uint16_t *hrow = p.out + row * F + t.nt * 128;
-        uint16_t *arow = p.out2 + row * 2 * F + t.nt * 128;
-        uint16_t *brow = arow + F;
-#pragma unroll 1
-        for (int c = 0; c < 128; c += 32) {
-          uint32_t ra[32], rb[32];
-          tc::tmem_ld_32x32b_x32(tb + c, ra);
-          tc::tmem_ld_32x32b_x32(tb + 128 + c, rb);
-          tc::tmem_ld_wait();
-#pragma unroll
-          for (int v = 0; v < 4; ++v) {
-            float fa[8], fb[8], fh[8];
-#pragma unroll
-            for (int i = 0; i < 8; ++i) {
-              fa[i] = __uint_as_float(ra[v * 8 + i]);
-              fb[i] = __uint_as_float(rb[v * 8 + i]);
-              fh[i] = silu_f(fa[i]) * fb[i];
-            }
-            stg_v4(hrow + c + v * 8, pack8(fh));
-            stg_v4(arow + c + v * 8, pack8(fa));
-            stg_v4(brow + c + v * 8, pack8(fb));
-          }
-        }
-      } else if (MODE == kDgradDown) {
-        const int F = p.F;
-        const size_t row = size_t(t.goff) + t.mt * BM + r_in_tile;
-        const int f0 = t.nt * BN;
-        const uint16_t *arow = p.aux + row * 2 * F + f0;
-        const uint16_t *brow = arow + F;
-        uint16_t *darow = p.out + row * 2 * F + f0;
-        uint16_t *dbrow = darow + F;
-#pragma unroll 1
-        for (int c = 0; c < BN; c += 32) {
-          uint4 va[4], vb[4];
-#pragma unroll
-          for (int v = 0; v < 4; ++v) {
-            va[v] = ldg_nc_v4(arow + c + v * 8);
-            vb[v] = ldg_nc_v4(brow + c + v * 8);
-          }
-          uint32_t r[32];
-          tc::tmem_ld_32x32b_x32(tb + c, r);
-          tc::tmem_ld_wait();
-#pragma unroll
-          for (int v = 0; v < 4; ++v) {
-            float fa[8], fb[8], da[8], db[8];
-            unpack8(va[v], fa);
-            unpack8(vb[v], fb);
-#pragma unroll
-            for (int i = 0; i < 8; ++i) {
-              const float dh = __uint_as_float(r[v * 8 + i]);
-              const float sg = 1.f / (1.f + __expf(-fa[i]));
-              da[i] = dh * fb[i] * (sg * (1.f + fa[i] * (1.f - sg)));
-              db[i] = dh * fa[i] * sg;
-            }
-            stg_v4(darow + c + v * 8, pack8(da));
-            stg_v4(dbrow + c + v * 8, pack8(db));
-          }
-        }
-      } else {
-        uint16_t *orow;
-        if (Tr::WGRAD) {
-          const int M_out = p.m_tiles_w * BM, N_out = p.n_tiles * BN;
-          orow = p.out + (size_t(t.e) * M_out + t.mt * BM + r_in_tile) * N_out + t.nt * BN;
-        } else {
-          const size_t row = size_t(t.goff) + t.mt * BM + r_in_tile;
-          orow = p.out + row * p.d + t.nt * BN;
-        }
-#pragma unroll 1
-        for (int c = 0; c < BN; c += 32) {
-          uint32_t r[32];
-          tc::tmem_ld_32x32b_x32(tb + c, r);
-          tc::tmem_ld_wait();
-          store_row_bf16(orow + c, r);
-        }
-      }
+      epilogue_tile<MODE, BN>(p, tb, size_t(t.goff) + size_t(t.mt) * BM + r_in_tile,
+                              t.mt * BM + r_in_tile, t.e, t.nt);
       tc::fence_before_sync();
       __syncwarp();
       if (lane == 0) tc::mbar_arrive(tempty_bar(a));
@@ -407,6 +417,281 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (warp == 1) {
     tc::fence_after_sync();
     tc::tmem_dealloc(tmem_base, Sh::TMEM_COLS);
+  }
+}
+
+
+// ============================================================================
+// CTA-pair variant (cta_group::2): a cluster of two CTAs on two SMs computes a
+// 256 x BN tile. Each CTA stages its own 128 rows of A and half of B (BN/2 rows)
+// per k-block; one thread of the even CTA issues M=256 MMAs that read both CTAs'
+// shared memory and write each CTA's 128 accumulator rows into its own TMEM.
+// Per SM this moves 32 KB per k-block instead of 48 KB through shared memory
+// and L2, and the ring gets 6 stages (BN 256) or 8 (BN 128).
+// Synchronization: both CTAs' loads complete on the even CTA's `full` barrier
+// (it expects both CTAs' bytes); the MMA commit arrives on the `empty` and
+// `tfull` barriers of both CTAs; both CTAs' epilogue warps arrive on the even
+// CTA's `tempty` barrier. Tiles whose odd row block lies past the group (a group
+// with an odd number of 128-row blocks) are computed but not stored.
+// ============================================================================
+template <int BN> struct PairShape {
+  static constexpr int BNH = BN / 2;  // B rows staged by each CTA
+  static constexpr int STAGES = BN == 256 ? 6 : 8;
+  static constexpr uint32_t A_BYTES = BM * BK * 2;
+  static constexpr uint32_t B_BYTES = BNH * BK * 2;
+  static constexpr uint32_t STAGE_BYTES = A_BYTES + B_BYTES;
+  static constexpr int NBARS = 2 * STAGES + 5;
+  static constexpr size_t SMEM = 1024 + size_t(STAGES) * STAGE_BYTES + NBARS * 8 +
+                                 (4 + 257 + 256 + 257) * 4;
+  static constexpr uint32_t TMEM_COLS = 2 * BN;
+};
+
+struct PairTile {
+  int e, goff, mp, nt, nkb, mtiles;
+};
+
+template <int MODE, int BN>
+__global__ void __launch_bounds__(kThreads, 1)
+    grouped_gemm_pair_kernel(const __grid_constant__ CUtensorMap tmA,
+                             const __grid_constant__ CUtensorMap tmB, const GemmParams p) {
+  using Tr = Traits<MODE>;
+  using Sh = PairShape<BN>;
+  constexpr int STAGES = Sh::STAGES;
+  constexpr int BNH = Sh::BNH;
+  constexpr uint32_t IDESC = tc::idesc_bf16_f32(2 * BM, BN, Tr::A_MN, Tr::B_MN);
+
+  extern __shared__ uint8_t smem_raw[];
+  const uint32_t raw = tc::smem_u32(smem_raw);
+  const uint32_t pad = (1024u - (raw & 1023u)) & 1023u;
+  uint8_t *smem = smem_raw + pad;
+  const uint32_t sA0 = raw + pad;
+  const uint32_t sB0 = sA0 + STAGES * Sh::A_BYTES;
+  uint64_t *bars = reinterpret_cast<uint64_t *>(smem + STAGES * Sh::STAGE_BYTES);
+  int *misc = reinterpret_cast<int *>(bars + Sh::NBARS);
+  int *s_goff = misc + 4;
+  int *s_order = s_goff + 257;
+  int *s_prefix = s_order + 256;
+  volatile int *abort_flag = misc + 1;
+  volatile int no_abort = 0;
+
+  const uint32_t bar0 = tc::smem_u32(bars);
+  auto full_bar = [&](int s) { return bar0 + 8u * s; };
+  auto empty_bar = [&](int s) { return bar0 + 8u * (STAGES + s); };
+  auto tfull_bar = [&](int a) { return bar0 + 8u * (2 * STAGES + a); };
+  auto tempty_bar = [&](int a) { return bar0 + 8u * (2 * STAGES + 2 + a); };
+  const uint32_t drain_bar = bar0 + 8u * (2 * STAGES + 4);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int E = p.E;
+  const uint32_t rank = tc::cluster_ctarank();
+  const bool leader = rank == 0;
+  const int cluster = int(tc::cluster_id_x());
+  const int nclusters = int(tc::cluster_count_x());
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < STAGES; ++s) {
+      tc::mbar_init(full_bar(s), 1);
+      tc::mbar_init(empty_bar(s), 1);
+    }
+    for (int a = 0; a < 2; ++a) {
+      tc::mbar_init(tfull_bar(a), 1);
+      tc::mbar_init(tempty_bar(a), 8);  // 4 epilogue warps in each CTA of the pair
+    }
+    tc::mbar_init(drain_bar, 1);
+    tc::fence_mbar_init();
+    misc[1] = 0;
+  }
+  if (warp == 0 && lane == 0) {
+    tc::tma_prefetch_desc(&tmA);
+    tc::tma_prefetch_desc(&tmB);
+  }
+  if (warp == 1) {
+    tc::tmem_alloc_pair(tc::smem_u32(misc), Sh::TMEM_COLS);
+    tc::tmem_relinquish_pair();
+  }
+  // ---- tile schedule: identical in both CTAs of every pair ----
+  for (int e = threadIdx.x; e <= E; e += kThreads) s_goff[e] = p.group_offsets[e];
+  __syncthreads();
+  if (Tr::WGRAD) {
+    for (int e = threadIdx.x; e < E; e += kThreads) {
+      const int ce = s_goff[e + 1] - s_goff[e];
+      int r = 0;
+      for (int q = 0; q < E; ++q) {
+        const int cq = s_goff[q + 1] - s_goff[q];
+        r += (cq > ce) || (cq == ce && q < e);
+      }
+      s_order[r] = e;
+    }
+  } else {
+    for (int e = threadIdx.x; e < E; e += kThreads) s_order[e] = e;
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    int acc = 0;
+    for (int i = 0; i < E; ++i) {
+      s_prefix[i] = acc;
+      const int e = s_order[i];
+      const int mt = Tr::WGRAD ? p.m_tiles_w : (s_goff[e + 1] - s_goff[e]) / BM;
+      acc += ((mt + 1) / 2) * p.n_tiles;
+    }
+    s_prefix[E] = acc;
+  }
+  tc::fence_before_sync();
+  __syncthreads();
+  tc::cluster_sync();  // barriers of both CTAs initialized before any remote use
+  tc::fence_after_sync();
+  const uint32_t tmem_base = static_cast<uint32_t>(misc[0]);
+  const int total = s_prefix[E];
+
+  auto decode = [&](int tile) {
+    int lo = 0, hi = E - 1;
+    while (lo < hi) {
+      const int mid = (lo + hi + 1) >> 1;
+      if (s_prefix[mid] <= tile) lo = mid; else hi = mid - 1;
+    }
+    PairTile t;
+    const int local = tile - s_prefix[lo];
+    t.e = s_order[lo];
+    t.goff = s_goff[t.e];
+    t.mp = local / p.n_tiles;
+    t.nt = local - t.mp * p.n_tiles;
+    const int rows = s_goff[t.e + 1] - t.goff;
+    t.nkb = Tr::WGRAD ? rows / BK : p.nkb;
+    t.mtiles = Tr::WGRAD ? p.m_tiles_w : rows / BM;
+    return t;
+  };
+
+  if (warp == 0) {
+    // ============ TMA producer (one thread in each CTA) ============
+    if (lane == 0) {
+      const uint32_t full_leader = tc::mapa(full_bar(0), 0);
+      uint32_t it = 0;
+      bool ok = true;
+      for (int tile = cluster; tile < total && ok; tile += nclusters) {
+        const PairTile t = decode(tile);
+        const int mt = 2 * t.mp + int(rank);  // this CTA's 128-row block
+        for (int kb = 0; kb < t.nkb; ++kb, ++it) {
+          const int s = it % STAGES;
+          const uint32_t ph = (it / STAGES) & 1u;
+          if (!tc::mbar_wait(empty_bar(s), ph ^ 1u, kWaitLimitNs, abort_flag)) { fail(abort_flag); ok = false; break; }
+          if (leader) tc::mbar_arrive_expect_tx(full_bar(s), 2 * Sh::STAGE_BYTES);
+          const uint32_t a_dst = sA0 + s * Sh::A_BYTES, b_dst = sB0 + s * Sh::B_BYTES;
+          const uint32_t fb = full_leader + 8u * s;
+          const int k0 = kb * BK;
+          if (MODE == kGateUp) {  // even CTA: gate rows, odd CTA: up rows
+            tc::tma_load_2d_pair(a_dst, &tmA, fb, k0, t.goff + mt * BM);
+            tc::tma_load_2d_pair(b_dst, &tmB, fb, k0, t.e * 2 * p.F + int(rank) * p.F + t.nt * 128);
+          } else if (MODE == kDown) {
+            tc::tma_load_2d_pair(a_dst, &tmA, fb, k0, t.goff + mt * BM);
+            tc::tma_load_2d_pair(b_dst, &tmB, fb, k0, t.e * p.d + t.nt * BN + int(rank) * BNH);
+          } else if (MODE == kDgradDown || MODE == kDgradGateUp) {
+            tc::tma_load_2d_pair(a_dst, &tmA, fb, k0, t.goff + mt * BM);
+            const int krow = (MODE == kDgradDown ? t.e * p.d : t.e * 2 * p.F) + k0;
+#pragma unroll
+            for (int i = 0; i < BNH / 64; ++i)
+              tc::tma_load_2d_pair(b_dst + i * 64 * 128, &tmB, fb, t.nt * BN + int(rank) * BNH + i * 64, krow);
+          } else {  // weight gradients: both operands MN-major, K = group rows
+            const int krow = t.goff + k0;
+#pragma unroll
+            for (int i = 0; i < BM / 64; ++i)
+              tc::tma_load_2d_pair(a_dst + i * 64 * 128, &tmA, fb, mt * BM + i * 64, krow);
+#pragma unroll
+            for (int i = 0; i < BNH / 64; ++i)
+              tc::tma_load_2d_pair(b_dst + i * 64 * 128, &tmB, fb, t.nt * BN + int(rank) * BNH + i * 64, krow);
+          }
+        }
+      }
+      // Drain (even CTA): its full barriers count the loads of both CTAs.
+      if (leader) {
+        for (int s = 0; s < STAGES; ++s) {
+          if (it > uint32_t(s)) {
+            const uint32_t n = (it - 1 - s) / STAGES;
+            if (!tc::mbar_wait(full_bar(s), n & 1u, kWaitLimitNs, &no_abort)) fail(abort_flag);
+          }
+        }
+      }
+    }
+  } else if (warp == 1) {
+    // ============ MMA issuer (one thread of the even CTA) ============
+    if (leader && lane == 0) {
+      uint32_t it = 0, tcount = 0;
+      bool ok = true, issued = false;
+      for (int tile = cluster; tile < total && ok; tile += nclusters) {
+        const PairTile t = decode(tile);
+        if (t.nkb == 0) continue;
+        const uint32_t a = tcount & 1u, aph = (tcount >> 1) & 1u;
+        if (!tc::mbar_wait(tempty_bar(a), aph ^ 1u, kWaitLimitNs, abort_flag)) { fail(abort_flag); break; }
+        tc::fence_after_sync();
+        const uint32_t d_tmem = tmem_base + a * BN;
+        for (int kb = 0; kb < t.nkb; ++kb, ++it) {
+          const int s = it % STAGES;
+          const uint32_t ph = (it / STAGES) & 1u;
+          if (!tc::mbar_wait(full_bar(s), ph, kWaitLimitNs, abort_flag)) { fail(abort_flag); ok = false; break; }
+          tc::fence_after_sync();
+          const uint32_t a_s = sA0 + s * Sh::A_BYTES, b_s = sB0 + s * Sh::B_BYTES;
+#pragma unroll
+          for (int kk = 0; kk < BK / UMMA_K; ++kk) {
+            const uint64_t ad = Tr::A_MN ? tc::smem_desc_sw128(a_s + kk * 2048, 8192, 1024)
+                                         : tc::smem_desc_sw128(a_s + kk * 32, 16, 1024);
+            const uint64_t bd = Tr::B_MN ? tc::smem_desc_sw128(b_s + kk * 2048, 8192, 1024)
+                                         : tc::smem_desc_sw128(b_s + kk * 32, 16, 1024);
+            tc::mma_bf16_pair(d_tmem, ad, bd, IDESC, (kb | kk) != 0);
+          }
+          tc::mma_commit_pair_mc(empty_bar(s), 0x3);  // frees the stage in both CTAs
+          issued = true;
+        }
+        if (!ok) break;
+        tc::mma_commit_pair_mc(tfull_bar(a), 0x3);  // both halves of the accumulator ready
+        ++tcount;
+      }
+      if (issued) {
+        tc::mma_commit_pair(drain_bar);
+        if (!tc::mbar_wait(drain_bar, 0, kWaitLimitNs, &no_abort)) fail(abort_flag);
+      }
+    }
+  } else {
+    // ============ epilogue (warps 2..5 of each CTA) ============
+    const int q = warp & 3;
+    const int r_in_tile = q * 32 + lane;
+    const uint32_t tempty_leader = tc::mapa(tempty_bar(0), 0);
+    uint32_t tcount = 0;
+    for (int tile = cluster; tile < total; tile += nclusters) {
+      const PairTile t = decode(tile);
+      const int mt = 2 * t.mp + int(rank);
+      const bool mine = mt < t.mtiles;  // this CTA's row block exists
+      if (Tr::WGRAD && t.nkb == 0) {
+        if (mine) {  // empty group: its weight gradient is exactly zero
+          const int M_out = p.m_tiles_w * BM, N_out = p.n_tiles * BN;
+          uint16_t *o = p.out + (size_t(t.e) * M_out + mt * BM + r_in_tile) * N_out + t.nt * BN;
+          const uint4 z = make_uint4(0, 0, 0, 0);
+#pragma unroll 4
+          for (int c = 0; c < BN; c += 8) stg_v4(o + c, z);
+        }
+        continue;
+      }
+      const uint32_t a = tcount & 1u, aph = (tcount >> 1) & 1u;
+      const bool ok = tc::mbar_wait(tfull_bar(a), aph, kWaitLimitNs, abort_flag);
+      __syncwarp();
+      if (!ok) { fail(abort_flag); break; }
+      tc::fence_after_sync();
+      if (mine) {
+        const uint32_t tb = tmem_base + (uint32_t(q * 32) << 16) + a * BN;
+        epilogue_tile<MODE, BN>(p, tb, size_t(t.goff) + size_t(mt) * BM + r_in_tile,
+                                mt * BM + r_in_tile, t.e, t.nt);
+      }
+      tc::fence_before_sync();
+      __syncwarp();
+      if (lane == 0) tc::mbar_arrive_cluster(tempty_leader + 8u * a);
+      ++tcount;
+    }
+  }
+
+  tc::fence_before_sync();
+  __syncthreads();
+  tc::cluster_sync();  // no CTA leaves while its peer may still signal it
+  if (warp == 1) {
+    tc::fence_after_sync();
+    tc::tmem_dealloc_pair(tmem_base, Sh::TMEM_COLS);
   }
 }
 
@@ -447,16 +732,20 @@ int make_map(CUtensorMap *m, const void *base, uint64_t rows, uint64_t cols, uin
   if (r != CUDA_SUCCESS) return moe::set_error(MOE_ERR_CUDA, "tensor map for %s: CUresult %d", what, int(r));
   return MOE_OK;
 }
-int map_kmajor(CUtensorMap *m, const void *base, uint64_t rows, uint64_t cols, const char *w) {
-  return make_map(m, base, rows, cols, BK, BM, w);
-}
-int map_mnmajor(CUtensorMap *m, const void *base, uint64_t rows, uint64_t cols, const char *w) {
-  return make_map(m, base, rows, cols, 64, BK, w);
+// The CTA-pair kernel is the default; MOE_GEMM_1SM=1 selects the one-SM kernel
+// (kept for A/B measurements).
+bool use_pair() {
+  static int v = -1;
+  if (v < 0) {
+    const char *e = getenv("MOE_GEMM_1SM");
+    v = (e && e[0] == '1') ? 0 : 1;
+  }
+  return v == 1;
 }
 
 template <int MODE, int BN>
-int launch(const CUtensorMap &a, const CUtensorMap &b, const GemmParams &p, cudaStream_t s,
-           const char *what) {
+int launch_one(const CUtensorMap &a, const CUtensorMap &b, const GemmParams &p, cudaStream_t s,
+               const char *what) {
   using Sh = Shape<BN>;
   static bool attr = false;
   if (!attr) {
@@ -469,15 +758,62 @@ int launch(const CUtensorMap &a, const CUtensorMap &b, const GemmParams &p, cuda
   return moe::launch_status(what);
 }
 
-template <int MODE>
-int launch_bn(int N, const CUtensorMap &a, const CUtensorMap &b, GemmParams p, cudaStream_t s,
-              const char *what) {
-  if (N % 256 == 0) {
-    p.n_tiles = N / 256;
-    return launch<MODE, 256>(a, b, p, s, what);
+template <int MODE, int BN>
+int launch_pair(const CUtensorMap &a, const CUtensorMap &b, const GemmParams &p, cudaStream_t s,
+                const char *what) {
+  using Sh = PairShape<BN>;
+  auto kern = grouped_gemm_pair_kernel<MODE, BN>;
+  cudaLaunchAttribute at[1];
+  at[0].id = cudaLaunchAttributeClusterDimension;
+  at[0].val.clusterDim.x = 2;
+  at[0].val.clusterDim.y = 1;
+  at[0].val.clusterDim.z = 1;
+  cudaLaunchConfig_t cfg = {};
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = Sh::SMEM;
+  cfg.stream = s;
+  cfg.attrs = at;
+  cfg.numAttrs = 1;
+  static int nclusters = 0;
+  if (!nclusters) {
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, int(Sh::SMEM));
+    if (e != cudaSuccess) return moe::cuda_status(e, what);
+    cfg.gridDim = dim3(2 * (moe::num_sms() / 2));
+    int n = 0;
+    e = cudaOccupancyMaxActiveClusters(&n, kern, &cfg);
+    if (e != cudaSuccess) return moe::cuda_status(e, what);
+    if (n <= 0) return moe::set_error(MOE_ERR_CUDA, "%s: no co-resident CTA pair fits", what);
+    nclusters = n;
   }
-  p.n_tiles = N / 128;
-  return launch<MODE, 128>(a, b, p, s, what);
+  cfg.gridDim = dim3(2 * nclusters);
+  MOE_LAUNCH(kGemmName[MODE], s, cudaLaunchKernelEx(&cfg, kern, a, b, p));
+  return moe::launch_status(what);
+}
+
+// Builds the tensor maps for one GEMM and launches it. A: [a_rows, a_cols] row-major
+// bf16; B likewise. N = output columns (for kGateUp: 2F, in tiles of 128 gate + 128 up).
+template <int MODE>
+int run_gemm(int N, const void *a_base, uint64_t a_rows, uint64_t a_cols, const void *b_base,
+             uint64_t b_rows, uint64_t b_cols, GemmParams p, cudaStream_t s, const char *what) {
+  using Tr = Traits<MODE>;
+  const bool pair = use_pair();
+  const int BN = (MODE == kGateUp || N % 256 == 0) ? 256 : 128;
+  p.n_tiles = (MODE == kGateUp) ? N / 256 : N / BN;
+  CUtensorMap ma, mb;
+  int st;
+  if ((st = Tr::A_MN ? make_map(&ma, a_base, a_rows, a_cols, 64, BK, what)
+                     : make_map(&ma, a_base, a_rows, a_cols, BK, BM, what)))
+    return st;
+  const uint32_t b_box_rows = pair ? uint32_t(BN / 2) : 128u;
+  if ((st = Tr::B_MN ? make_map(&mb, b_base, b_rows, b_cols, 64, BK, what)
+                     : make_map(&mb, b_base, b_rows, b_cols, BK, b_box_rows, what)))
+    return st;
+  if (pair) {
+    return BN == 256 ? launch_pair<MODE, 256>(ma, mb, p, s, what)
+                     : launch_pair<MODE, 128>(ma, mb, p, s, what);
+  }
+  return BN == 256 ? launch_one<MODE, 256>(ma, mb, p, s, what)
+                   : launch_one<MODE, 128>(ma, mb, p, s, what);
 }
 
 int check_common(int E, int d, int F, int64_t rows_cap, const char *fn) {
@@ -510,26 +846,25 @@ int moe_grouped_ffn_fwd(const uint16_t *x_perm, const int32_t *group_offsets, in
   const void *ptrs[] = {x_perm, group_offsets, w_gate_up, w_down, ab_saved, h, out_perm};
   for (const void *q : ptrs)
     if (!q || !moe::aligned16(q)) return moe::set_error(MOE_ERR_ARG, "moe_grouped_ffn_fwd: null or unaligned pointer");
-  CUtensorMap mX, mWgu, mH, mWd;
-  int st;
-  if ((st = map_kmajor(&mX, x_perm, rows_cap, d, "x_perm"))) return st;
-  if ((st = map_kmajor(&mWgu, w_gate_up, uint64_t(E) * 2 * F, d, "w_gate_up"))) return st;
-  if ((st = map_kmajor(&mH, h, rows_cap, F, "h"))) return st;
-  if ((st = map_kmajor(&mWd, w_down, uint64_t(E) * d, F, "w_down"))) return st;
+  const uint64_t R = uint64_t(rows_cap);
   GemmParams p{};
   p.group_offsets = group_offsets;
   p.E = E; p.d = d; p.F = F;
+  // [A | B] = X W_gate_up^T, H = silu(A) * B
   p.nkb = d / BK;
-  p.n_tiles = F / 128;
   p.out = h;
   p.out2 = ab_saved;
-  if ((st = launch<kGateUp, 256>(mX, mWgu, p, s, "moe_grouped_ffn_fwd: gate/up GEMM"))) return st;
+  if (int st = run_gemm<kGateUp>(2 * F, x_perm, R, d, w_gate_up, uint64_t(E) * 2 * F, d, p, s,
+                                 "moe_grouped_ffn_fwd: gate/up GEMM"))
+    return st;
+  // O = H W_down^T
   GemmParams q{};
   q.group_offsets = group_offsets;
   q.E = E; q.d = d; q.F = F;
   q.nkb = F / BK;
   q.out = out_perm;
-  return launch_bn<kDown>(d, mH, mWd, q, s, "moe_grouped_ffn_fwd: down GEMM");
+  return run_gemm<kDown>(d, h, R, F, w_down, uint64_t(E) * d, F, q, s,
+                         "moe_grouped_ffn_fwd: down GEMM");
 }
 
 int moe_grouped_ffn_bwd(const uint16_t *d_out_perm, const uint16_t *x_perm,
@@ -546,17 +881,8 @@ int moe_grouped_ffn_bwd(const uint16_t *d_out_perm, const uint16_t *x_perm,
                         d_ab, dx_perm, dw_gate_up, dw_down};
   for (const void *q : ptrs)
     if (!q || !moe::aligned16(q)) return moe::set_error(MOE_ERR_ARG, "moe_grouped_ffn_bwd: null or unaligned pointer");
-  CUtensorMap mdO_k, mWd_mn, mdAB_k, mWgu_mn, mdO_mn, mH_mn, mdAB_mn, mX_mn;
+  const uint64_t R = uint64_t(rows_cap);
   int st;
-  if ((st = map_kmajor(&mdO_k, d_out_perm, rows_cap, d, "d_out_perm"))) return st;
-  if ((st = map_mnmajor(&mWd_mn, w_down, uint64_t(E) * d, F, "w_down"))) return st;
-  if ((st = map_kmajor(&mdAB_k, d_ab, rows_cap, 2 * F, "d_ab"))) return st;
-  if ((st = map_mnmajor(&mWgu_mn, w_gate_up, uint64_t(E) * 2 * F, d, "w_gate_up"))) return st;
-  if ((st = map_mnmajor(&mdO_mn, d_out_perm, rows_cap, d, "d_out_perm"))) return st;
-  if ((st = map_mnmajor(&mH_mn, h, rows_cap, F, "h"))) return st;
-  if ((st = map_mnmajor(&mdAB_mn, d_ab, rows_cap, 2 * F, "d_ab"))) return st;
-  if ((st = map_mnmajor(&mX_mn, x_perm, rows_cap, d, "x_perm"))) return st;
-
   GemmParams p{};
   p.group_offsets = group_offsets;
   p.E = E; p.d = d; p.F = F;
@@ -564,21 +890,28 @@ int moe_grouped_ffn_bwd(const uint16_t *d_out_perm, const uint16_t *x_perm,
   p.nkb = d / BK;
   p.out = d_ab;
   p.aux = ab_saved;
-  if ((st = launch_bn<kDgradDown>(F, mdO_k, mWd_mn, p, s, "moe_grouped_ffn_bwd: dH GEMM"))) return st;
+  if ((st = run_gemm<kDgradDown>(F, d_out_perm, R, d, w_down, uint64_t(E) * d, F, p, s,
+                                 "moe_grouped_ffn_bwd: dH GEMM")))
+    return st;
   // dX = [dA | dB] W_gate_up
   p.nkb = 2 * F / BK;
   p.out = dx_perm;
   p.aux = nullptr;
-  if ((st = launch_bn<kDgradGateUp>(d, mdAB_k, mWgu_mn, p, s, "moe_grouped_ffn_bwd: dX GEMM"))) return st;
+  if ((st = run_gemm<kDgradGateUp>(d, d_ab, R, 2 * F, w_gate_up, uint64_t(E) * 2 * F, d, p, s,
+                                   "moe_grouped_ffn_bwd: dX GEMM")))
+    return st;
   // dW_down[e] = dO_e^T H_e   ([d, F])
   p.nkb = 0;
   p.m_tiles_w = d / BM;
   p.out = dw_down;
-  if ((st = launch_bn<kWgradDown>(F, mdO_mn, mH_mn, p, s, "moe_grouped_ffn_bwd: dW_down GEMM"))) return st;
+  if ((st = run_gemm<kWgradDown>(F, d_out_perm, R, d, h, R, F, p, s,
+                                 "moe_grouped_ffn_bwd: dW_down GEMM")))
+    return st;
   // dW_gate_up[e] = [dA | dB]_e^T X_e   ([2F, d])
   p.m_tiles_w = 2 * F / BM;
   p.out = dw_gate_up;
-  return launch_bn<kWgradGateUp>(d, mdAB_mn, mX_mn, p, s, "moe_grouped_ffn_bwd: dW_gate_up GEMM");
+  return run_gemm<kWgradGateUp>(d, d_ab, R, 2 * F, x_perm, R, d, p, s,
+                                "moe_grouped_ffn_bwd: dW_gate_up GEMM");
 }
 
 }  // extern "C"

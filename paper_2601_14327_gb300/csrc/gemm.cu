@@ -9,7 +9,8 @@
 // the expert loads, and empty groups produce no tile. In the weight-gradient
 // GEMMs (reduction over a group's rows, so tile cost ~ group size) the
 // experts are ordered heaviest first, the longest-processing-time order that
-// Algorithm 2's greedy balancing also uses.
+// Algorithm 2's greedy balancing also uses (experts without rows go first: their
+// tiles are zero stores that overlap the first MMAs).
 //
 // Six GEMM shapes share one kernel template:
 //   kGateUp      [A|B] = X W_gu^T        (A: K-major rows, B: K-major weights)
@@ -244,11 +245,15 @@ __global__ void __launch_bounds__(kThreads, 1)
   __syncthreads();
   if (Tr::WGRAD) {
     for (int e = threadIdx.x; e < E; e += kThreads) {
+      // empty experts first (their zero tiles are stores only and overlap the
+      // first MMAs), then heaviest first; ties keep the expert order
       const int ce = s_goff[e + 1] - s_goff[e];
+      const unsigned ke = ce == 0 ? 0xffffffffu : unsigned(ce);
       int r = 0;
       for (int q = 0; q < E; ++q) {
         const int cq = s_goff[q + 1] - s_goff[q];
-        r += (cq > ce) || (cq == ce && q < e);
+        const unsigned kq = cq == 0 ? 0xffffffffu : unsigned(cq);
+        r += (kq > ke) || (kq == ke && q < e);
       }
       s_order[r] = e;
     }
@@ -514,11 +519,15 @@ __global__ void __launch_bounds__(kThreads, 1)
   __syncthreads();
   if (Tr::WGRAD) {
     for (int e = threadIdx.x; e < E; e += kThreads) {
+      // empty experts first (their zero tiles are stores only and overlap the
+      // first MMAs), then heaviest first; ties keep the expert order
       const int ce = s_goff[e + 1] - s_goff[e];
+      const unsigned ke = ce == 0 ? 0xffffffffu : unsigned(ce);
       int r = 0;
       for (int q = 0; q < E; ++q) {
         const int cq = s_goff[q + 1] - s_goff[q];
-        r += (cq > ce) || (cq == ce && q < e);
+        const unsigned kq = cq == 0 ? 0xffffffffu : unsigned(cq);
+        r += (kq > ke) || (kq == ke && q < e);
       }
       s_order[r] = e;
     }

@@ -13,16 +13,19 @@ MOE_DEV_ERR_DECL
 namespace {
 
 constexpr int kRouteThreads = 256;
-constexpr int kBK = 32;  // reduction chunk of the logit contraction
+constexpr int kBK = 16;  // reduction chunk of the logit contraction
+constexpr int kBM = 64;  // tokens per CTA
 
-// Padded expert count NE -> tokens per thread TM (accumulators TM x NE/32).
+// Padded expert count NE (multiple of 64). 16 x 16 threads: thread (tx, ty) owns
+// tokens ty*4 .. ty*4+3 and experts j*64 + tx*4 + q (j < NE/64, q < 4), so the
+// shared-memory reads of one row of W are contiguous float4s across tx.
 template <int NE> struct RouteShape {
-  static constexpr int TN = NE / 32;
-  static constexpr int TM = NE == 64 ? 16 : (NE == 128 ? 8 : 4);
-  static constexpr int BM = 8 * TM;  // tokens per CTA
-  static constexpr int LDL = NE + 1; // logits row stride in shared memory
-  static constexpr size_t kGemmSmem = size_t(kBK) * BM * 4 + size_t(kBK) * NE * 4;
-  static constexpr size_t kLogitSmem = size_t(BM) * LDL * 4;
+  static constexpr int TN = NE / 16;   // experts per thread
+  static constexpr int TM = 4;         // tokens per thread
+  static constexpr int LDL = NE + 1;   // logits row stride in shared memory
+  static constexpr size_t kStage = size_t(kBK) * kBM * 4 + size_t(kBK) * NE * 4;
+  static constexpr size_t kGemmSmem = 2 * kStage;
+  static constexpr size_t kLogitSmem = size_t(kBM) * LDL * 4;
   static constexpr size_t kSmem = (kGemmSmem > kLogitSmem ? kGemmSmem : kLogitSmem) + NE * 4;
 };
 
@@ -34,8 +37,10 @@ __global__ void zero_i32_kernel(int32_t *p, int n) {
   for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < n; i += gridDim.x * blockDim.x) p[i] = 0;
 }
 
-// One CTA: BM tokens x all experts. Logits by FFMA in fp32 (x converted from
-// bf16 exactly), then one warp per token runs k rounds of a warp arg-max.
+// One CTA: 64 tokens x all experts. Logits by FFMA in fp32 (x converted from
+// bf16 exactly) with the next k-chunk prefetched into registers while the
+// current one is multiplied; then one warp per token runs k rounds of a warp
+// arg-max over the logits row.
 template <int NE>
 __global__ void __launch_bounds__(kRouteThreads) route_kernel(
     const uint16_t *__restrict__ x, const float *__restrict__ w_router,
@@ -43,65 +48,82 @@ __global__ void __launch_bounds__(kRouteThreads) route_kernel(
     int k, const float *__restrict__ logits_in, float *__restrict__ logits_out,
     int32_t *__restrict__ topk_idx, float *__restrict__ topk_gate, int32_t *__restrict__ counts) {
   using S = RouteShape<NE>;
-  constexpr int TM = S::TM, TN = S::TN, BM = S::BM, LDL = S::LDL;
+  constexpr int TM = S::TM, TN = S::TN, LDL = S::LDL, BM = kBM;
+  constexpr int WPT = kBK * NE / kRouteThreads;  // W elements each thread stages per chunk
   extern __shared__ __align__(16) float smem[];
-  float *Xs = smem;                 // [kBK][BM]
-  float *Ws = smem + kBK * BM;      // [kBK][NE]
-  float *Ls = smem;                 // [BM][LDL] (reuses the GEMM buffers)
+  float *Ls = smem;  // [BM][LDL] (reuses the staging buffers)
   int *hist = reinterpret_cast<int *>(
       smem + (S::kGemmSmem > S::kLogitSmem ? S::kGemmSmem : S::kLogitSmem) / 4);
 
   const int tid = threadIdx.x;
-  const int tx = tid & 31, ty = tid >> 5;
   const int t0 = blockIdx.x * BM;
   for (int e = tid; e < NE; e += kRouteThreads) hist[e] = 0;
 
   if (logits_in == nullptr) {
+    const int tx = tid & 15, ty = tid >> 4;
     float acc[TM][TN];
 #pragma unroll
     for (int i = 0; i < TM; ++i)
 #pragma unroll
       for (int j = 0; j < TN; ++j) acc[i][j] = 0.f;
-
-    for (int k0 = 0; k0 < d; k0 += kBK) {
-      // x tile: BM rows x kBK columns, 8 bf16 per 16-byte load, stored transposed.
-      for (int v = tid; v < BM * (kBK / 8); v += kRouteThreads) {
-        const int r = v / (kBK / 8), c = (v % (kBK / 8)) * 8;
-        float f[8];
-        if (t0 + r < T && k0 + c < d) {
-          unpack8(ldg_nc_v4(x + size_t(t0 + r) * d + k0 + c), f);
+    // register staging of one chunk: x (threads 0..127: one row, 8 columns) and W
+    float xr[8];
+    float wr[WPT];
+    const int xrow = tid >> 1, xcol = (tid & 1) * 8;
+    auto load_chunk = [&](int k0) {
+      if (tid < BM * kBK / 8) {
+        if (t0 + xrow < T && k0 + xcol < d) {
+          unpack8(ldg_nc_v4(x + size_t(t0 + xrow) * d + k0 + xcol), xr);
         } else {
 #pragma unroll
-          for (int q = 0; q < 8; ++q) f[q] = 0.f;
+          for (int q = 0; q < 8; ++q) xr[q] = 0.f;
         }
-#pragma unroll
-        for (int q = 0; q < 8; ++q) Xs[(c + q) * BM + r] = f[q];
       }
-      for (int v = tid; v < kBK * NE; v += kRouteThreads) {
+#pragma unroll
+      for (int i = 0; i < WPT; ++i) {
+        const int v = tid + i * kRouteThreads;
         const int kk = v / NE, e = v % NE;
-        Ws[v] = (e < E && k0 + kk < d) ? __ldg(w_router + size_t(k0 + kk) * E + e) : 0.f;
+        wr[i] = (e < E && k0 + kk < d) ? __ldg(w_router + size_t(k0 + kk) * E + e) : 0.f;
       }
-      __syncthreads();
-#pragma unroll 4
+    };
+    auto store_chunk = [&](int buf) {
+      float *Xs = smem + buf * (S::kStage / 4);  // [kBK][BM]
+      float *Ws = Xs + kBK * BM;                 // [kBK][NE]
+      if (tid < BM * kBK / 8) {
+#pragma unroll
+        for (int q = 0; q < 8; ++q) Xs[(xcol + q) * BM + xrow] = xr[q];
+      }
+#pragma unroll
+      for (int i = 0; i < WPT; ++i) Ws[tid + i * kRouteThreads] = wr[i];
+    };
+    const int nchunks = (d + kBK - 1) / kBK;
+    load_chunk(0);
+    store_chunk(0);
+    __syncthreads();
+    for (int ch = 0; ch < nchunks; ++ch) {
+      if (ch + 1 < nchunks) load_chunk((ch + 1) * kBK);
+      const float *Xs = smem + (ch & 1) * (S::kStage / 4);
+      const float *Ws = Xs + kBK * BM;
+#pragma unroll
       for (int kk = 0; kk < kBK; ++kk) {
-        float xv[TM], wv[TN];
+        const float4 xv = *reinterpret_cast<const float4 *>(&Xs[kk * BM + ty * TM]);
+        const float xs[4] = {xv.x, xv.y, xv.z, xv.w};
 #pragma unroll
-        for (int i = 0; i < TM; i += 4) {
-          const float4 q = *reinterpret_cast<const float4 *>(&Xs[kk * BM + ty * TM + i]);
-          xv[i] = q.x; xv[i + 1] = q.y; xv[i + 2] = q.z; xv[i + 3] = q.w;
+        for (int j4 = 0; j4 < NE / 64; ++j4) {
+          const float4 wv = *reinterpret_cast<const float4 *>(&Ws[kk * NE + j4 * 64 + tx * 4]);
+          const float ws[4] = {wv.x, wv.y, wv.z, wv.w};
+#pragma unroll
+          for (int i = 0; i < TM; ++i)
+#pragma unroll
+            for (int q = 0; q < 4; ++q) acc[i][j4 * 4 + q] = fmaf(xs[i], ws[q], acc[i][j4 * 4 + q]);
         }
-#pragma unroll
-        for (int j = 0; j < TN; ++j) wv[j] = Ws[kk * NE + tx + 32 * j];
-#pragma unroll
-        for (int i = 0; i < TM; ++i)
-#pragma unroll
-          for (int j = 0; j < TN; ++j) acc[i][j] = fmaf(xv[i], wv[j], acc[i][j]);
       }
+      if (ch + 1 < nchunks) store_chunk((ch + 1) & 1);
       __syncthreads();
     }
 #pragma unroll
     for (int j = 0; j < TN; ++j) {
-      const int e = tx + 32 * j;
+      const int e = (j >> 2) * 64 + tx * 4 + (j & 3);
       const float b = (bias != nullptr && e < E) ? bias[e] : 0.f;
 #pragma unroll
       for (int i = 0; i < TM; ++i) Ls[(ty * TM + i) * LDL + e] = acc[i][j] + b;
@@ -126,14 +148,16 @@ __global__ void __launch_bounds__(kRouteThreads) route_kernel(
     }
   }
 
-  // Top-k per token: warp ty handles tokens ty, ty+8, ...
+  // Top-k per token: warp w handles tokens w, w+8, ...
+  const int tx = tid & 31, ty = tid >> 5;
   for (int m = ty; m < BM; m += 8) {
     const int t = t0 + m;
     if (t >= T) break;
-    float v[TN];
+    constexpr int TK = NE / 32;  // logits per lane
+    float v[TK];
     unsigned taken = 0;
 #pragma unroll
-    for (int j = 0; j < TN; ++j) v[j] = Ls[m * LDL + tx + 32 * j];
+    for (int j = 0; j < TK; ++j) v[j] = Ls[m * LDL + tx + 32 * j];
     float sel_v[8];
     int sel_e[8];
 #pragma unroll
@@ -142,7 +166,7 @@ __global__ void __launch_bounds__(kRouteThreads) route_kernel(
       float bv = -INFINITY;
       int be = 0x7fffffff;
 #pragma unroll
-      for (int j = 0; j < TN; ++j) {
+      for (int j = 0; j < TK; ++j) {
         const int e = tx + 32 * j;
         if (e < E && !((taken >> j) & 1u) && better(v[j], e, bv, be)) { bv = v[j]; be = e; }
       }
@@ -163,7 +187,11 @@ __global__ void __launch_bounds__(kRouteThreads) route_kernel(
     for (int s = 0; s < 8; ++s) {
       if (s < k) { ex[s] = expf(sel_v[s] - zmax); den += ex[s]; }
     }
-    if (tx == 0 && sel_v[k - 1] == -INFINITY) dev_flag(&g_dev_err, MOE_DEV_TOO_FEW_LIVE);
+    bool too_few = false;
+#pragma unroll
+    for (int s = 0; s < 8; ++s)
+      if (s < k && sel_v[s] == -INFINITY) too_few = true;
+    if (tx == 0 && too_few) dev_flag(&g_dev_err, MOE_DEV_TOO_FEW_LIVE);
 #pragma unroll
     for (int s = 0; s < 8; ++s) {
       if (s < k && tx == s) {
@@ -285,7 +313,7 @@ int launch_route(const uint16_t *x, const float *w, const float *b, const uint8_
     if (e != cudaSuccess) return moe::cuda_status(e, "moe_route: set smem attribute");
     attr_set = true;
   }
-  const int grid = (T + S::BM - 1) / S::BM;
+  const int grid = (T + kBM - 1) / kBM;
   MOE_LAUNCH("route", s, route_kernel<NE><<<grid, kRouteThreads, S::kSmem, s>>>(x, w, b, mask, T, d, E, k, lin, lout,
                                                         idx, gate, counts));
   return moe::launch_status("moe_route: launch");

@@ -144,6 +144,45 @@ int laep_prune_mask(const int32_t *counts_host, int E, int64_t S, int k, double 
                     double beta, int prune_count, uint8_t *active_mask_host, int *n_pruned);
 
 /*
+ * laep_layer_alpha - layer-adaptive alpha (Sec. 3.4.3; Table 5 caption): the
+ * first and the last floor(L/6) layers use alpha_edge (0.2 in the paper), the
+ * other layers alpha_middle (0.4). HOST call; returns alpha for `layer`.
+ */
+double laep_layer_alpha(int L, int layer, double alpha_edge, double alpha_middle);
+
+/*
+ * laep_prune_layers - Algorithm 1 (Expert Pruning) over a recorded history.
+ * Step 1's ETN[ITER, L, E] is etn_host (row-major, e.g. filled by
+ * moe_load_stats into slot (iter*L + layer)*E). Step 2: for every iteration and
+ * layer, experts are visited in ascending load order (ties: lower id) with a
+ * running load sum that restarts per (iteration, layer); an expert is flagged
+ * when the sum is < S*k*beta and its load is < S*k*alpha[layer]/E; Exp_dis
+ * counts the flags of a layer and Marker those of each expert. Step 3: a layer
+ * prunes N = the mean flagged count over the iterations (rounded half up) of
+ * its experts, in descending Marker order (ties: lower total load, then lower
+ * id), only experts flagged at least once, and keeps at least k.
+ * HOST call. alpha_host [L]; mask_host [L, E] (out: 1 keep, 0 pruned);
+ * n_pruned_host [L] (out, may be NULL). With ITER = 1 it equals
+ * laep_prune_mask's alpha/beta rule layer by layer.
+ */
+int laep_prune_layers(const int32_t *etn_host, int iters, int L, int E, int64_t S, int k,
+                      const double *alpha_host, double beta, uint8_t *mask_host,
+                      int32_t *n_pruned_host);
+
+/*
+ * laep_rearrange - Algorithm 2 (Expert Rearranging): experts taken in
+ * descending load order (ties: lower id) each go to the group with the
+ * smallest load sum that still has room (ties: lower group; a full group
+ * leaves the choice); capacity n/n_groups, rounded up when it does not divide.
+ * HOST call. load_host [n]; order_host [n] (out: expert ids group after
+ * group); group_of_host [n] and group_load_host [n_groups] (out, may be NULL).
+ * In this library the same heaviest-first rule orders the weight-gradient
+ * tiles of the grouped GEMM.
+ */
+int laep_rearrange(const int64_t *load_host, int n, int n_groups, int32_t *order_host,
+                   int32_t *group_of_host, int64_t *group_load_host);
+
+/*
  * moe_permute - dispatch: token rows into contiguous per-expert groups
  * (the data movement of expert-parallel dispatch, Sec. 3.3, on one GPU).
  * Stable counting sort of the A assignments by (expert, token, slot), then

@@ -25,6 +25,18 @@ its reason in the design notes):
   R8  count mode: prune the P smallest counts (Eq. 2's largest=False top-K).
   R9  at least k experts are always kept (the paper does not say; routing
       needs k live experts).
+  R11 Algorithm 1 over ITER iterations: the running load sum restarts for every
+      (iteration, layer); Marker counts how often each expert (by id, not by
+      sorted position) is flagged; the number pruned per layer is the mean
+      flagged count over the iterations, rounded half up; experts are pruned in
+      descending Marker order, ties to the lower total load over the
+      iterations, then the lower id; only experts flagged at least once.
+  R12 Layer-adaptive alpha: the first and the last floor(L/6) layers use the
+      edge value (0.2 in the paper), the others the middle value (0.4).
+  R13 Algorithm 2: ties in the descending sort go to the lower expert id, ties
+      in argmin to the lower group; when the expert count is not a multiple of
+      the group count the per-group capacity is rounded up (the listing would
+      otherwise never place the remainder).
 """
 from __future__ import annotations
 
@@ -372,3 +384,87 @@ def expert_weight_grad_columns(e, feats, x_rows, dy_rows, gates_rows, w_gate_up,
         dwg[i] = (dh * b * silu_grad(a)) @ X
         dwu[i] = (dh * silu(a)) @ X
     return dwd, dwg, dwu
+
+
+# ----------------------------------------------------------------------------
+# Algorithm 1 over iterations and layers; the layer-adaptive alpha schedule
+# ----------------------------------------------------------------------------
+
+
+def layer_alpha(L, layer, alpha_edge=0.2, alpha_middle=0.4):
+    """alpha of one layer (reading R12; Sec. 3.4.3 and the Table 5 caption)."""
+    n6 = L // 6
+    return alpha_edge if (layer < n6 or layer >= L - n6) else alpha_middle
+
+
+def prune_layers(etn, S, k, alphas, beta):
+    """Algorithm 1 with the ETN history of ITER iterations and L layers.
+
+    etn: [ITER, L, E] per-expert token counts; alphas: [L]; returns
+    (mask uint8 [L, E], n_pruned [L]) (reading R11).
+    """
+    etn = np.asarray(etn, np.int64)
+    ITER, L, E = etn.shape
+    marker = np.zeros((L, E), np.int64)
+    exp_dis = np.zeros(L, np.int64)
+    for it in range(ITER):
+        for layer in range(L):
+            counts = etn[it, layer]
+            beta_thr = float(S) * float(k) * float(beta)
+            alpha_thr = float(S) * float(k) * float(alphas[layer]) / float(E)
+            order = np.argsort(counts, kind="stable")
+            running = 0
+            for e in order:
+                running += int(counts[e])
+                if running < beta_thr and int(counts[e]) < alpha_thr:
+                    exp_dis[layer] += 1
+                    marker[layer, e] += 1
+    mask = np.ones((L, E), np.uint8)
+    n_pruned = np.zeros(L, np.int64)
+    total = etn.sum(axis=0)  # [L, E] load summed over the iterations
+    for layer in range(L):
+        n = (2 * int(exp_dis[layer]) + ITER) // (2 * ITER)
+        n = min(n, E - k, int(np.count_nonzero(marker[layer])))
+        ranked = sorted(range(E), key=lambda e: (-marker[layer, e], total[layer, e], e))
+        for e in ranked[:n]:
+            mask[layer, e] = 0
+        n_pruned[layer] = n
+    return mask, n_pruned
+
+
+# ----------------------------------------------------------------------------
+# Algorithm 2: expert rearrangement across n_g groups (devices)
+# ----------------------------------------------------------------------------
+
+
+def rearrange(loads, n_groups):
+    """Greedy placement of experts into n_groups groups of equal size.
+
+    Experts are taken in descending load order; each goes to the group with the
+    smallest load sum that still has room (a full group is taken out of the
+    argmin). Returns (order [n] = experts group by group, group_of [n],
+    group_load [n_groups]) (reading R13).
+    """
+    loads = np.asarray(loads, np.int64)
+    n = loads.shape[0]
+    cap = -(-n // n_groups)  # == n // n_groups when n divides evenly
+    order_desc = sorted(range(n), key=lambda e: (-loads[e], e))
+    members = [[] for _ in range(n_groups)]
+    sums = [0] * n_groups
+    full = [False] * n_groups
+    for e in order_desc:
+        while True:
+            g = min((g for g in range(n_groups)),
+                    key=lambda g: (float("inf") if full[g] else sums[g], g))
+            if len(members[g]) < cap:
+                members[g].append(e)
+                sums[g] += int(loads[e])
+                break
+            full[g] = True
+    order = np.array([e for g in range(n_groups) for e in members[g]], np.int64)
+    group_of = np.empty(n, np.int64)
+    for g in range(n_groups):
+        for e in members[g]:
+            group_of[e] = g
+    return order, group_of, np.array(sums, np.int64)
+

@@ -46,6 +46,9 @@ _SIGS = {
     "moe_route": (I, [P, P, P, P, I, I, I, I, P, P, P, P, P, P]),
     "moe_load_stats": (I, [P, I, I, I, P, I, P]),
     "laep_prune_mask": (I, [P, I, I64, I, D, D, I, P, P]),
+    "laep_layer_alpha": (D, [I, I, D, D]),
+    "laep_prune_layers": (I, [P, I, I, I, I64, I, P, D, P, P]),
+    "laep_rearrange": (I, [P, I, I, P, P, P]),
     "moe_permute": (I, [P, P, P, I, I, I, I, I64, P, P, P, P, P, SZ, P]),
     "moe_permute_noalloc": (I, [P, P, P, I, I, I, I, I64, P, P, P, P, P]),
     "moe_grouped_ffn_fwd": (I, [P, P, I, I, I, I64, P, P, P, P, P, P, SZ, P]),
@@ -163,6 +166,37 @@ def laep_prune_mask(counts, S, k, alpha=0.0, beta=0.0, prune_count=-1):
         ctypes.cast(c, P), E, int(S), int(k), float(alpha), float(beta), int(prune_count),
         ctypes.cast(m, P), ctypes.byref(n)))
     return list(m), n.value
+
+
+def laep_layer_alpha(L, layer, alpha_edge=0.2, alpha_middle=0.4):
+    return float(load().laep_layer_alpha(L, layer, alpha_edge, alpha_middle))
+
+
+def laep_prune_layers(etn, S, k, alphas, beta):
+    """Host call. etn: int array [ITER, L, E]; alphas: [L]. Returns (mask [L,E], n_pruned [L])."""
+    import numpy as np
+    etn = np.ascontiguousarray(etn, dtype=np.int32)
+    iters, L, E = etn.shape
+    a = np.ascontiguousarray(alphas, dtype=np.float64)
+    mask = np.empty((L, E), np.uint8)
+    n = np.empty(L, np.int32)
+    _check("laep_prune_layers", load().laep_prune_layers(
+        etn.ctypes.data, iters, L, E, int(S), int(k), a.ctypes.data, float(beta),
+        mask.ctypes.data, n.ctypes.data))
+    return mask, n
+
+
+def laep_rearrange(loads, n_groups):
+    """Host call. Returns (order [n], group_of [n], group_load [n_groups])."""
+    import numpy as np
+    ld = np.ascontiguousarray(loads, dtype=np.int64)
+    n = ld.shape[0]
+    order = np.empty(n, np.int32)
+    group_of = np.empty(n, np.int32)
+    gl = np.empty(n_groups, np.int64)
+    _check("laep_rearrange", load().laep_rearrange(ld.ctypes.data, n, n_groups, order.ctypes.data,
+                                                   group_of.ctypes.data, gl.ctypes.data))
+    return order, group_of, gl
 
 
 def moe_permute(x, topk_idx, counts, T, d, E, k, rows_cap, group_offsets, group_counts,

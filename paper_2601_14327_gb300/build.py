@@ -17,7 +17,7 @@ ROOT = os.path.dirname(HERE)
 CSRC = os.path.join(HERE, "csrc")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(BUILD, "libmoe_laep.so")
-SOURCES = ["api.cu", "route.cu", "permute.cu", "gemm.cu"]
+SOURCES = ["api.cu", "laep.cu", "route.cu", "permute.cu", "gemm.cu"]
 HEADERS = ["common.cuh", "tc_ptx.cuh"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 

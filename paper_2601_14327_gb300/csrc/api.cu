@@ -1,4 +1,4 @@
-// Host-side entry points: errors, sizes, and the LAEP pruning decision.
+// Host-side entry points: errors, sizes, workspace layout, kernel timing.
 #include <stdarg.h>
 #include <stdio.h>
 
@@ -190,45 +190,6 @@ int moe_timing_read(char *buf, size_t buf_len, int reset) {
     }
     t.recs.clear();
   }
-  return MOE_OK;
-}
-
-// LAEP pruning decision (Sec. 3.2 Eq. 1-2, Algorithm 1 with one histogram).
-int laep_prune_mask(const int32_t *counts_host, int E, int64_t S, int k, double alpha,
-                    double beta, int prune_count, uint8_t *active_mask_host, int *n_pruned) {
-  if (!counts_host || !active_mask_host)
-    return moe::set_error(MOE_ERR_ARG, "laep_prune_mask: null pointer");
-  if (E <= 0 || k <= 0 || k > E || S < 0)
-    return moe::set_error(MOE_ERR_ARG, "laep_prune_mask: bad sizes E=%d k=%d S=%lld", E, k,
-                          (long long)S);
-  for (int e = 0; e < E; ++e)
-    if (counts_host[e] < 0) return moe::set_error(MOE_ERR_ARG, "laep_prune_mask: negative count");
-  // Ascending load order; equal loads keep index order (lower index first).
-  std::vector<int> order(E);
-  std::iota(order.begin(), order.end(), 0);
-  std::stable_sort(order.begin(), order.end(),
-                   [&](int a, int b) { return counts_host[a] < counts_host[b]; });
-  for (int e = 0; e < E; ++e) active_mask_host[e] = 1;
-  const int max_prune = E - k;  // routing needs k live experts
-  int pruned = 0;
-  if (prune_count >= 0) {
-    pruned = std::min(prune_count, max_prune);
-    for (int r = 0; r < pruned; ++r) active_mask_host[order[r]] = 0;
-  } else {
-    // Thresholds of Algorithm 1: cumulative < S*topK*beta, individual < S*topK*alpha/E.
-    const double beta_thr = double(S) * double(k) * beta;
-    const double alpha_thr = double(S) * double(k) * alpha / double(E);
-    int64_t running = 0;
-    for (int r = 0; r < E; ++r) {
-      const int e = order[r];
-      running += counts_host[e];
-      if (double(running) < beta_thr && double(counts_host[e]) < alpha_thr && pruned < max_prune) {
-        active_mask_host[e] = 0;
-        ++pruned;
-      }
-    }
-  }
-  if (n_pruned) *n_pruned = pruned;
   return MOE_OK;
 }
 

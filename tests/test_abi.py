@@ -90,3 +90,41 @@ def test_argument_validation_without_launch(lib):
     assert e.value.status == -6
     with pytest.raises(L.MoEError):
         L.laep_prune_mask([1, 2, 3], 2, 4)  # k > E
+
+
+def test_laep_algorithms_golden(lib):
+    g = json.load(open(os.path.join(GOLDEN, "laep_algorithms_cases.json")))
+    for c in g["prune_layers"]:
+        mask, n = L.laep_prune_layers(np.array(c["etn"]), c["S"], c["k"], c["alphas"], c["beta"])
+        assert mask.tolist() == c["mask"] and n.tolist() == c["n_pruned"], c["name"]
+    for c in g["layer_alpha"]:
+        got = [L.laep_layer_alpha(c["L"], l) for l in range(c["L"])]
+        if "alpha" in c:
+            assert got == c["alpha"]
+        else:
+            assert sum(a == 0.2 for a in got) == c["edge_layers"]
+    for c in g["rearrange"]:
+        order, group_of, gl = L.laep_rearrange(c["loads"], c["n_groups"])
+        assert order.tolist() == c["order"] and gl.tolist() == c["group_load"], c["name"]
+
+
+def test_laep_algorithms_match_oracle_random(lib):
+    rng = np.random.default_rng(11)
+    for _ in range(150):
+        E = int(rng.integers(2, 257))
+        k = int(rng.integers(1, min(E, 8) + 1))
+        iters, nl = int(rng.integers(1, 5)), int(rng.integers(1, 7))
+        S = int(rng.integers(1, 3000))
+        etn = np.stack([[rng.multinomial(S * k, rng.dirichlet(np.full(E, 0.25)))
+                         for _ in range(nl)] for _ in range(iters)])
+        alphas = [O.layer_alpha(nl, l, float(rng.uniform(0, 1)), float(rng.uniform(0, 1.5)))
+                  for l in range(nl)]
+        beta = float(rng.uniform(0, 0.4))
+        m, n = L.laep_prune_layers(etn, S, k, alphas, beta)
+        om, on = O.prune_layers(etn, S, k, alphas, beta)
+        assert (m == om).all() and (n == on).all()
+        ng = int(rng.integers(1, 9))
+        loads = rng.integers(0, 10 ** 6, size=ng * int(rng.integers(1, 40)) + int(rng.integers(0, ng)))
+        order, group_of, gl = L.laep_rearrange(loads, ng)
+        oo, og, ogl = O.rearrange(loads, ng)
+        assert (order == oo).all() and (group_of == og).all() and (gl == ogl).all()

@@ -240,3 +240,28 @@ def test_tiny_workload_end_to_end_gpu_logits():
         assert_close("dw_gate_up", to_np(b.dw_gate_up), ref["dw_gate_up"])
         assert_close("dw_down", to_np(b.dw_down), ref["dw_down"])
         assert_close("dw_router", b.dw_router.cpu().numpy(), ref["dw_router"])
+
+
+def test_etn_history_recorded_on_device_drives_algorithm_1():
+    """ETN[ITER, L, E] filled slot by slot by moe_load_stats from routings made
+    on the GPU, then the host-side Algorithm 1 vs the oracle on the oracle's
+    own routing of the same logits."""
+    ITER, NL, T, E, k = 3, 4, 700, 32, 4
+    rng = np.random.default_rng(21)
+    etn = torch.zeros(ITER, NL, E, dtype=torch.int32, device="cuda")
+    etn_ref = np.zeros((ITER, NL, E), np.int64)
+    for it in range(ITER):
+        for layer in range(NL):
+            skew = np.log(rng.dirichlet(np.full(E, 0.3)) + 1e-9).astype(np.float32)
+            z = (rng.standard_normal((T, E)).astype(np.float32) + skew[None, :])
+            idx, _, _, _ = _route_only(T, E, k, z)
+            L.moe_load_stats(torch.from_numpy(idx).cuda(), T, k, E, etn[it, layer])
+            oidx, _ = O.route_topk(z, k)
+            etn_ref[it, layer] = O.expert_counts(oidx, E)
+    torch.cuda.synchronize()
+    got = etn.cpu().numpy()
+    assert (got == etn_ref).all()
+    alphas = [O.layer_alpha(NL, l, 0.2, 0.4) for l in range(NL)]
+    m, n = L.laep_prune_layers(got, T, k, alphas, 0.1)
+    om, on = O.prune_layers(etn_ref, T, k, alphas, 0.1)
+    assert (m == om).all() and (n == on).all()

@@ -284,3 +284,67 @@ def test_prune_alpha_beta_brute_force_prefix():
         assert (mask == want).all() and n == pruned
         kept = [order.index(e) for e in range(E) if mask[e] == 0]
         assert sorted(kept) == list(range(len(kept)))  # a prefix of the order
+
+
+# ---------------------------------- Algorithm 1 over iterations, Algorithm 2 ---
+
+def _algos():
+    with open(os.path.join(GOLDEN, "laep_algorithms_cases.json")) as f:
+        return json.load(f)
+
+
+def test_prune_layers_golden():
+    for c in _algos()["prune_layers"]:
+        mask, n = O.prune_layers(c["etn"], c["S"], c["k"], c["alphas"], c["beta"])
+        assert mask.tolist() == c["mask"] and n.tolist() == c["n_pruned"], c["name"]
+
+
+def test_prune_layers_single_iteration_is_single_histogram_rule():
+    rng = np.random.default_rng(4)
+    for _ in range(200):
+        E = int(rng.integers(2, 20))
+        k = int(rng.integers(1, E + 1))
+        L = int(rng.integers(1, 4))
+        S = int(rng.integers(1, 80))
+        etn = np.stack([rng.multinomial(S * k, rng.dirichlet(np.full(E, 0.3))) for _ in range(L)])
+        alphas = rng.uniform(0, 2, size=L)
+        beta = float(rng.uniform(0, 0.6))
+        mask, n = O.prune_layers(etn[None], S, k, alphas, beta)
+        for layer in range(L):
+            m1, n1 = O.prune_mask_alpha_beta(etn[layer], S, k, alphas[layer], beta)
+            assert (mask[layer] == m1).all() and n[layer] == n1
+
+
+def test_prune_layers_identical_iterations_repeat_the_decision():
+    rng = np.random.default_rng(8)
+    E, k, S = 16, 2, 500
+    etn1 = rng.multinomial(S * k, rng.dirichlet(np.full(E, 0.2)))
+    m1, n1 = O.prune_mask_alpha_beta(etn1, S, k, 0.4, 0.1)
+    mask, n = O.prune_layers(np.tile(etn1, (5, 1, 1)), S, k, [0.4], 0.1)
+    assert (mask[0] == m1).all() and n[0] == n1
+
+
+def test_layer_alpha_golden():
+    for c in _algos()["layer_alpha"]:
+        got = [O.layer_alpha(c["L"], l) for l in range(c["L"])]
+        if "alpha" in c:
+            assert got == c["alpha"]
+        else:
+            assert sum(a == 0.2 for a in got) == c["edge_layers"]
+
+
+def test_rearrange_golden_and_invariants():
+    for c in _algos()["rearrange"]:
+        order, group_of, gl = O.rearrange(c["loads"], c["n_groups"])
+        assert order.tolist() == c["order"] and gl.tolist() == c["group_load"], c["name"]
+    rng = np.random.default_rng(2)
+    for _ in range(200):
+        ng = int(rng.integers(1, 9))
+        n = ng * int(rng.integers(1, 9))
+        loads = rng.integers(0, 1000, size=n)
+        order, group_of, gl = O.rearrange(loads, ng)
+        assert sorted(order.tolist()) == list(range(n))
+        assert all((group_of == g).sum() == n // ng for g in range(ng))
+        assert all(gl[g] == loads[group_of == g].sum() for g in range(ng))
+        # greedy balance: no group exceeds the mean by more than the largest load
+        assert gl.max() <= loads.sum() / ng + loads.max()

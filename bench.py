@@ -203,14 +203,20 @@ class Workload:
 # ------------------------------------------------------------------ the arms
 
 def dist_setup(n_gpus):
+    """One process per GPU (torchrun sets RANK/LOCAL_RANK/WORLD_SIZE). Each rank runs
+    an independent replica of the layer step: the path has no exchange, so the only
+    collectives are the barrier and the max over ranks of the timed region."""
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
     local = int(os.environ.get("LOCAL_RANK", "0"))
     if world > 1:
         import torch.distributed as dist
-        torch.cuda.set_device(local)
-        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
-    else:
+        if torch.cuda.is_available():
+            torch.cuda.set_device(local)
+            dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+        else:
+            dist.init_process_group("gloo")
+    elif torch.cuda.is_available():
         torch.cuda.set_device(0)
     return world, rank, local
 
@@ -222,12 +228,19 @@ def barrier(world):
 
 
 def max_over_ranks(x, world):
+    """Largest value of x over the ranks (the slowest replica sets the job time)."""
     if world > 1:
         import torch.distributed as dist
-        t = torch.tensor([x], dtype=torch.float64, device="cuda")
+        dev = "cuda" if dist.get_backend() == "nccl" else "cpu"
+        t = torch.tensor([x], dtype=torch.float64, device=dev)
         dist.all_reduce(t, op=dist.ReduceOp.MAX)
         return float(t.item())
     return x
+
+
+def replica_throughput(world, tokens_per_rank, steps, ms_max):
+    """Whole-job tokens/s of `world` replicas, timed by the slowest one."""
+    return world * tokens_per_rank * steps / (ms_max / 1e3)
 
 
 def oracle_sample(wl_inputs_host, mask_host, k, n_tok):
@@ -326,7 +339,7 @@ def laep_comparison(args, world, local, pruned_tps, wl_pruned):
     for _ in range(args.warmup):
         wl_u.step()
     ms_u, _, _ = timed_steps(wl_u, steps, world, local)
-    tps_u = world * wl_u.shape.T * steps / (ms_u / 1e3)
+    tps_u = replica_throughput(world, wl_u.shape.T, steps, ms_u)
     unpruned_params = 3 * wl_u.shape.E * wl_u.shape.d * wl_u.shape.F
     del wl_u
     torch.cuda.empty_cache()
@@ -355,7 +368,7 @@ def run_ours(args):
     stream = torch.cuda.current_stream()
     ms_total, per_kernel, clk = timed_steps(wl, args.steps, world, local)
     ms_step = ms_total / args.steps
-    tokens_per_s = world * s.T * args.steps / (ms_total / 1e3)
+    tokens_per_s = replica_throughput(world, s.T, args.steps, ms_total)
     launches = sum(n for n, _ in per_kernel.values())
 
     # dominant kernel and its roofline
@@ -401,7 +414,8 @@ def run_ours(args):
         barrier(world)
         e_ms = max_over_ranks(ev0.elapsed_time(ev1), world)
         nbytes = x_h.numel() * 2
-        e2e = {"value": round(world * s.T * args.steps / (e_ms / 1e3), 1), "unit": "tokens/s",
+        e2e = {"value": round(replica_throughput(world, s.T, args.steps, e_ms), 1),
+               "unit": "tokens/s",
                "h2d_bytes_per_step": 2 * nbytes, "d2h_bytes_per_step": 2 * nbytes}
 
     cpu = None

@@ -9,8 +9,8 @@
 // the expert loads, and empty groups produce no tile. In the weight-gradient
 // GEMMs (reduction over a group's rows, so tile cost ~ group size) the
 // experts are ordered heaviest first, the longest-processing-time order that
-// Algorithm 2's greedy balancing also uses (experts without rows go first: their
-// tiles are zero stores that overlap the first MMAs).
+// Algorithm 2's greedy balancing also uses; experts without rows come last (their
+// tiles are zero stores only).
 //
 // Six GEMM shapes share one kernel template:
 //   kGateUp      [A|B] = X W_gu^T        (A: K-major rows, B: K-major weights)
@@ -245,15 +245,11 @@ __global__ void __launch_bounds__(kThreads, 1)
   __syncthreads();
   if (Tr::WGRAD) {
     for (int e = threadIdx.x; e < E; e += kThreads) {
-      // empty experts first (their zero tiles are stores only and overlap the
-      // first MMAs), then heaviest first; ties keep the expert order
       const int ce = s_goff[e + 1] - s_goff[e];
-      const unsigned ke = ce == 0 ? 0xffffffffu : unsigned(ce);
       int r = 0;
       for (int q = 0; q < E; ++q) {
         const int cq = s_goff[q + 1] - s_goff[q];
-        const unsigned kq = cq == 0 ? 0xffffffffu : unsigned(cq);
-        r += (kq > ke) || (kq == ke && q < e);
+        r += (cq > ce) || (cq == ce && q < e);
       }
       s_order[r] = e;
     }
@@ -519,15 +515,11 @@ __global__ void __launch_bounds__(kThreads, 1)
   __syncthreads();
   if (Tr::WGRAD) {
     for (int e = threadIdx.x; e < E; e += kThreads) {
-      // empty experts first (their zero tiles are stores only and overlap the
-      // first MMAs), then heaviest first; ties keep the expert order
       const int ce = s_goff[e + 1] - s_goff[e];
-      const unsigned ke = ce == 0 ? 0xffffffffu : unsigned(ce);
       int r = 0;
       for (int q = 0; q < E; ++q) {
         const int cq = s_goff[q + 1] - s_goff[q];
-        const unsigned kq = cq == 0 ? 0xffffffffu : unsigned(cq);
-        r += (kq > ke) || (kq == ke && q < e);
+        r += (cq > ce) || (cq == ce && q < e);
       }
       s_order[r] = e;
     }
@@ -741,15 +733,17 @@ int make_map(CUtensorMap *m, const void *base, uint64_t rows, uint64_t cols, uin
   if (r != CUDA_SUCCESS) return moe::set_error(MOE_ERR_CUDA, "tensor map for %s: CUresult %d", what, int(r));
   return MOE_OK;
 }
-// The CTA-pair kernel is the default; MOE_GEMM_1SM=1 selects the one-SM kernel
-// (kept for A/B measurements).
-bool use_pair() {
+// CTA-pair kernel for every shape except dH (its epilogue reads and writes two
+// [rows, F] tensors, so it is epilogue-bound and the one-SM kernel with its
+// longer mainloop per tile is faster). MOE_GEMM_1SM=1 selects the one-SM kernel
+// everywhere (for A/B measurements).
+template <int MODE> bool use_pair() {
   static int v = -1;
   if (v < 0) {
     const char *e = getenv("MOE_GEMM_1SM");
     v = (e && e[0] == '1') ? 0 : 1;
   }
-  return v == 1;
+  return v == 1 && MODE != kDgradDown;
 }
 
 template <int MODE, int BN>
@@ -805,7 +799,7 @@ template <int MODE>
 int run_gemm(int N, const void *a_base, uint64_t a_rows, uint64_t a_cols, const void *b_base,
              uint64_t b_rows, uint64_t b_cols, GemmParams p, cudaStream_t s, const char *what) {
   using Tr = Traits<MODE>;
-  const bool pair = use_pair();
+  const bool pair = use_pair<MODE>();
   const int BN = (MODE == kGateUp || N % 256 == 0) ? 256 : 128;
   p.n_tiles = (MODE == kGateUp) ? N / 256 : N / BN;
   CUtensorMap ma, mb;

@@ -13,17 +13,17 @@ MOE_DEV_ERR_DECL
 namespace {
 
 constexpr int kRouteThreads = 256;
-constexpr int kBK = 16;  // reduction chunk of the logit contraction
 constexpr int kBM = 64;  // tokens per CTA
 
 // Padded expert count NE (multiple of 64). 16 x 16 threads: thread (tx, ty) owns
 // tokens ty*4 .. ty*4+3 and experts j*64 + tx*4 + q (j < NE/64, q < 4), so the
 // shared-memory reads of one row of W are contiguous float4s across tx.
 template <int NE> struct RouteShape {
+  static constexpr int BK = NE <= 128 ? 32 : 16;  // reduction chunk (registers stage one)
   static constexpr int TN = NE / 16;   // experts per thread
   static constexpr int TM = 4;         // tokens per thread
   static constexpr int LDL = NE + 1;   // logits row stride in shared memory
-  static constexpr size_t kStage = size_t(kBK) * kBM * 4 + size_t(kBK) * NE * 4;
+  static constexpr size_t kStage = size_t(BK) * kBM * 4 + size_t(BK) * NE * 4;
   static constexpr size_t kGemmSmem = 2 * kStage;
   static constexpr size_t kLogitSmem = size_t(kBM) * LDL * 4;
   static constexpr size_t kSmem = (kGemmSmem > kLogitSmem ? kGemmSmem : kLogitSmem) + NE * 4;
@@ -48,7 +48,7 @@ __global__ void __launch_bounds__(kRouteThreads) route_kernel(
     int k, const float *__restrict__ logits_in, float *__restrict__ logits_out,
     int32_t *__restrict__ topk_idx, float *__restrict__ topk_gate, int32_t *__restrict__ counts) {
   using S = RouteShape<NE>;
-  constexpr int TM = S::TM, TN = S::TN, LDL = S::LDL, BM = kBM;
+  constexpr int TM = S::TM, TN = S::TN, LDL = S::LDL, BM = kBM, kBK = S::BK;
   constexpr int WPT = kBK * NE / kRouteThreads;  // W elements each thread stages per chunk
   extern __shared__ __align__(16) float smem[];
   float *Ls = smem;  // [BM][LDL] (reuses the staging buffers)
@@ -69,7 +69,8 @@ __global__ void __launch_bounds__(kRouteThreads) route_kernel(
     // register staging of one chunk: x (threads 0..127: one row, 8 columns) and W
     float xr[8];
     float wr[WPT];
-    const int xrow = tid >> 1, xcol = (tid & 1) * 8;
+    constexpr int XSEG = kBK / 8;  // 16-byte segments of x per row and chunk
+    const int xrow = tid / XSEG, xcol = (tid % XSEG) * 8;
     auto load_chunk = [&](int k0) {
       if (tid < BM * kBK / 8) {
         if (t0 + xrow < T && k0 + xcol < d) {

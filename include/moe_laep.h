@@ -232,10 +232,12 @@ int moe_permute_noalloc(const uint16_t *x, const int32_t *topk_idx, const int32_
  *   O_e = H_e * W_down[e]^T
  * bf16 operands, fp32 accumulation in tensor memory, bf16 results.
  * x_perm [rows_cap,d]; group_offsets [E+1]; w_gate_up [E,2F,d] bf16 (rows
- * 0..F-1 gate, F..2F-1 up); w_down [E,d,F] bf16; outputs ab_saved
- * [rows_cap,2F] bf16 (A in columns 0..F-1, B in F..2F-1; kept for the
- * backward), h [rows_cap,F] bf16, out_perm [rows_cap,d] bf16. Only rows below
- * group_offsets[E] are written. Groups of 0 rows cost nothing.
+ * 0..F-1 gate, F..2F-1 up); w_down [E,d,F] bf16; outputs ab_saved (the
+ * [rows, 2F] matrix [A|B], kept for the backward, rows_cap*2F bf16, stored in
+ * 32-row blocks: element (r, c) at ((r/32)*(2F/8) + c/8)*256 + (r%32)*8 + c%8,
+ * so that the 32 rows one warp handles are contiguous), h [rows_cap,F] bf16,
+ * out_perm [rows_cap,d] bf16. Only rows below group_offsets[E] are written.
+ * Groups of 0 rows cost nothing.
  * Limits: d % 128 == 0, F % 128 == 0, all pointers 16-byte aligned.
  */
 int moe_grouped_ffn_fwd(const uint16_t *x_perm, const int32_t *group_offsets, int E, int d,

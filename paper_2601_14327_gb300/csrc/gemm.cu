@@ -12,9 +12,12 @@
 // Algorithm 2's greedy balancing also uses; experts without rows come last (their
 // tiles are zero stores only).
 //
+// Warps: 0 issues TMA loads, 1 owns TMEM and issues the MMAs, 2..9 are the epilogue
+// (two per TMEM lane quarter, each taking half of the tile's columns).
+//
 // Six GEMM shapes share one kernel template:
 //   kGateUp      [A|B] = X W_gu^T        (A: K-major rows, B: K-major weights)
-//                epilogue: H = silu(A)*B, keeps A and B for the backward
+//                epilogue: H = silu(A)*B, keeps A and B (32-row blocked) for the backward
 //   kDown        O = H W_down^T
 //   kDgradDown   dH = dO W_down           (B is MN-major)
 //                epilogue: dA = dH*B*silu'(A), dB = dH*silu(A)
@@ -47,7 +50,8 @@ const char *const kGemmName[] = {"gemm_gate_up",       "gemm_down",
 constexpr int BM = 128;   // tile rows (TMEM lanes)
 constexpr int BK = 64;    // k-block: 64 bf16 = one 128-byte swizzle row
 constexpr int UMMA_K = 16;
-constexpr int kThreads = 192;  // warp 0 TMA, warp 1 MMA + TMEM owner, warps 2-5 epilogue
+constexpr int kEpiWarps = 8;   // two epilogue warps per TMEM lane quarter, each half the columns
+constexpr int kThreads = 64 + 32 * kEpiWarps;  // warp 0 TMA, warp 1 MMA + TMEM owner, epilogue
 constexpr uint64_t kWaitLimitNs = 2000000000ull;
 
 template <int MODE> struct Traits {
@@ -74,7 +78,7 @@ struct GemmParams {
   int m_tiles_w;   // weight-gradient modes: row tiles of one expert's output
   int nkb;         // k-blocks per tile (activation modes)
   uint16_t *out;   // primary output
-  uint16_t *out2;  // kGateUp: pre-activations [rows, 2F]
+  uint16_t *out2;  // kGateUp: pre-activations [A|B] (32-row blocked, see ab_block_index)
   const uint16_t *aux;  // kDgradDown: saved pre-activations [rows, 2F]
 };
 
@@ -101,21 +105,28 @@ __device__ __forceinline__ void store_row_bf16(uint16_t *dst, const uint32_t (&r
 
 __device__ __forceinline__ float silu_f(float a) { return a / (1.f + __expf(-a)); }
 
-// Epilogue of one accumulator tile for the 32 rows this warp owns: reads the fp32
+// Saved pre-activations [A|B] are stored in 32-row blocks: element (r, c) of the
+// [rows, 2F] matrix lives at ((r/32)*(2F/8) + c/8)*256 + (r%32)*8 + c%8, so the
+// 32 rows a warp owns in the epilogue touch 512 contiguous bytes per 8 columns
+// (one coalesced warp access in the forward's store and the backward's load).
+__device__ __forceinline__ size_t ab_block_index(size_t row, int col, int F) {
+  return ((row >> 5) * size_t(2 * F / 8) + size_t(col >> 3)) * 256 + (row & 31) * 8 + (col & 7);
+}
+
+// Epilogue of one accumulator tile for the 32 rows and the column half (`half`) this
+// warp owns: reads the fp32
 // accumulator from tensor memory at `tb` (lane base and column base included) and
 // writes the mode's outputs. `row` = row of this thread in the grouped layout
 // (activation modes), `out_row` = row in the expert's weight-gradient matrix.
 template <int MODE, int BN>
 __device__ __forceinline__ void epilogue_tile(const GemmParams &p, uint32_t tb, size_t row,
-                                              int out_row, int e, int nt) {
+                                              int out_row, int e, int nt, int half) {
   using Tr = Traits<MODE>;
   if (MODE == kGateUp) {
     const int F = p.F;
     uint16_t *hrow = p.out + row * F + nt * 128;
-    uint16_t *arow = p.out2 + row * 2 * F + nt * 128;
-    uint16_t *brow = arow + F;
 #pragma unroll 1
-    for (int c = 0; c < 128; c += 32) {
+    for (int c = half * 64; c < half * 64 + 64; c += 32) {
       uint32_t ra[32], rb[32];
       tc::tmem_ld_32x32b_x32(tb + c, ra);
       tc::tmem_ld_32x32b_x32(tb + 128 + c, rb);
@@ -129,25 +140,24 @@ __device__ __forceinline__ void epilogue_tile(const GemmParams &p, uint32_t tb, 
           fb[i] = __uint_as_float(rb[v * 8 + i]);
           fh[i] = silu_f(fa[i]) * fb[i];
         }
+        const int col = nt * 128 + c + v * 8;
         stg_v4(hrow + c + v * 8, pack8(fh));
-        stg_v4(arow + c + v * 8, pack8(fa));
-        stg_v4(brow + c + v * 8, pack8(fb));
+        stg_v4(p.out2 + ab_block_index(row, col, F), pack8(fa));
+        stg_v4(p.out2 + ab_block_index(row, F + col, F), pack8(fb));
       }
     }
   } else if (MODE == kDgradDown) {
     const int F = p.F;
     const int f0 = nt * BN;
-    const uint16_t *arow = p.aux + row * 2 * F + f0;
-    const uint16_t *brow = arow + F;
     uint16_t *darow = p.out + row * 2 * F + f0;
     uint16_t *dbrow = darow + F;
 #pragma unroll 1
-    for (int c = 0; c < BN; c += 32) {
+    for (int c = half * (BN / 2); c < (half + 1) * (BN / 2); c += 32) {
       uint4 va[4], vb[4];
 #pragma unroll
       for (int v = 0; v < 4; ++v) {
-        va[v] = ldg_nc_v4(arow + c + v * 8);
-        vb[v] = ldg_nc_v4(brow + c + v * 8);
+        va[v] = ldg_nc_v4(p.aux + ab_block_index(row, f0 + c + v * 8, F));
+        vb[v] = ldg_nc_v4(p.aux + ab_block_index(row, F + f0 + c + v * 8, F));
       }
       uint32_t r[32];
       tc::tmem_ld_32x32b_x32(tb + c, r);
@@ -177,7 +187,7 @@ __device__ __forceinline__ void epilogue_tile(const GemmParams &p, uint32_t tb, 
       orow = p.out + row * p.d + nt * BN;
     }
 #pragma unroll 1
-    for (int c = 0; c < BN; c += 32) {
+    for (int c = half * (BN / 2); c < (half + 1) * (BN / 2); c += 32) {
       uint32_t r[32];
       tc::tmem_ld_32x32b_x32(tb + c, r);
       tc::tmem_ld_wait();
@@ -226,7 +236,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     for (int a = 0; a < 2; ++a) {
       tc::mbar_init(tfull_bar(a), 1);
-      tc::mbar_init(tempty_bar(a), 4);
+      tc::mbar_init(tempty_bar(a), kEpiWarps);
     }
     tc::mbar_init(drain_bar, 1);
     tc::fence_mbar_init();
@@ -384,6 +394,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   } else {
     // ===================== epilogue (warps 2..5) =====================
     const int q = warp & 3;  // TMEM lane quarter this warp may access
+    const int half = (warp - 2) / 4;  // column half this warp handles
     const int r_in_tile = q * 32 + lane;
     uint32_t tcount = 0;
     for (int tile = blockIdx.x; tile < total; tile += gridDim.x) {
@@ -394,7 +405,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         uint16_t *o = p.out + (size_t(t.e) * M_out + t.mt * BM + r_in_tile) * N_out + t.nt * BN;
         const uint4 z = make_uint4(0, 0, 0, 0);
 #pragma unroll 4
-        for (int c = 0; c < BN; c += 8) stg_v4(o + c, z);
+        for (int c = half * (BN / 2); c < (half + 1) * (BN / 2); c += 8) stg_v4(o + c, z);
         continue;
       }
       const uint32_t a = tcount & 1u, aph = (tcount >> 1) & 1u;
@@ -405,7 +416,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       const uint32_t tb = tmem_base + (uint32_t(q * 32) << 16) + a * BN;
 
       epilogue_tile<MODE, BN>(p, tb, size_t(t.goff) + size_t(t.mt) * BM + r_in_tile,
-                              t.mt * BM + r_in_tile, t.e, t.nt);
+                              t.mt * BM + r_in_tile, t.e, t.nt, half);
       tc::fence_before_sync();
       __syncwarp();
       if (lane == 0) tc::mbar_arrive(tempty_bar(a));
@@ -496,7 +507,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     for (int a = 0; a < 2; ++a) {
       tc::mbar_init(tfull_bar(a), 1);
-      tc::mbar_init(tempty_bar(a), 8);  // 4 epilogue warps in each CTA of the pair
+      tc::mbar_init(tempty_bar(a), 2 * kEpiWarps);  // the epilogue warps of both CTAs
     }
     tc::mbar_init(drain_bar, 1);
     tc::fence_mbar_init();
@@ -653,6 +664,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   } else {
     // ============ epilogue (warps 2..5 of each CTA) ============
     const int q = warp & 3;
+    const int half = (warp - 2) / 4;
     const int r_in_tile = q * 32 + lane;
     const uint32_t tempty_leader = tc::mapa(tempty_bar(0), 0);
     uint32_t tcount = 0;
@@ -666,7 +678,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           uint16_t *o = p.out + (size_t(t.e) * M_out + mt * BM + r_in_tile) * N_out + t.nt * BN;
           const uint4 z = make_uint4(0, 0, 0, 0);
 #pragma unroll 4
-          for (int c = 0; c < BN; c += 8) stg_v4(o + c, z);
+          for (int c = half * (BN / 2); c < (half + 1) * (BN / 2); c += 8) stg_v4(o + c, z);
         }
         continue;
       }
@@ -678,7 +690,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (mine) {
         const uint32_t tb = tmem_base + (uint32_t(q * 32) << 16) + a * BN;
         epilogue_tile<MODE, BN>(p, tb, size_t(t.goff) + size_t(mt) * BM + r_in_tile,
-                                mt * BM + r_in_tile, t.e, t.nt);
+                                mt * BM + r_in_tile, t.e, t.nt, half);
       }
       tc::fence_before_sync();
       __syncwarp();
@@ -733,17 +745,15 @@ int make_map(CUtensorMap *m, const void *base, uint64_t rows, uint64_t cols, uin
   if (r != CUDA_SUCCESS) return moe::set_error(MOE_ERR_CUDA, "tensor map for %s: CUresult %d", what, int(r));
   return MOE_OK;
 }
-// CTA-pair kernel for every shape except dH (its epilogue reads and writes two
-// [rows, F] tensors, so it is epilogue-bound and the one-SM kernel with its
-// longer mainloop per tile is faster). MOE_GEMM_1SM=1 selects the one-SM kernel
-// everywhere (for A/B measurements).
+// The CTA-pair kernel runs every shape; MOE_GEMM_1SM=1 selects the one-SM kernel
+// instead (kept for A/B measurements of the two forms).
 template <int MODE> bool use_pair() {
   static int v = -1;
   if (v < 0) {
     const char *e = getenv("MOE_GEMM_1SM");
     v = (e && e[0] == '1') ? 0 : 1;
   }
-  return v == 1 && MODE != kDgradDown;
+  return v == 1;
 }
 
 template <int MODE, int BN>

@@ -59,6 +59,15 @@ def run_gpu_layer(inp, E, k, mask=None, logits_in=None, backward=True):
     return b
 
 
+def unblock_ab(ab_flat, F):
+    """[rows, 2F] matrix from the 32-row blocked layout of the saved pre-activations:
+    element (r, c) sits at ((r/32)*(2F/8) + c/8)*256 + (r%32)*8 + c%8."""
+    a = np.asarray(ab_flat).reshape(-1)
+    nblk = a.size // (32 * 2 * F)
+    a = a[:nblk * 32 * 2 * F].reshape(nblk, 2 * F // 8, 32, 8)
+    return a.transpose(0, 2, 1, 3).reshape(nblk * 32, 2 * F)
+
+
 def topk_margin(z32, k):
     """Smallest gap among the k+1 largest logits per token: above the rounding of
     the logits, the ordered top-k is unique (inf gaps past the last expert)."""

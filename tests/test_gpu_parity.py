@@ -13,7 +13,7 @@ from paper_2601_14327_gb300 import _lib as L
 from paper_2601_14327_gb300 import layer
 
 from gpu_helpers import (assert_close, case_inputs, oracle_inputs, rel_err, run_gpu_layer, to_np,
-                         topk_margin)
+                         topk_margin, unblock_ab)
 
 pytestmark = pytest.mark.gpu
 
@@ -200,8 +200,9 @@ def test_layer_fwd_bwd_against_oracle(T, d, E, k, F, bias, n_masked):
     flat = row.reshape(-1)
     nrows = lambda a: a.reshape(T * k, -1)
     np.testing.assert_allclose(b.topk_gate.cpu().numpy(), ref["gates"], rtol=0, atol=2e-6)
-    assert_close("a", to_np(b.ab)[flat][:, :F], nrows(ref["a"]))
-    assert_close("b", to_np(b.ab)[flat][:, F:], nrows(ref["b"]))
+    ab = unblock_ab(to_np(b.ab), F)
+    assert_close("a", ab[flat][:, :F], nrows(ref["a"]))
+    assert_close("b", ab[flat][:, F:], nrows(ref["b"]))
     assert_close("h", to_np(b.h)[flat], nrows(ref["h"]))
     assert_close("o", to_np(b.out_perm)[flat], nrows(ref["o"]))
     assert_close("y", to_np(b.y), ref["y"])

@@ -287,6 +287,23 @@ int moe_grouped_ffn_bwd(const uint16_t *d_out_perm, const uint16_t *x_perm,
                         size_t ws_bytes, moe_stream_t stream);
 
 /*
+ * moe_grouped_ffn_bwd_dgrad / moe_grouped_ffn_bwd_wgrad - the two halves of
+ * moe_grouped_ffn_bwd (which calls them in this order on one stream), for
+ * callers that overlap other work with the weight gradients:
+ *   dgrad: dH = dO W_down, [dA|dB] (into d_ab), dX = [dA|dB] W_gate_up
+ *   wgrad: dW_down = dO^T H, dW_gate_up = [dA|dB]^T X  (needs d_ab from dgrad)
+ * Arguments as in moe_grouped_ffn_bwd.
+ */
+int moe_grouped_ffn_bwd_dgrad(const uint16_t *d_out_perm, const uint16_t *ab_saved,
+                              const int32_t *group_offsets, int E, int d, int F, int64_t rows_cap,
+                              const uint16_t *w_gate_up, const uint16_t *w_down, uint16_t *d_ab,
+                              uint16_t *dx_perm, moe_stream_t stream);
+int moe_grouped_ffn_bwd_wgrad(const uint16_t *d_out_perm, const uint16_t *x_perm,
+                              const uint16_t *h, const uint16_t *d_ab,
+                              const int32_t *group_offsets, int E, int d, int F, int64_t rows_cap,
+                              uint16_t *dw_gate_up, uint16_t *dw_down, moe_stream_t stream);
+
+/*
  * moe_route_bwd - backward of the router's softmax over the selected experts:
  *   d_logits[t,j] = g[t,j] * (d_gate[t,j] - sum_i g[t,i] * d_gate[t,i])
  *   dw_router[:, e] = sum over assignments (t,j) to e of d_logits[t,j] * x[t,:]

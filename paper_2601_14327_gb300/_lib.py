@@ -55,6 +55,8 @@ _SIGS = {
     "moe_unpermute_combine": (I, [P, P, P, I, I, I, P, P]),
     "moe_unpermute_combine_bwd": (I, [P, P, P, P, P, P, I, I, I, I, P, P, P]),
     "moe_grouped_ffn_bwd": (I, [P, P, P, P, P, I, I, I, I64, P, P, P, P, P, P, P, SZ, P]),
+    "moe_grouped_ffn_bwd_dgrad": (I, [P, P, P, I, I, I, I64, P, P, P, P, P]),
+    "moe_grouped_ffn_bwd_wgrad": (I, [P, P, P, P, P, I, I, I, I64, P, P, P]),
     "moe_route_bwd": (I, [P, P, P, P, P, P, P, I, I, I, I, I64, P, P, P, SZ, P]),
     "moe_permute_bwd": (I, [P, P, P, P, P, I, I, I, I, P, P, SZ, P]),
 }
@@ -241,6 +243,20 @@ def moe_grouped_ffn_bwd(d_out_perm, x_perm, ab_saved, h, group_offsets, E, d, F,
         _ptr(d_out_perm), _ptr(x_perm), _ptr(ab_saved), _ptr(h), _ptr(group_offsets), E, d, F,
         rows_cap, _ptr(w_gate_up), _ptr(w_down), _ptr(d_ab), _ptr(dx_perm), _ptr(dw_gate_up),
         _ptr(dw_down), _ptr(ws), ws_bytes, _stream(stream)))
+
+
+def moe_grouped_ffn_bwd_dgrad(d_out_perm, ab_saved, group_offsets, E, d, F, rows_cap, w_gate_up,
+                              w_down, d_ab, dx_perm, stream=None):
+    _check("moe_grouped_ffn_bwd_dgrad", load().moe_grouped_ffn_bwd_dgrad(
+        _ptr(d_out_perm), _ptr(ab_saved), _ptr(group_offsets), E, d, F, rows_cap,
+        _ptr(w_gate_up), _ptr(w_down), _ptr(d_ab), _ptr(dx_perm), _stream(stream)))
+
+
+def moe_grouped_ffn_bwd_wgrad(d_out_perm, x_perm, h, d_ab, group_offsets, E, d, F, rows_cap,
+                              dw_gate_up, dw_down, stream=None):
+    _check("moe_grouped_ffn_bwd_wgrad", load().moe_grouped_ffn_bwd_wgrad(
+        _ptr(d_out_perm), _ptr(x_perm), _ptr(h), _ptr(d_ab), _ptr(group_offsets), E, d, F,
+        rows_cap, _ptr(dw_gate_up), _ptr(dw_down), _stream(stream)))
 
 
 def moe_route_bwd(x_perm, topk_idx, topk_gate, d_gate, row_of_assignment, group_offsets,

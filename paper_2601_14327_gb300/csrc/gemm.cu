@@ -880,20 +880,15 @@ int moe_grouped_ffn_fwd(const uint16_t *x_perm, const int32_t *group_offsets, in
                          "moe_grouped_ffn_fwd: down GEMM");
 }
 
-int moe_grouped_ffn_bwd(const uint16_t *d_out_perm, const uint16_t *x_perm,
-                        const uint16_t *ab_saved, const uint16_t *h, const int32_t *group_offsets,
-                        int E, int d, int F, int64_t rows_cap, const uint16_t *w_gate_up,
-                        const uint16_t *w_down, uint16_t *d_ab, uint16_t *dx_perm,
-                        uint16_t *dw_gate_up, uint16_t *dw_down, void *ws, size_t ws_bytes,
-                        moe_stream_t stream) {
-  (void)ws;
-  (void)ws_bytes;
+int moe_grouped_ffn_bwd_dgrad(const uint16_t *d_out_perm, const uint16_t *ab_saved,
+                              const int32_t *group_offsets, int E, int d, int F, int64_t rows_cap,
+                              const uint16_t *w_gate_up, const uint16_t *w_down, uint16_t *d_ab,
+                              uint16_t *dx_perm, moe_stream_t stream) {
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-  if (int st = check_common(E, d, F, rows_cap, "moe_grouped_ffn_bwd")) return st;
-  const void *ptrs[] = {d_out_perm, x_perm, ab_saved, h, group_offsets, w_gate_up, w_down,
-                        d_ab, dx_perm, dw_gate_up, dw_down};
+  if (int st = check_common(E, d, F, rows_cap, "moe_grouped_ffn_bwd_dgrad")) return st;
+  const void *ptrs[] = {d_out_perm, ab_saved, group_offsets, w_gate_up, w_down, d_ab, dx_perm};
   for (const void *q : ptrs)
-    if (!q || !moe::aligned16(q)) return moe::set_error(MOE_ERR_ARG, "moe_grouped_ffn_bwd: null or unaligned pointer");
+    if (!q || !moe::aligned16(q)) return moe::set_error(MOE_ERR_ARG, "moe_grouped_ffn_bwd_dgrad: null or unaligned pointer");
   const uint64_t R = uint64_t(rows_cap);
   int st;
   GemmParams p{};
@@ -910,9 +905,24 @@ int moe_grouped_ffn_bwd(const uint16_t *d_out_perm, const uint16_t *x_perm,
   p.nkb = 2 * F / BK;
   p.out = dx_perm;
   p.aux = nullptr;
-  if ((st = run_gemm<kDgradGateUp>(d, d_ab, R, 2 * F, w_gate_up, uint64_t(E) * 2 * F, d, p, s,
-                                   "moe_grouped_ffn_bwd: dX GEMM")))
-    return st;
+  return run_gemm<kDgradGateUp>(d, d_ab, R, 2 * F, w_gate_up, uint64_t(E) * 2 * F, d, p, s,
+                                "moe_grouped_ffn_bwd: dX GEMM");
+}
+
+int moe_grouped_ffn_bwd_wgrad(const uint16_t *d_out_perm, const uint16_t *x_perm,
+                              const uint16_t *h, const uint16_t *d_ab,
+                              const int32_t *group_offsets, int E, int d, int F, int64_t rows_cap,
+                              uint16_t *dw_gate_up, uint16_t *dw_down, moe_stream_t stream) {
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if (int st = check_common(E, d, F, rows_cap, "moe_grouped_ffn_bwd_wgrad")) return st;
+  const void *ptrs[] = {d_out_perm, x_perm, h, d_ab, group_offsets, dw_gate_up, dw_down};
+  for (const void *q : ptrs)
+    if (!q || !moe::aligned16(q)) return moe::set_error(MOE_ERR_ARG, "moe_grouped_ffn_bwd_wgrad: null or unaligned pointer");
+  const uint64_t R = uint64_t(rows_cap);
+  int st;
+  GemmParams p{};
+  p.group_offsets = group_offsets;
+  p.E = E; p.d = d; p.F = F;
   // dW_down[e] = dO_e^T H_e   ([d, F])
   p.nkb = 0;
   p.m_tiles_w = d / BM;
@@ -925,6 +935,21 @@ int moe_grouped_ffn_bwd(const uint16_t *d_out_perm, const uint16_t *x_perm,
   p.out = dw_gate_up;
   return run_gemm<kWgradGateUp>(d, d_ab, R, 2 * F, x_perm, R, d, p, s,
                                 "moe_grouped_ffn_bwd: dW_gate_up GEMM");
+}
+
+int moe_grouped_ffn_bwd(const uint16_t *d_out_perm, const uint16_t *x_perm,
+                        const uint16_t *ab_saved, const uint16_t *h, const int32_t *group_offsets,
+                        int E, int d, int F, int64_t rows_cap, const uint16_t *w_gate_up,
+                        const uint16_t *w_down, uint16_t *d_ab, uint16_t *dx_perm,
+                        uint16_t *dw_gate_up, uint16_t *dw_down, void *ws, size_t ws_bytes,
+                        moe_stream_t stream) {
+  (void)ws;
+  (void)ws_bytes;
+  if (int st = moe_grouped_ffn_bwd_dgrad(d_out_perm, ab_saved, group_offsets, E, d, F, rows_cap,
+                                         w_gate_up, w_down, d_ab, dx_perm, stream))
+    return st;
+  return moe_grouped_ffn_bwd_wgrad(d_out_perm, x_perm, h, d_ab, group_offsets, E, d, F, rows_cap,
+                                   dw_gate_up, dw_down, stream);
 }
 
 }  // extern "C"

@@ -70,6 +70,14 @@ __device__ __forceinline__ void tma_load_2d(uint32_t dst, const void *map, uint3
       : "memory");
 }
 
+// L2 prefetch of a 2-D tile (no shared memory, no completion signal).
+__device__ __forceinline__ void tma_prefetch_2d(const void *map, int c0, int c1) {
+  asm volatile("cp.async.bulk.prefetch.tensor.2d.L2.global.tile [%0, {%1, %2}];" ::"l"(
+                   reinterpret_cast<uint64_t>(map)),
+               "r"(c0), "r"(c1)
+               : "memory");
+}
+
 // ---- clusters -------------------------------------------------------------------
 __device__ __forceinline__ uint32_t cluster_ctarank() {
   uint32_t r;

@@ -59,6 +59,9 @@ class MoELayerBuffers:
             self.d_logits = torch.empty(s.T, s.k, dtype=f32, device=dev)
             self.dw_router = torch.empty(s.d, s.E, dtype=f32, device=dev)
             self.dx = torch.empty(s.T, s.d, dtype=bf16, device=dev)
+            # second stream: the router backward and the unpermute-sum run beside
+            # the grouped GEMMs (whose CTAs leave registers and threads free)
+            self.side = torch.cuda.Stream(device=dev) if dev.type == "cuda" else None
 
 
 def route(b: MoELayerBuffers, x, w_router, bias, active_mask=None, logits_in=None,
@@ -83,22 +86,42 @@ def forward(b: MoELayerBuffers, x, w_router, bias, w_gate_up, w_down, active_mas
     return b.y
 
 
-def backward(b: MoELayerBuffers, dy, w_router, w_gate_up, w_down, stream=None):
-    """combine bwd -> grouped FFN bwd -> router bwd -> permute bwd.
+def backward(b: MoELayerBuffers, dy, w_router, w_gate_up, w_down, stream=None,
+             overlap: bool = True):
+    """combine bwd -> grouped FFN bwd (dgrad, then wgrad) -> router bwd -> permute bwd.
+
+    With overlap, the router backward (after the combine backward) and the
+    unpermute-sum (after the dX GEMM) run on a second stream while the main stream
+    computes the weight gradients; the main stream waits for them at the end.
     Returns (dx, dw_gate_up, dw_down, dw_router)."""
     s = b.shape
     R = s.rows_cap
+    main = torch.cuda.current_stream() if stream is None else stream
+    side = b.side if overlap else main
     L.moe_unpermute_combine_bwd(dy, b.out_perm, b.row_of_assignment, b.topk_gate,
                                 b.group_offsets, b.group_counts, s.T, s.d, s.E, s.k,
-                                b.d_out_perm, b.d_gate, stream)
-    L.moe_grouped_ffn_bwd(b.d_out_perm, b.x_perm, b.ab, b.h, b.group_offsets, s.E, s.d, s.F, R,
-                          w_gate_up, w_down, b.d_ab, b.dx_perm, b.dw_gate_up, b.dw_down, b.ws,
-                          b.ws_bytes, stream)
+                                b.d_out_perm, b.d_gate, main)
+    if overlap:
+        ev = torch.cuda.Event()
+        ev.record(main)
+        side.wait_event(ev)
     L.moe_route_bwd(b.x_perm, b.topk_idx, b.topk_gate, b.d_gate, b.row_of_assignment,
                     b.group_offsets, b.group_counts, s.T, s.d, s.E, s.k, R, b.d_logits,
-                    b.dw_router, b.ws, b.ws_bytes, stream)
+                    b.dw_router, b.ws, b.ws_bytes, side)
+    L.moe_grouped_ffn_bwd_dgrad(b.d_out_perm, b.ab, b.group_offsets, s.E, s.d, s.F, R,
+                                w_gate_up, w_down, b.d_ab, b.dx_perm, main)
+    if overlap:
+        ev = torch.cuda.Event()
+        ev.record(main)
+        side.wait_event(ev)
     L.moe_permute_bwd(b.dx_perm, b.row_of_assignment, b.topk_idx, b.d_logits, w_router, s.T,
-                      s.d, s.E, s.k, b.dx, b.ws, b.ws_bytes, stream)
+                      s.d, s.E, s.k, b.dx, b.ws, b.ws_bytes, side)
+    L.moe_grouped_ffn_bwd_wgrad(b.d_out_perm, b.x_perm, b.h, b.d_ab, b.group_offsets, s.E, s.d,
+                                s.F, R, b.dw_gate_up, b.dw_down, main)
+    if overlap:
+        ev = torch.cuda.Event()
+        ev.record(side)
+        main.wait_event(ev)
     return b.dx, b.dw_gate_up, b.dw_down, b.dw_router
 
 

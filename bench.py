@@ -141,12 +141,13 @@ class Workload:
     """Inputs, the one-time LAEP prune, and the buffers of one layer step."""
 
     def __init__(self, cfg_id: int, device: str, compact_override=None, tokens=None,
-                 experts=None, no_prune=False):
+                 experts=None, no_prune=False, bias=None):
         c = synth.CONFIGS[cfg_id]
-        if tokens or experts or no_prune:  # a smaller case of the same kernels (profiling)
+        if tokens or experts or no_prune or bias:  # a variant of the workload (profiling)
             import dataclasses
-            c = dataclasses.replace(c, name=c.name + f"_small_T{tokens or c.T}_E{experts or c.E}",
-                                    T=tokens or c.T, E=experts or c.E,
+            c = dataclasses.replace(c, name=c.name + f"_variant_T{tokens or c.T}_E{experts or c.E}"
+                                    f"_{bias or c.bias}", T=tokens or c.T, E=experts or c.E,
+                                    bias=bias or c.bias,
                                     prune_lowest=0 if no_prune else c.prune_lowest)
         self.cfg = c
         self.cfg_id = cfg_id
@@ -183,12 +184,32 @@ class Workload:
         self.E_live = E - (self.n_pruned if self.mask is not None else 0)
         self.bufs = layer.MoELayerBuffers(self.shape, device, backward=True)
 
+        self.graph = None
+
     def step(self, x=None, dy=None):
+        if self.graph is not None and x is None and dy is None:
+            self.graph.replay()
+            return
+        self.eager_step(x, dy)
+
+    def eager_step(self, x=None, dy=None):
         i, b = self.inp, self.bufs
         layer.forward(b, i["x"] if x is None else x, i["w_router"], i["bias"], i["w_gate_up"],
                       i["w_down"], self.mask)
         layer.backward(b, i["dy"] if dy is None else dy, i["w_router"], i["w_gate_up"],
                        i["w_down"])
+
+    def capture(self):
+        """Records one whole step (both streams) into a CUDA graph; later steps replay it.
+        The library's calls allocate nothing and never synchronize, so they capture as is;
+        everything they set up once (tensor-map encoder, occupancy, attributes) ran in the
+        eager warm-up steps before."""
+        torch.cuda.synchronize()
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            self.eager_step()
+        torch.cuda.synchronize()
+        self.graph = g
 
     def gemm_flops(self):
         """Algorithmic FLOPs per GEMM kernel launch (real assignments only)."""
@@ -265,12 +286,12 @@ def host_inputs(inp, n_tok):
     return out
 
 
-def timed_steps(wl, steps, world, local):
+def timed_steps(wl, steps, world, local, per_kernel_timing=True):
     """K timed steps between barrier+synchronize; returns (max-over-ranks ms, per-kernel
     CUDA-event table, clock samples)."""
     stream = torch.cuda.current_stream()
     clocks = ClockSampler(local)
-    L.moe_timing_enable(True)
+    L.moe_timing_enable(per_kernel_timing)
     L.moe_timing_read(reset=True)
     ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     barrier(world)
@@ -338,7 +359,11 @@ def laep_comparison(args, world, local, pruned_tps, wl_pruned):
     wl_u = Workload(args.config, "cuda", no_prune=True)
     for _ in range(args.warmup):
         wl_u.step()
-    ms_u, _, _ = timed_steps(wl_u, steps, world, local)
+    if args.graph:
+        wl_u.capture()
+        for _ in range(args.warmup):
+            wl_u.step()
+    ms_u, _, _ = timed_steps(wl_u, steps, world, local, per_kernel_timing=not args.graph)
     tps_u = replica_throughput(world, wl_u.shape.T, steps, ms_u)
     unpruned_params = 3 * wl_u.shape.E * wl_u.shape.d * wl_u.shape.F
     del wl_u
@@ -357,7 +382,7 @@ def run_ours(args):
     L.load()
     peaks = measured_peaks()
     wl = Workload(args.config, "cuda", tokens=args.tokens, experts=args.experts,
-                  no_prune=args.no_prune)
+                  no_prune=args.no_prune, bias=args.bias)
     s = wl.shape
     torch.cuda.synchronize()
     for _ in range(args.warmup):
@@ -366,7 +391,15 @@ def run_ours(args):
     assert L.moe_device_error(clear=True) == 0, "device error during warm-up"
 
     stream = torch.cuda.current_stream()
-    ms_total, per_kernel, clk = timed_steps(wl, args.steps, world, local)
+    if args.graph:
+        # per-kernel CUDA-event table from eager steps, the timed steps replay a graph
+        _, per_kernel, _ = timed_steps(wl, args.steps, world, local, per_kernel_timing=True)
+        wl.capture()
+        for _ in range(args.warmup):
+            wl.step()
+        ms_total, _, clk = timed_steps(wl, args.steps, world, local, per_kernel_timing=False)
+    else:
+        ms_total, per_kernel, clk = timed_steps(wl, args.steps, world, local)
     ms_step = ms_total / args.steps
     tokens_per_s = replica_throughput(world, s.T, args.steps, ms_total)
     launches = sum(n for n, _ in per_kernel.values())
@@ -381,7 +414,8 @@ def run_ours(args):
     peak = peaks["bf16_tflops_sustained"]
     kernel_table = kernel_report(wl, per_kernel, args.steps, peaks)
     laep = None
-    if wl.cfg.compact and args.tokens is None and args.experts is None and not args.no_prune:
+    if (wl.cfg.compact and args.tokens is None and args.experts is None and not args.no_prune
+            and args.bias is None):
         laep = laep_comparison(args, world, local, tokens_per_s, wl)
 
     # end to end through the public API: pinned host inputs in, results out
@@ -446,8 +480,10 @@ def run_ours(args):
         "roofline": {"kernel": dom, "bound": "tensor", "achieved": round(dom_tflops, 1),
                      "peak": peak, "unit": "TFLOP/s", "frac": round(dom_tflops / peak, 4),
                      "traffic": (committed_traffic(dom) if wl.cfg_id == 2 and args.tokens is None
-                                 and args.experts is None and not args.no_prune else None),
+                                 and args.experts is None and not args.no_prune
+                                 and args.bias is None else None),
                      "peak_source": f"bf16 sustained ({peaks['source']})"},
+        "timed_as": "CUDA graph replay of the whole step" if args.graph else "eager launches",
         "kernels": kernel_table,
         "laep": laep,
         "gpu_launches": launches,
@@ -516,10 +552,13 @@ def main():
     ap.add_argument("--ref-tokens", type=int, default=64)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--graph", type=int, default=1,
+                    help="time replays of a CUDA graph of the whole step (1) or eager steps (0)")
     # smaller cases of the same kernels, for profiler captures
     ap.add_argument("--tokens", type=int, default=None)
     ap.add_argument("--experts", type=int, default=None)
     ap.add_argument("--no-prune", action="store_true")
+    ap.add_argument("--bias", choices=["none", "zipf", "loguniform"], default=None)
     args = ap.parse_args()
     if args.warmup < 3 and args.impl == "ours":
         args.warmup = 3

@@ -67,7 +67,7 @@ template <int BN> struct Shape {
   static constexpr uint32_t STAGE_BYTES = A_BYTES + B_BYTES;
   static constexpr int NBARS = 2 * STAGES + 5;
   static constexpr size_t SMEM = 1024 + size_t(STAGES) * STAGE_BYTES + NBARS * 8 +
-                                 (4 + 257 + 256 + 257) * 4;
+                                 (4 + 257 + 256 + 257) * 4 + 1024 + kEpiWarps * 2048;
   static constexpr uint32_t TMEM_COLS = 2 * BN;
 };
 
@@ -91,18 +91,6 @@ __device__ __forceinline__ void fail(volatile int *abort_flag) {
   *abort_flag = 1;
 }
 
-__device__ __forceinline__ void store_row_bf16(uint16_t *dst, const uint32_t (&r)[32]) {
-#pragma unroll
-  for (int v = 0; v < 4; ++v) {
-    uint4 o;
-    o.x = pack_bf16x2(__uint_as_float(r[v * 8 + 0]), __uint_as_float(r[v * 8 + 1]));
-    o.y = pack_bf16x2(__uint_as_float(r[v * 8 + 2]), __uint_as_float(r[v * 8 + 3]));
-    o.z = pack_bf16x2(__uint_as_float(r[v * 8 + 4]), __uint_as_float(r[v * 8 + 5]));
-    o.w = pack_bf16x2(__uint_as_float(r[v * 8 + 6]), __uint_as_float(r[v * 8 + 7]));
-    stg_v4(dst + v * 8, o);
-  }
-}
-
 __device__ __forceinline__ float silu_f(float a) { return a / (1.f + __expf(-a)); }
 
 // Saved pre-activations [A|B] are stored in 32-row blocks: element (r, c) of the
@@ -118,19 +106,61 @@ __device__ __forceinline__ size_t ab_block_index(size_t row, int col, int F) {
 // accumulator from tensor memory at `tb` (lane base and column base included) and
 // writes the mode's outputs. `row` = row of this thread in the grouped layout
 // (activation modes), `out_row` = row in the expert's weight-gradient matrix.
+// Output staging: each epilogue warp owns a 2 KB shared-memory buffer that holds
+// one 32-row x 32-column bf16 chunk in the 64-byte-swizzle layout of a TMA tile
+// (row r, 16-byte chunk c at r*64 + ((c ^ ((r >> 1) & 3)) * 16): conflict-free
+// when every lane writes its own row); one lane then issues a TMA tensor store.
+constexpr uint32_t kStageBytes = 32 * 64;
+
+__device__ __forceinline__ void st_shared_v4(uint32_t addr, const uint4 &v) {
+  asm volatile("st.shared.v4.u32 [%0], {%1,%2,%3,%4};" ::"r"(addr), "r"(v.x), "r"(v.y), "r"(v.z),
+               "r"(v.w)
+               : "memory");
+}
+
+// Writes this lane's 32 bf16 values (row `lane` of the chunk) to the staging
+// buffer and stores the chunk at (col, trow) of tensor map `tm`.
+__device__ __forceinline__ void stage_and_store(const CUtensorMap *tm, uint32_t stage, int lane,
+                                                const uint4 (&v)[4], int col, int trow) {
+  if (lane == 0) tc::bulk_wait_read0();  // the previous chunk has left the buffer
+  __syncwarp();
+  const uint32_t rowbase = stage + uint32_t(lane) * 64u;
+  const uint32_t sw = (uint32_t(lane) >> 1) & 3u;
+#pragma unroll
+  for (uint32_t c = 0; c < 4; ++c) st_shared_v4(rowbase + ((c ^ sw) << 4), v[c]);
+  tc::fence_proxy_async_smem();
+  __syncwarp();
+  if (lane == 0) {
+    tc::tma_store_2d(tm, stage, col, trow);
+    tc::bulk_commit();
+  }
+}
+
+__device__ __forceinline__ void pack32(const uint32_t (&r)[32], uint4 (&v)[4]) {
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    v[q].x = pack_bf16x2(__uint_as_float(r[q * 8 + 0]), __uint_as_float(r[q * 8 + 1]));
+    v[q].y = pack_bf16x2(__uint_as_float(r[q * 8 + 2]), __uint_as_float(r[q * 8 + 3]));
+    v[q].z = pack_bf16x2(__uint_as_float(r[q * 8 + 4]), __uint_as_float(r[q * 8 + 5]));
+    v[q].w = pack_bf16x2(__uint_as_float(r[q * 8 + 6]), __uint_as_float(r[q * 8 + 7]));
+  }
+}
+
 template <int MODE, int BN>
-__device__ __forceinline__ void epilogue_tile(const GemmParams &p, uint32_t tb, size_t row,
+__device__ __forceinline__ void epilogue_tile(const GemmParams &p, const CUtensorMap *tmO,
+                                              uint32_t stage, int lane, uint32_t tb, size_t row,
                                               int out_row, int e, int nt, int half) {
   using Tr = Traits<MODE>;
   if (MODE == kGateUp) {
     const int F = p.F;
-    uint16_t *hrow = p.out + row * F + nt * 128;
+    const int trow = int(row) - lane;
 #pragma unroll 1
     for (int c = half * 64; c < half * 64 + 64; c += 32) {
       uint32_t ra[32], rb[32];
       tc::tmem_ld_32x32b_x32(tb + c, ra);
       tc::tmem_ld_32x32b_x32(tb + 128 + c, rb);
       tc::tmem_ld_wait();
+      uint4 vh[4];
 #pragma unroll
       for (int v = 0; v < 4; ++v) {
         float fa[8], fb[8], fh[8];
@@ -141,16 +171,16 @@ __device__ __forceinline__ void epilogue_tile(const GemmParams &p, uint32_t tb, 
           fh[i] = silu_f(fa[i]) * fb[i];
         }
         const int col = nt * 128 + c + v * 8;
-        stg_v4(hrow + c + v * 8, pack8(fh));
+        vh[v] = pack8(fh);
         stg_v4(p.out2 + ab_block_index(row, col, F), pack8(fa));
         stg_v4(p.out2 + ab_block_index(row, F + col, F), pack8(fb));
       }
+      stage_and_store(tmO, stage, lane, vh, nt * 128 + c, trow);
     }
   } else if (MODE == kDgradDown) {
     const int F = p.F;
     const int f0 = nt * BN;
-    uint16_t *darow = p.out + row * 2 * F + f0;
-    uint16_t *dbrow = darow + F;
+    const int trow = int(row) - lane;
 #pragma unroll 1
     for (int c = half * (BN / 2); c < (half + 1) * (BN / 2); c += 32) {
       uint4 va[4], vb[4];
@@ -162,6 +192,7 @@ __device__ __forceinline__ void epilogue_tile(const GemmParams &p, uint32_t tb, 
       uint32_t r[32];
       tc::tmem_ld_32x32b_x32(tb + c, r);
       tc::tmem_ld_wait();
+      uint4 vda[4], vdb[4];
 #pragma unroll
       for (int v = 0; v < 4; ++v) {
         float fa[8], fb[8], da[8], db[8];
@@ -174,32 +205,55 @@ __device__ __forceinline__ void epilogue_tile(const GemmParams &p, uint32_t tb, 
           da[i] = dh * fb[i] * (sg * (1.f + fa[i] * (1.f - sg)));
           db[i] = dh * fa[i] * sg;
         }
-        stg_v4(darow + c + v * 8, pack8(da));
-        stg_v4(dbrow + c + v * 8, pack8(db));
+        vda[v] = pack8(da);
+        vdb[v] = pack8(db);
       }
+      stage_and_store(tmO, stage, lane, vda, f0 + c, trow);
+      stage_and_store(tmO, stage, lane, vdb, F + f0 + c, trow);
     }
   } else {
-    uint16_t *orow;
+    int trow;
     if (Tr::WGRAD) {
-      const int M_out = p.m_tiles_w * BM, N_out = p.n_tiles * BN;
-      orow = p.out + (size_t(e) * M_out + out_row) * N_out + nt * BN;
+      const int M_out = p.m_tiles_w * BM;
+      trow = e * M_out + out_row - lane;
     } else {
-      orow = p.out + row * p.d + nt * BN;
+      trow = int(row) - lane;
     }
 #pragma unroll 1
     for (int c = half * (BN / 2); c < (half + 1) * (BN / 2); c += 32) {
       uint32_t r[32];
       tc::tmem_ld_32x32b_x32(tb + c, r);
       tc::tmem_ld_wait();
-      store_row_bf16(orow + c, r);
+      uint4 v[4];
+      pack32(r, v);
+      stage_and_store(tmO, stage, lane, v, nt * BN + c, trow);
     }
+  }
+}
+
+// Zero weight gradient of an expert without rows: this warp's 32 rows and column half.
+template <int BN>
+__device__ __forceinline__ void zero_tile_store(const CUtensorMap *tmO, uint32_t stage, int lane,
+                                                int trow, int nt, int half) {
+  if (lane == 0) tc::bulk_wait_read0();
+  __syncwarp();
+  const uint4 z = make_uint4(0, 0, 0, 0);
+#pragma unroll
+  for (uint32_t c = 0; c < 4; ++c) st_shared_v4(stage + uint32_t(lane) * 64u + c * 16u, z);
+  tc::fence_proxy_async_smem();
+  __syncwarp();
+  if (lane == 0) {
+    for (int c = half * (BN / 2); c < (half + 1) * (BN / 2); c += 32)
+      tc::tma_store_2d(tmO, stage, nt * BN + c, trow);
+    tc::bulk_commit();
   }
 }
 
 template <int MODE, int BN>
 __global__ void __launch_bounds__(kThreads, 1)
     grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA,
-                        const __grid_constant__ CUtensorMap tmB, const GemmParams p) {
+                        const __grid_constant__ CUtensorMap tmB,
+                        const __grid_constant__ CUtensorMap tmO, const GemmParams p) {
   using Tr = Traits<MODE>;
   using Sh = Shape<BN>;
   constexpr int STAGES = Sh::STAGES;
@@ -216,6 +270,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   int *s_goff = misc + 4;          // [E+1]
   int *s_order = s_goff + 257;     // [E]   experts in schedule order
   int *s_prefix = s_order + 256;   // [E+1] first tile of each scheduled expert
+  const uint32_t stage_base =
+      (tc::smem_u32(s_prefix + 257) + 1023u) & ~1023u;  // epilogue staging, 2 KB per warp
   volatile int *abort_flag = misc + 1;
   volatile int no_abort = 0;
 
@@ -245,6 +301,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (warp == 0 && lane == 0) {
     tc::tma_prefetch_desc(&tmA);
     tc::tma_prefetch_desc(&tmB);
+    tc::tma_prefetch_desc(&tmO);
   }
   if (warp == 1) {
     tc::tmem_alloc(tc::smem_u32(misc), Sh::TMEM_COLS);
@@ -395,17 +452,15 @@ __global__ void __launch_bounds__(kThreads, 1)
     // ===================== epilogue (warps 2..5) =====================
     const int q = warp & 3;  // TMEM lane quarter this warp may access
     const int half = (warp - 2) / 4;  // column half this warp handles
+    const uint32_t stage = stage_base + uint32_t(warp - 2) * kStageBytes;
     const int r_in_tile = q * 32 + lane;
     uint32_t tcount = 0;
     for (int tile = blockIdx.x; tile < total; tile += gridDim.x) {
       const Tile t = decode(tile);
       if (Tr::WGRAD && t.nkb == 0) {
         // empty group: its weight gradient is exactly zero
-        const int M_out = p.m_tiles_w * BM, N_out = p.n_tiles * BN;
-        uint16_t *o = p.out + (size_t(t.e) * M_out + t.mt * BM + r_in_tile) * N_out + t.nt * BN;
-        const uint4 z = make_uint4(0, 0, 0, 0);
-#pragma unroll 4
-        for (int c = half * (BN / 2); c < (half + 1) * (BN / 2); c += 8) stg_v4(o + c, z);
+        const int M_out = p.m_tiles_w * BM;
+        zero_tile_store<BN>(&tmO, stage, lane, t.e * M_out + t.mt * BM + q * 32, t.nt, half);
         continue;
       }
       const uint32_t a = tcount & 1u, aph = (tcount >> 1) & 1u;
@@ -415,13 +470,16 @@ __global__ void __launch_bounds__(kThreads, 1)
       tc::fence_after_sync();
       const uint32_t tb = tmem_base + (uint32_t(q * 32) << 16) + a * BN;
 
-      epilogue_tile<MODE, BN>(p, tb, size_t(t.goff) + size_t(t.mt) * BM + r_in_tile,
+      epilogue_tile<MODE, BN>(p, &tmO, stage, lane, tb,
+                              size_t(t.goff) + size_t(t.mt) * BM + r_in_tile,
                               t.mt * BM + r_in_tile, t.e, t.nt, half);
       tc::fence_before_sync();
       __syncwarp();
       if (lane == 0) tc::mbar_arrive(tempty_bar(a));
       ++tcount;
     }
+    if (lane == 0) tc::bulk_wait0();  // this warp's output stores are complete
+    __syncwarp();
   }
 
   tc::fence_before_sync();
@@ -454,7 +512,7 @@ template <int BN> struct PairShape {
   static constexpr uint32_t STAGE_BYTES = A_BYTES + B_BYTES;
   static constexpr int NBARS = 2 * STAGES + 5;
   static constexpr size_t SMEM = 1024 + size_t(STAGES) * STAGE_BYTES + NBARS * 8 +
-                                 (4 + 257 + 256 + 257) * 4;
+                                 (4 + 257 + 256 + 257) * 4 + 1024 + kEpiWarps * 2048;
   static constexpr uint32_t TMEM_COLS = 2 * BN;
 };
 
@@ -465,7 +523,8 @@ struct PairTile {
 template <int MODE, int BN>
 __global__ void __launch_bounds__(kThreads, 1)
     grouped_gemm_pair_kernel(const __grid_constant__ CUtensorMap tmA,
-                             const __grid_constant__ CUtensorMap tmB, const GemmParams p) {
+                             const __grid_constant__ CUtensorMap tmB,
+                             const __grid_constant__ CUtensorMap tmO, const GemmParams p) {
   using Tr = Traits<MODE>;
   using Sh = PairShape<BN>;
   constexpr int STAGES = Sh::STAGES;
@@ -483,6 +542,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   int *s_goff = misc + 4;
   int *s_order = s_goff + 257;
   int *s_prefix = s_order + 256;
+  const uint32_t stage_base =
+      (tc::smem_u32(s_prefix + 257) + 1023u) & ~1023u;  // epilogue staging, 2 KB per warp
   volatile int *abort_flag = misc + 1;
   volatile int no_abort = 0;
 
@@ -516,6 +577,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (warp == 0 && lane == 0) {
     tc::tma_prefetch_desc(&tmA);
     tc::tma_prefetch_desc(&tmB);
+    tc::tma_prefetch_desc(&tmO);
   }
   if (warp == 1) {
     tc::tmem_alloc_pair(tc::smem_u32(misc), Sh::TMEM_COLS);
@@ -665,6 +727,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     // ============ epilogue (warps 2..5 of each CTA) ============
     const int q = warp & 3;
     const int half = (warp - 2) / 4;
+    const uint32_t stage = stage_base + uint32_t(warp - 2) * kStageBytes;
     const int r_in_tile = q * 32 + lane;
     const uint32_t tempty_leader = tc::mapa(tempty_bar(0), 0);
     uint32_t tcount = 0;
@@ -674,11 +737,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       const bool mine = mt < t.mtiles;  // this CTA's row block exists
       if (Tr::WGRAD && t.nkb == 0) {
         if (mine) {  // empty group: its weight gradient is exactly zero
-          const int M_out = p.m_tiles_w * BM, N_out = p.n_tiles * BN;
-          uint16_t *o = p.out + (size_t(t.e) * M_out + mt * BM + r_in_tile) * N_out + t.nt * BN;
-          const uint4 z = make_uint4(0, 0, 0, 0);
-#pragma unroll 4
-          for (int c = half * (BN / 2); c < (half + 1) * (BN / 2); c += 8) stg_v4(o + c, z);
+          const int M_out = p.m_tiles_w * BM;
+          zero_tile_store<BN>(&tmO, stage, lane, t.e * M_out + mt * BM + q * 32, t.nt, half);
         }
         continue;
       }
@@ -689,7 +749,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       tc::fence_after_sync();
       if (mine) {
         const uint32_t tb = tmem_base + (uint32_t(q * 32) << 16) + a * BN;
-        epilogue_tile<MODE, BN>(p, tb, size_t(t.goff) + size_t(mt) * BM + r_in_tile,
+        epilogue_tile<MODE, BN>(p, &tmO, stage, lane, tb,
+                                size_t(t.goff) + size_t(mt) * BM + r_in_tile,
                                 mt * BM + r_in_tile, t.e, t.nt, half);
       }
       tc::fence_before_sync();
@@ -697,6 +758,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (lane == 0) tc::mbar_arrive_cluster(tempty_leader + 8u * a);
       ++tcount;
     }
+    if (lane == 0) tc::bulk_wait0();  // this warp's output stores are complete
+    __syncwarp();
   }
 
   tc::fence_before_sync();
@@ -730,9 +793,11 @@ EncodeTiledFn encode_fn() {
   return fn;
 }
 
-// bf16 row-major [rows, cols]; box = box_cols (inner) x box_rows; 128-byte swizzle.
+// bf16 row-major [rows, cols]; box = box_cols (inner) x box_rows; 128-byte swizzle
+// (operands) or 64-byte swizzle (the epilogue's 32 x 32 output chunks).
 int make_map(CUtensorMap *m, const void *base, uint64_t rows, uint64_t cols, uint32_t box_cols,
-             uint32_t box_rows, const char *what) {
+             uint32_t box_rows, const char *what,
+             CUtensorMapSwizzle swizzle = CU_TENSOR_MAP_SWIZZLE_128B) {
   EncodeTiledFn fn = encode_fn();
   if (!fn) return moe::set_error(MOE_ERR_CUDA, "cuTensorMapEncodeTiled unavailable");
   cuuint64_t dims[2] = {cols, rows};
@@ -740,7 +805,7 @@ int make_map(CUtensorMap *m, const void *base, uint64_t rows, uint64_t cols, uin
   cuuint32_t box[2] = {box_cols, box_rows};
   cuuint32_t es[2] = {1, 1};
   CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(base), dims, strides,
-                  box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                  box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, swizzle,
                   CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   if (r != CUDA_SUCCESS) return moe::set_error(MOE_ERR_CUDA, "tensor map for %s: CUresult %d", what, int(r));
   return MOE_OK;
@@ -757,8 +822,8 @@ template <int MODE> bool use_pair() {
 }
 
 template <int MODE, int BN>
-int launch_one(const CUtensorMap &a, const CUtensorMap &b, const GemmParams &p, cudaStream_t s,
-               const char *what) {
+int launch_one(const CUtensorMap &a, const CUtensorMap &b, const CUtensorMap &o,
+               const GemmParams &p, cudaStream_t s, const char *what) {
   using Sh = Shape<BN>;
   static bool attr = false;
   if (!attr) {
@@ -767,13 +832,13 @@ int launch_one(const CUtensorMap &a, const CUtensorMap &b, const GemmParams &p, 
     if (e != cudaSuccess) return moe::cuda_status(e, what);
     attr = true;
   }
-  MOE_LAUNCH(kGemmName[MODE], s, grouped_gemm_kernel<MODE, BN><<<moe::num_sms(), kThreads, Sh::SMEM, s>>>(a, b, p));
+  MOE_LAUNCH(kGemmName[MODE], s, grouped_gemm_kernel<MODE, BN><<<moe::num_sms(), kThreads, Sh::SMEM, s>>>(a, b, o, p));
   return moe::launch_status(what);
 }
 
 template <int MODE, int BN>
-int launch_pair(const CUtensorMap &a, const CUtensorMap &b, const GemmParams &p, cudaStream_t s,
-                const char *what) {
+int launch_pair(const CUtensorMap &a, const CUtensorMap &b, const CUtensorMap &o,
+                const GemmParams &p, cudaStream_t s, const char *what) {
   using Sh = PairShape<BN>;
   auto kern = grouped_gemm_pair_kernel<MODE, BN>;
   cudaLaunchAttribute at[1];
@@ -799,15 +864,17 @@ int launch_pair(const CUtensorMap &a, const CUtensorMap &b, const GemmParams &p,
     nclusters = n;
   }
   cfg.gridDim = dim3(2 * nclusters);
-  MOE_LAUNCH(kGemmName[MODE], s, cudaLaunchKernelEx(&cfg, kern, a, b, p));
+  MOE_LAUNCH(kGemmName[MODE], s, cudaLaunchKernelEx(&cfg, kern, a, b, o, p));
   return moe::launch_status(what);
 }
 
 // Builds the tensor maps for one GEMM and launches it. A: [a_rows, a_cols] row-major
 // bf16; B likewise. N = output columns (for kGateUp: 2F, in tiles of 128 gate + 128 up).
+// The output p.out is [o_rows, o_cols] row-major bf16.
 template <int MODE>
 int run_gemm(int N, const void *a_base, uint64_t a_rows, uint64_t a_cols, const void *b_base,
-             uint64_t b_rows, uint64_t b_cols, GemmParams p, cudaStream_t s, const char *what) {
+             uint64_t b_rows, uint64_t b_cols, uint64_t o_rows, uint64_t o_cols, GemmParams p,
+             cudaStream_t s, const char *what) {
   using Tr = Traits<MODE>;
   const bool pair = use_pair<MODE>();
   const int BN = (MODE == kGateUp || N % 256 == 0) ? 256 : 128;
@@ -821,12 +888,14 @@ int run_gemm(int N, const void *a_base, uint64_t a_rows, uint64_t a_cols, const 
   if ((st = Tr::B_MN ? make_map(&mb, b_base, b_rows, b_cols, 64, BK, what)
                      : make_map(&mb, b_base, b_rows, b_cols, BK, b_box_rows, what)))
     return st;
+  CUtensorMap mo;  // the epilogue's output, in 32 x 32 chunks
+  if ((st = make_map(&mo, p.out, o_rows, o_cols, 32, 32, what, CU_TENSOR_MAP_SWIZZLE_64B))) return st;
   if (pair) {
-    return BN == 256 ? launch_pair<MODE, 256>(ma, mb, p, s, what)
-                     : launch_pair<MODE, 128>(ma, mb, p, s, what);
+    return BN == 256 ? launch_pair<MODE, 256>(ma, mb, mo, p, s, what)
+                     : launch_pair<MODE, 128>(ma, mb, mo, p, s, what);
   }
-  return BN == 256 ? launch_one<MODE, 256>(ma, mb, p, s, what)
-                   : launch_one<MODE, 128>(ma, mb, p, s, what);
+  return BN == 256 ? launch_one<MODE, 256>(ma, mb, mo, p, s, what)
+                   : launch_one<MODE, 128>(ma, mb, mo, p, s, what);
 }
 
 int check_common(int E, int d, int F, int64_t rows_cap, const char *fn) {
@@ -867,8 +936,8 @@ int moe_grouped_ffn_fwd(const uint16_t *x_perm, const int32_t *group_offsets, in
   p.nkb = d / BK;
   p.out = h;
   p.out2 = ab_saved;
-  if (int st = run_gemm<kGateUp>(2 * F, x_perm, R, d, w_gate_up, uint64_t(E) * 2 * F, d, p, s,
-                                 "moe_grouped_ffn_fwd: gate/up GEMM"))
+  if (int st = run_gemm<kGateUp>(2 * F, x_perm, R, d, w_gate_up, uint64_t(E) * 2 * F, d, R, F, p,
+                                 s, "moe_grouped_ffn_fwd: gate/up GEMM"))
     return st;
   // O = H W_down^T
   GemmParams q{};
@@ -876,7 +945,7 @@ int moe_grouped_ffn_fwd(const uint16_t *x_perm, const int32_t *group_offsets, in
   q.E = E; q.d = d; q.F = F;
   q.nkb = F / BK;
   q.out = out_perm;
-  return run_gemm<kDown>(d, h, R, F, w_down, uint64_t(E) * d, F, q, s,
+  return run_gemm<kDown>(d, h, R, F, w_down, uint64_t(E) * d, F, R, d, q, s,
                          "moe_grouped_ffn_fwd: down GEMM");
 }
 
@@ -898,15 +967,15 @@ int moe_grouped_ffn_bwd_dgrad(const uint16_t *d_out_perm, const uint16_t *ab_sav
   p.nkb = d / BK;
   p.out = d_ab;
   p.aux = ab_saved;
-  if ((st = run_gemm<kDgradDown>(F, d_out_perm, R, d, w_down, uint64_t(E) * d, F, p, s,
-                                 "moe_grouped_ffn_bwd: dH GEMM")))
+  if ((st = run_gemm<kDgradDown>(F, d_out_perm, R, d, w_down, uint64_t(E) * d, F, R, 2 * F, p,
+                                 s, "moe_grouped_ffn_bwd: dH GEMM")))
     return st;
   // dX = [dA | dB] W_gate_up
   p.nkb = 2 * F / BK;
   p.out = dx_perm;
   p.aux = nullptr;
-  return run_gemm<kDgradGateUp>(d, d_ab, R, 2 * F, w_gate_up, uint64_t(E) * 2 * F, d, p, s,
-                                "moe_grouped_ffn_bwd: dX GEMM");
+  return run_gemm<kDgradGateUp>(d, d_ab, R, 2 * F, w_gate_up, uint64_t(E) * 2 * F, d, R, d, p,
+                                s, "moe_grouped_ffn_bwd: dX GEMM");
 }
 
 int moe_grouped_ffn_bwd_wgrad(const uint16_t *d_out_perm, const uint16_t *x_perm,
@@ -927,13 +996,13 @@ int moe_grouped_ffn_bwd_wgrad(const uint16_t *d_out_perm, const uint16_t *x_perm
   p.nkb = 0;
   p.m_tiles_w = d / BM;
   p.out = dw_down;
-  if ((st = run_gemm<kWgradDown>(F, d_out_perm, R, d, h, R, F, p, s,
+  if ((st = run_gemm<kWgradDown>(F, d_out_perm, R, d, h, R, F, uint64_t(E) * d, F, p, s,
                                  "moe_grouped_ffn_bwd: dW_down GEMM")))
     return st;
   // dW_gate_up[e] = [dA | dB]_e^T X_e   ([2F, d])
   p.m_tiles_w = 2 * F / BM;
   p.out = dw_gate_up;
-  return run_gemm<kWgradGateUp>(d, d_ab, R, 2 * F, x_perm, R, d, p, s,
+  return run_gemm<kWgradGateUp>(d, d_ab, R, 2 * F, x_perm, R, d, uint64_t(E) * 2 * F, d, p, s,
                                 "moe_grouped_ffn_bwd: dW_gate_up GEMM");
 }
 

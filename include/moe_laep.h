@@ -109,14 +109,18 @@ size_t moe_workspace_size(int T, int d, int E, int k, int F);
  * uint8 or NULL (all live); logits_in [T,E] fp32 or NULL: when given it
  * replaces x*w_router+bias (x, w_router, bias are then not read; the mask is
  * still applied); logits_out [T,E] fp32 or NULL receives the masked z;
- * topk_idx [T,k] int32; topk_gate [T,k] fp32; counts [E] int32 or NULL.
+ * topk_idx [T,k] int32; topk_gate [T,k] fp32; counts [E] int32 or NULL;
+ * ws, ws_bytes: workspace (moe_workspace_size; may be NULL with logits_in),
+ * it holds the partial logits of the split reduction over d. The logits are
+ * summed in a fixed order, so the routing is deterministic.
  * Limits: 1 <= E <= 256, 1 <= k <= min(E, 8), d % 8 == 0, T >= 0.
  * A token with fewer than k live experts sets MOE_DEV_TOO_FEW_LIVE.
  */
 int moe_route(const uint16_t *x, const float *w_router, const float *bias,
               const uint8_t *active_mask, int T, int d, int E, int k,
               const float *logits_in, float *logits_out, int32_t *topk_idx,
-              float *topk_gate, int32_t *counts, moe_stream_t stream);
+              float *topk_gate, int32_t *counts, void *ws, size_t ws_bytes,
+              moe_stream_t stream);
 
 /*
  * moe_load_stats - per-expert token number of one routing: the ETN statistic

@@ -43,7 +43,7 @@ _SIGS = {
     "moe_timing_read": (I, [ctypes.c_char_p, SZ, I]),
     "moe_perm_rows_max": (I64, [I, I, I]),
     "moe_workspace_size": (SZ, [I, I, I, I, I]),
-    "moe_route": (I, [P, P, P, P, I, I, I, I, P, P, P, P, P, P]),
+    "moe_route": (I, [P, P, P, P, I, I, I, I, P, P, P, P, P, P, SZ, P]),
     "moe_load_stats": (I, [P, I, I, I, P, I, P]),
     "laep_prune_mask": (I, [P, I, I64, I, D, D, I, P, P]),
     "laep_layer_alpha": (D, [I, I, D, D]),
@@ -147,10 +147,11 @@ def moe_timing_read(reset=True):
 
 
 def moe_route(x, w_router, bias, active_mask, T, d, E, k, logits_in, logits_out, topk_idx,
-              topk_gate, counts, stream=None):
+              topk_gate, counts, ws=None, ws_bytes=0, stream=None):
     _check("moe_route", load().moe_route(
         _ptr(x), _ptr(w_router), _ptr(bias), _ptr(active_mask), T, d, E, k, _ptr(logits_in),
-        _ptr(logits_out), _ptr(topk_idx), _ptr(topk_gate), _ptr(counts), _stream(stream)))
+        _ptr(logits_out), _ptr(topk_idx), _ptr(topk_gate), _ptr(counts), _ptr(ws), ws_bytes,
+        _stream(stream)))
 
 
 def moe_load_stats(topk_idx, T, k, E, counts, accumulate=False, stream=None):

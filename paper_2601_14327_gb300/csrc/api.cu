@@ -113,6 +113,8 @@ WsLayout ws_layout(int T, int d, int E, int k, int F) {
   off += align256(size_t(rows / kGroupPad) * d * 4);
   w.w_router_t = off;
   off += align256(size_t(E) * d * 4);
+  w.route_partial = off;
+  off += align256(route_partial_bytes(T, d, E));
   w.total = off;
   return w;
 }

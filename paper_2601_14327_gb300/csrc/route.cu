@@ -13,21 +13,36 @@ MOE_DEV_ERR_DECL
 namespace {
 
 constexpr int kRouteThreads = 256;
-constexpr int kBM = 64;  // tokens per CTA
+constexpr int kRouteBK = 16;            // reduction chunk of the logit contraction
+constexpr int kRouteTargetCtas = 304;   // split the reduction until about this many CTAs
 
-// Padded expert count NE (multiple of 64). 16 x 16 threads: thread (tx, ty) owns
-// tokens ty*4 .. ty*4+3 and experts j*64 + tx*4 + q (j < NE/64, q < 4), so the
-// shared-memory reads of one row of W are contiguous float4s across tx.
+// Logits kernel shape for the padded expert count NE (multiple of 64). Thread
+// (eg, tg) owns 8 tokens (tg*8 ..) and 8 experts {j*4*EG + eg*4 + q : j < 2,
+// q < 4}: per k it reads 8 x values and 8 W values as float4s (0.5-1 byte of
+// shared memory per FFMA; the float4 reads of one W row are contiguous across
+// eg) and keeps 64 accumulators, so two CTAs fit on an SM (<= 128 registers).
 template <int NE> struct RouteShape {
-  static constexpr int BK = NE <= 128 ? 32 : 16;  // reduction chunk (registers stage one)
-  static constexpr int TN = NE / 16;   // experts per thread
-  static constexpr int TM = 4;         // tokens per thread
-  static constexpr int LDL = NE + 1;   // logits row stride in shared memory
-  static constexpr size_t kStage = size_t(BK) * kBM * 4 + size_t(BK) * NE * 4;
-  static constexpr size_t kGemmSmem = 2 * kStage;
-  static constexpr size_t kLogitSmem = size_t(kBM) * LDL * 4;
-  static constexpr size_t kSmem = (kGemmSmem > kLogitSmem ? kGemmSmem : kLogitSmem) + NE * 4;
+  static constexpr int EG = NE / 8;                       // threads along the experts
+  static constexpr int THREADS = NE == 192 ? 384 : 256;
+  static constexpr int TN = 8;                            // experts per thread
+  static constexpr int TG = THREADS / EG;                 // threads along the tokens
+  static constexpr int TM = 8;                            // tokens per thread
+  static constexpr int BM = TG * TM;                      // tokens per CTA
+  static constexpr int MIN_BLOCKS = NE == 192 ? 1 : 2;
+  static constexpr size_t kStage = size_t(kRouteBK) * BM * 4 + size_t(kRouteBK) * NE * 4;
+  static constexpr size_t kSmem = 2 * kStage;
 };
+
+// Reduction split so that T/BM token tiles give about kRouteTargetCtas CTAs (at
+// most 8, never more CTAs than that target); fixed by (T, NE) alone, so the
+// workspace size is too.
+template <int NE> int route_splits(int T, int d) {
+  const int tiles = (T + RouteShape<NE>::BM - 1) / RouteShape<NE>::BM;
+  const int chunks = (d + kRouteBK - 1) / kRouteBK;
+  const int s = kRouteTargetCtas / std::max(tiles, 1);
+  return std::max(1, std::min({s, 8, chunks}));
+}
+int padded_experts(int E) { return E <= 64 ? 64 : (E <= 128 ? 128 : (E <= 192 ? 192 : 256)); }
 
 __device__ __forceinline__ bool better(float v, int e, float bv, int be) {
   return v > bv || (v == bv && e < be);
@@ -37,128 +52,137 @@ __global__ void zero_i32_kernel(int32_t *p, int n) {
   for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < n; i += gridDim.x * blockDim.x) p[i] = 0;
 }
 
-// One CTA: 64 tokens x all experts. Logits by FFMA in fp32 (x converted from
-// bf16 exactly) with the next k-chunk prefetched into registers while the
-// current one is multiplied; then one warp per token runs k rounds of a warp
-// arg-max over the logits row.
+// partial[split][t][e] = sum over this split's k range of x[t,k] * W_r[k,e]
+// (fp32 FFMA, x converted from bf16 exactly; columns e >= E are zero). The next
+// k-chunk is loaded into registers while the current one is multiplied.
 template <int NE>
-__global__ void __launch_bounds__(kRouteThreads) route_kernel(
-    const uint16_t *__restrict__ x, const float *__restrict__ w_router,
-    const float *__restrict__ bias, const uint8_t *__restrict__ active_mask, int T, int d, int E,
-    int k, const float *__restrict__ logits_in, float *__restrict__ logits_out,
-    int32_t *__restrict__ topk_idx, float *__restrict__ topk_gate, int32_t *__restrict__ counts) {
+__global__ void __launch_bounds__(RouteShape<NE>::THREADS, RouteShape<NE>::MIN_BLOCKS)
+    route_logits_kernel(
+    const uint16_t *__restrict__ x, const float *__restrict__ w_router, int T, int d, int E,
+    int k_per_split, float *__restrict__ partial) {
   using S = RouteShape<NE>;
-  constexpr int TM = S::TM, TN = S::TN, LDL = S::LDL, BM = kBM, kBK = S::BK;
-  constexpr int WPT = kBK * NE / kRouteThreads;  // W elements each thread stages per chunk
+  constexpr int TM = S::TM, TN = S::TN, EG = S::EG, BM = S::BM, BK = kRouteBK, NT = S::THREADS;
+  constexpr int XN = BM * BK / 8;             // 16-byte x loads per chunk
+  constexpr int XV = (XN + NT - 1) / NT;      // ... per thread
+  constexpr int WV = BK * NE / NT;            // W values per thread per chunk
   extern __shared__ __align__(16) float smem[];
-  float *Ls = smem;  // [BM][LDL] (reuses the staging buffers)
-  int *hist = reinterpret_cast<int *>(
-      smem + (S::kGemmSmem > S::kLogitSmem ? S::kGemmSmem : S::kLogitSmem) / 4);
-
   const int tid = threadIdx.x;
+  const int eg = tid % EG, tg = tid / EG;
   const int t0 = blockIdx.x * BM;
-  for (int e = tid; e < NE; e += kRouteThreads) hist[e] = 0;
+  const int kb = blockIdx.y * k_per_split, ke = min(d, kb + k_per_split);
 
-  if (logits_in == nullptr) {
-    const int tx = tid & 15, ty = tid >> 4;
-    float acc[TM][TN];
+  float acc[TM][TN];
 #pragma unroll
-    for (int i = 0; i < TM; ++i)
+  for (int i = 0; i < TM; ++i)
 #pragma unroll
-      for (int j = 0; j < TN; ++j) acc[i][j] = 0.f;
-    // register staging of one chunk: x (threads 0..127: one row, 8 columns) and W
-    float xr[8];
-    float wr[WPT];
-    constexpr int XSEG = kBK / 8;  // 16-byte segments of x per row and chunk
-    const int xrow = tid / XSEG, xcol = (tid % XSEG) * 8;
-    auto load_chunk = [&](int k0) {
-      if (tid < BM * kBK / 8) {
-        if (t0 + xrow < T && k0 + xcol < d) {
-          unpack8(ldg_nc_v4(x + size_t(t0 + xrow) * d + k0 + xcol), xr);
-        } else {
+    for (int j = 0; j < TN; ++j) acc[i][j] = 0.f;
+  float xr[XV][8], wr[WV];
+  auto load_chunk = [&](int k0) {
 #pragma unroll
-          for (int q = 0; q < 8; ++q) xr[q] = 0.f;
-        }
+    for (int i = 0; i < XV; ++i) {
+      const int v = tid + i * NT;
+      const int row = v / (BK / 8), col = (v % (BK / 8)) * 8;
+      if (v < XN && t0 + row < T && k0 + col < ke) {
+        unpack8(ldg_nc_v4(x + size_t(t0 + row) * d + k0 + col), xr[i]);
+      } else {
+#pragma unroll
+        for (int q = 0; q < 8; ++q) xr[i][q] = 0.f;
       }
+    }
 #pragma unroll
-      for (int i = 0; i < WPT; ++i) {
-        const int v = tid + i * kRouteThreads;
-        const int kk = v / NE, e = v % NE;
-        wr[i] = (e < E && k0 + kk < d) ? __ldg(w_router + size_t(k0 + kk) * E + e) : 0.f;
+    for (int i = 0; i < WV; ++i) {
+      const int v = tid + i * NT;
+      const int kk = v / NE, e = v % NE;
+      wr[i] = (e < E && k0 + kk < ke) ? __ldg(w_router + size_t(k0 + kk) * E + e) : 0.f;
+    }
+  };
+  auto store_chunk = [&](int buf) {
+    float *Xs = smem + buf * (S::kStage / 4);  // [BK][BM]
+    float *Ws = Xs + BK * BM;                  // [BK][NE]
+#pragma unroll
+    for (int i = 0; i < XV; ++i) {
+      const int v = tid + i * NT;
+      const int row = v / (BK / 8), col = (v % (BK / 8)) * 8;
+      if (v < XN) {
+#pragma unroll
+        for (int q = 0; q < 8; ++q) Xs[(col + q) * BM + row] = xr[i][q];
       }
-    };
-    auto store_chunk = [&](int buf) {
-      float *Xs = smem + buf * (S::kStage / 4);  // [kBK][BM]
-      float *Ws = Xs + kBK * BM;                 // [kBK][NE]
-      if (tid < BM * kBK / 8) {
+    }
 #pragma unroll
-        for (int q = 0; q < 8; ++q) Xs[(xcol + q) * BM + xrow] = xr[q];
-      }
-#pragma unroll
-      for (int i = 0; i < WPT; ++i) Ws[tid + i * kRouteThreads] = wr[i];
-    };
-    const int nchunks = (d + kBK - 1) / kBK;
-    load_chunk(0);
+    for (int i = 0; i < WV; ++i) Ws[tid + i * NT] = wr[i];
+  };
+  const int nchunks = (ke - kb + BK - 1) / BK;
+  if (nchunks > 0) {
+    load_chunk(kb);
     store_chunk(0);
-    __syncthreads();
-    for (int ch = 0; ch < nchunks; ++ch) {
-      if (ch + 1 < nchunks) load_chunk((ch + 1) * kBK);
-      const float *Xs = smem + (ch & 1) * (S::kStage / 4);
-      const float *Ws = Xs + kBK * BM;
+  }
+  __syncthreads();
+  for (int ch = 0; ch < nchunks; ++ch) {
+    if (ch + 1 < nchunks) load_chunk(kb + (ch + 1) * BK);
+    const float *Xs = smem + (ch & 1) * (S::kStage / 4);
+    const float *Ws = Xs + BK * BM;
 #pragma unroll
-      for (int kk = 0; kk < kBK; ++kk) {
-        const float4 xv = *reinterpret_cast<const float4 *>(&Xs[kk * BM + ty * TM]);
-        const float xs[4] = {xv.x, xv.y, xv.z, xv.w};
+    for (int kk = 0; kk < BK; ++kk) {
+      const float4 x0 = *reinterpret_cast<const float4 *>(&Xs[kk * BM + tg * TM]);
+      const float4 x1 = *reinterpret_cast<const float4 *>(&Xs[kk * BM + tg * TM + 4]);
+      const float xs[8] = {x0.x, x0.y, x0.z, x0.w, x1.x, x1.y, x1.z, x1.w};
 #pragma unroll
-        for (int j4 = 0; j4 < NE / 64; ++j4) {
-          const float4 wv = *reinterpret_cast<const float4 *>(&Ws[kk * NE + j4 * 64 + tx * 4]);
-          const float ws[4] = {wv.x, wv.y, wv.z, wv.w};
+      for (int j4 = 0; j4 < TN / 4; ++j4) {
+        const float4 wv = *reinterpret_cast<const float4 *>(&Ws[kk * NE + j4 * 4 * EG + eg * 4]);
+        const float ws[4] = {wv.x, wv.y, wv.z, wv.w};
 #pragma unroll
-          for (int i = 0; i < TM; ++i)
+        for (int i = 0; i < TM; ++i)
 #pragma unroll
-            for (int q = 0; q < 4; ++q) acc[i][j4 * 4 + q] = fmaf(xs[i], ws[q], acc[i][j4 * 4 + q]);
-        }
+          for (int q = 0; q < 4; ++q) acc[i][j4 * 4 + q] = fmaf(xs[i], ws[q], acc[i][j4 * 4 + q]);
       }
-      if (ch + 1 < nchunks) store_chunk((ch + 1) & 1);
-      __syncthreads();
     }
+    if (ch + 1 < nchunks) store_chunk((ch + 1) & 1);
+    __syncthreads();
+  }
+  float *out = partial + size_t(blockIdx.y) * T * NE;
 #pragma unroll
-    for (int j = 0; j < TN; ++j) {
-      const int e = (j >> 2) * 64 + tx * 4 + (j & 3);
-      const float b = (bias != nullptr && e < E) ? bias[e] : 0.f;
-#pragma unroll
-      for (int i = 0; i < TM; ++i) Ls[(ty * TM + i) * LDL + e] = acc[i][j] + b;
-    }
-  } else {
-    for (int v = tid; v < BM * NE; v += kRouteThreads) {
-      const int r = v / NE, e = v % NE;
-      Ls[r * LDL + e] = (t0 + r < T && e < E) ? logits_in[size_t(t0 + r) * E + e] : 0.f;
-    }
-  }
-  __syncthreads();
-  // Pruned experts and padding columns can never win.
-  for (int v = tid; v < BM * NE; v += kRouteThreads) {
-    const int r = v / NE, e = v % NE;
-    if (e >= E || (active_mask != nullptr && active_mask[e] == 0)) Ls[r * LDL + e] = -INFINITY;
-  }
-  __syncthreads();
-  if (logits_out != nullptr) {
-    for (int v = tid; v < BM * E; v += kRouteThreads) {
-      const int r = v / E, e = v % E;
-      if (t0 + r < T) logits_out[size_t(t0 + r) * E + e] = Ls[r * LDL + e];
-    }
-  }
-
-  // Top-k per token: warp w handles tokens w, w+8, ...
-  const int tx = tid & 31, ty = tid >> 5;
-  for (int m = ty; m < BM; m += 8) {
-    const int t = t0 + m;
+  for (int i = 0; i < TM; ++i) {
+    const int t = t0 + tg * TM + i;
     if (t >= T) break;
-    constexpr int TK = NE / 32;  // logits per lane
-    float v[TK];
-    unsigned taken = 0;
 #pragma unroll
-    for (int j = 0; j < TK; ++j) v[j] = Ls[m * LDL + tx + 32 * j];
+    for (int j4 = 0; j4 < TN / 4; ++j4)
+      *reinterpret_cast<float4 *>(out + size_t(t) * NE + j4 * 4 * EG + eg * 4) =
+          make_float4(acc[i][j4 * 4], acc[i][j4 * 4 + 1], acc[i][j4 * 4 + 2], acc[i][j4 * 4 + 3]);
+  }
+}
+
+// One warp per token: logits = sum of the split partials (fixed order) + bias,
+// pruned experts -inf, k rounds of a warp arg-max (ties to the lower index),
+// softmax over the selected logits, per-expert histogram.
+template <int NE>
+__global__ void __launch_bounds__(kRouteThreads) route_topk_kernel(
+    const float *__restrict__ partial, int splits, const float *__restrict__ logits_in,
+    const float *__restrict__ bias, const uint8_t *__restrict__ active_mask, int T, int E, int k,
+    float *__restrict__ logits_out, int32_t *__restrict__ topk_idx, float *__restrict__ topk_gate,
+    int32_t *__restrict__ counts) {
+  constexpr int TK = NE / 32;  // logits per lane
+  __shared__ int hist[NE];
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  for (int e = tid; e < NE; e += kRouteThreads) hist[e] = 0;
+  __syncthreads();
+  const int t = blockIdx.x * (kRouteThreads / 32) + warp;
+  if (t < T) {
+    float v[TK];
+#pragma unroll
+    for (int j = 0; j < TK; ++j) {
+      const int e = lane + 32 * j;
+      float z = 0.f;
+      if (logits_in != nullptr) {
+        z = e < E ? logits_in[size_t(t) * E + e] : 0.f;
+      } else {
+        for (int y = 0; y < splits; ++y) z += partial[(size_t(y) * T + t) * NE + e];
+        if (bias != nullptr && e < E) z += bias[e];
+      }
+      if (e >= E || (active_mask != nullptr && active_mask[e] == 0)) z = -INFINITY;
+      v[j] = z;
+      if (logits_out != nullptr && e < E) logits_out[size_t(t) * E + e] = z;
+    }
+    unsigned taken = 0;
     float sel_v[8];
     int sel_e[8];
 #pragma unroll
@@ -168,7 +192,7 @@ __global__ void __launch_bounds__(kRouteThreads) route_kernel(
       int be = 0x7fffffff;
 #pragma unroll
       for (int j = 0; j < TK; ++j) {
-        const int e = tx + 32 * j;
+        const int e = lane + 32 * j;
         if (e < E && !((taken >> j) & 1u) && better(v[j], e, bv, be)) { bv = v[j]; be = e; }
       }
 #pragma unroll
@@ -177,25 +201,26 @@ __global__ void __launch_bounds__(kRouteThreads) route_kernel(
         const int oe = __shfl_xor_sync(0xffffffffu, be, off);
         if (better(ov, oe, bv, be)) { bv = ov; be = oe; }
       }
-      if ((be & 31) == tx) taken |= 1u << (be >> 5);
+      if ((be & 31) == lane) taken |= 1u << (be >> 5);
       sel_v[s] = bv;
       sel_e[s] = be;
     }
     // softmax over the selected logits (renormalised top-k), fp32
     const float zmax = sel_v[0];
     float den = 0.f, ex[8];
-#pragma unroll
-    for (int s = 0; s < 8; ++s) {
-      if (s < k) { ex[s] = expf(sel_v[s] - zmax); den += ex[s]; }
-    }
     bool too_few = false;
 #pragma unroll
-    for (int s = 0; s < 8; ++s)
-      if (s < k && sel_v[s] == -INFINITY) too_few = true;
-    if (tx == 0 && too_few) dev_flag(&g_dev_err, MOE_DEV_TOO_FEW_LIVE);
+    for (int s = 0; s < 8; ++s) {
+      if (s < k) {
+        ex[s] = expf(sel_v[s] - zmax);
+        den += ex[s];
+        if (sel_v[s] == -INFINITY) too_few = true;
+      }
+    }
+    if (lane == 0 && too_few) dev_flag(&g_dev_err, MOE_DEV_TOO_FEW_LIVE);
 #pragma unroll
     for (int s = 0; s < 8; ++s) {
-      if (s < k && tx == s) {
+      if (s < k && lane == s) {
         topk_idx[size_t(t) * k + s] = sel_e[s];
         topk_gate[size_t(t) * k + s] = ex[s] / den;
         if (sel_e[s] >= 0 && sel_e[s] < E) atomicAdd(&hist[sel_e[s]], 1);
@@ -305,33 +330,56 @@ __global__ void route_bwd_reduce_kernel(const float *__restrict__ partial,
 template <int NE>
 int launch_route(const uint16_t *x, const float *w, const float *b, const uint8_t *mask, int T,
                  int d, int E, int k, const float *lin, float *lout, int32_t *idx, float *gate,
-                 int32_t *counts, cudaStream_t s) {
+                 int32_t *counts, float *partial, cudaStream_t s) {
   using S = RouteShape<NE>;
-  static bool attr_set = false;
-  if (!attr_set) {
-    cudaError_t e = cudaFuncSetAttribute(route_kernel<NE>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, int(S::kSmem));
-    if (e != cudaSuccess) return moe::cuda_status(e, "moe_route: set smem attribute");
-    attr_set = true;
+  int splits = 0;
+  if (lin == nullptr) {
+    static bool attr_set = false;
+    if (!attr_set) {
+      cudaError_t e = cudaFuncSetAttribute(route_logits_kernel<NE>,
+                                           cudaFuncAttributeMaxDynamicSharedMemorySize, int(S::kSmem));
+      if (e != cudaSuccess) return moe::cuda_status(e, "moe_route: set smem attribute");
+      attr_set = true;
+    }
+    splits = route_splits<NE>(T, d);
+    const int chunks = (d + kRouteBK - 1) / kRouteBK;
+    const int k_per_split = ((chunks + splits - 1) / splits) * kRouteBK;
+    dim3 grid((T + S::BM - 1) / S::BM, splits);
+    MOE_LAUNCH("route_logits", s, route_logits_kernel<NE><<<grid, S::THREADS, S::kSmem, s>>>(
+                                      x, w, T, d, E, k_per_split, partial));
+    if (int st = moe::launch_status("moe_route: logits")) return st;
   }
-  const int grid = (T + kBM - 1) / kBM;
-  MOE_LAUNCH("route", s, route_kernel<NE><<<grid, kRouteThreads, S::kSmem, s>>>(x, w, b, mask, T, d, E, k, lin, lout,
-                                                        idx, gate, counts));
-  return moe::launch_status("moe_route: launch");
+  const int grid2 = (T + kRouteThreads / 32 - 1) / (kRouteThreads / 32);
+  MOE_LAUNCH("route_topk", s, route_topk_kernel<NE><<<grid2, kRouteThreads, 0, s>>>(
+                                  partial, splits, lin, b, mask, T, E, k, lout, idx, gate, counts));
+  return moe::launch_status("moe_route: top-k");
 }
 
 }  // namespace
 
 namespace moe {
 MOE_DEV_ERR_DEFINE_READER(route_dev_error)
+
+size_t route_partial_bytes(int T, int d, int E) {
+  if (T <= 0) return 0;
+  const int NE = padded_experts(E);
+  int splits = 1;
+  switch (NE) {
+    case 64: splits = route_splits<64>(T, d); break;
+    case 128: splits = route_splits<128>(T, d); break;
+    case 192: splits = route_splits<192>(T, d); break;
+    default: splits = route_splits<256>(T, d); break;
+  }
+  return size_t(splits) * size_t(T) * size_t(NE) * 4;
+}
 }
 
 extern "C" {
 
 int moe_route(const uint16_t *x, const float *w_router, const float *bias,
               const uint8_t *active_mask, int T, int d, int E, int k, const float *logits_in,
-              float *logits_out, int32_t *topk_idx, float *topk_gate, int32_t *counts,
-              moe_stream_t stream) {
+              float *logits_out, int32_t *topk_idx, float *topk_gate, int32_t *counts, void *ws,
+              size_t ws_bytes, moe_stream_t stream) {
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   if (E < 1 || E > 256) return moe::set_error(MOE_ERR_UNSUPPORTED, "moe_route: E=%d not in [1,256]", E);
   if (k < 1 || k > 8 || k > E) return moe::set_error(MOE_ERR_UNSUPPORTED, "moe_route: k=%d", k);
@@ -339,15 +387,24 @@ int moe_route(const uint16_t *x, const float *w_router, const float *bias,
   if (!topk_idx || !topk_gate) return moe::set_error(MOE_ERR_ARG, "moe_route: null output");
   if (!logits_in && (!x || !w_router)) return moe::set_error(MOE_ERR_ARG, "moe_route: null x/w_router");
   if (x && !moe::aligned16(x)) return moe::set_error(MOE_ERR_ARG, "moe_route: x not 16-byte aligned");
+  float *partial = nullptr;
+  if (!logits_in) {
+    const moe::WsLayout L = moe::ws_layout(T, d, E, k, 0);
+    if (!ws || ws_bytes < L.total) return moe::set_error(MOE_ERR_WORKSPACE, "moe_route: workspace");
+    if (!moe::aligned16(ws)) return moe::set_error(MOE_ERR_ARG, "moe_route: ws alignment");
+    partial = reinterpret_cast<float *>(static_cast<char *>(ws) + L.route_partial);
+  }
   if (counts) {
     MOE_LAUNCH("zero_counts", s, zero_i32_kernel<<<1, 256, 0, s>>>(counts, E));
     if (int st = moe::launch_status("moe_route: zero counts")) return st;
   }
   if (T == 0) return MOE_OK;
-  if (E <= 64) return launch_route<64>(x, w_router, bias, active_mask, T, d, E, k, logits_in, logits_out, topk_idx, topk_gate, counts, s);
-  if (E <= 128) return launch_route<128>(x, w_router, bias, active_mask, T, d, E, k, logits_in, logits_out, topk_idx, topk_gate, counts, s);
-  if (E <= 192) return launch_route<192>(x, w_router, bias, active_mask, T, d, E, k, logits_in, logits_out, topk_idx, topk_gate, counts, s);
-  return launch_route<256>(x, w_router, bias, active_mask, T, d, E, k, logits_in, logits_out, topk_idx, topk_gate, counts, s);
+  switch (padded_experts(E)) {
+    case 64: return launch_route<64>(x, w_router, bias, active_mask, T, d, E, k, logits_in, logits_out, topk_idx, topk_gate, counts, partial, s);
+    case 128: return launch_route<128>(x, w_router, bias, active_mask, T, d, E, k, logits_in, logits_out, topk_idx, topk_gate, counts, partial, s);
+    case 192: return launch_route<192>(x, w_router, bias, active_mask, T, d, E, k, logits_in, logits_out, topk_idx, topk_gate, counts, partial, s);
+    default: return launch_route<256>(x, w_router, bias, active_mask, T, d, E, k, logits_in, logits_out, topk_idx, topk_gate, counts, partial, s);
+  }
 }
 
 int moe_load_stats(const int32_t *topk_idx, int T, int k, int E, int32_t *counts, int accumulate,

@@ -68,7 +68,8 @@ def route(b: MoELayerBuffers, x, w_router, bias, active_mask=None, logits_in=Non
           keep_logits: bool = False, stream=None):
     s = b.shape
     L.moe_route(x, w_router, bias, active_mask, s.T, s.d, s.E, s.k, logits_in,
-                b.logits if keep_logits else None, b.topk_idx, b.topk_gate, b.counts, stream)
+                b.logits if keep_logits else None, b.topk_idx, b.topk_gate, b.counts, b.ws,
+                b.ws_bytes, stream)
 
 
 def forward(b: MoELayerBuffers, x, w_router, bias, w_gate_up, w_down, active_mask=None,

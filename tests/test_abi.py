@@ -71,10 +71,10 @@ def test_laep_prune_mask_matches_oracle_random(lib):
 def test_argument_validation_without_launch(lib):
     # E too large, k too large, d not a multiple of 128: rejected on the host
     with pytest.raises(L.MoEError) as e:
-        L.moe_route(None, None, None, None, 10, 64, 300, 2, 1, None, 1, 1, None, stream=0)
+        L.moe_route(None, None, None, None, 10, 64, 300, 2, 1, None, 1, 1, None, None, 0, stream=0)
     assert e.value.status == -2
     with pytest.raises(L.MoEError) as e:
-        L.moe_route(None, None, None, None, 10, 64, 16, 9, 1, None, 1, 1, None, stream=0)
+        L.moe_route(None, None, None, None, 10, 64, 16, 9, 1, None, 1, 1, None, None, 0, stream=0)
     assert e.value.status == -2
     with pytest.raises(L.MoEError) as e:
         L.moe_grouped_ffn_fwd(16, 16, 8, 100, 256, 4096, 16, 16, 16, 16, 16, 16, 0, stream=0)

@@ -151,7 +151,8 @@ __global__ void __launch_bounds__(kThreads) perm_gather_kernel(
   }
 }
 
-// Zero the padding rows [group_offsets[e] + group_counts[e], group_offsets[e+1]).
+// Zero the padding rows [group_offsets[e] + group_counts[e], group_offsets[e+1]);
+// blockIdx.x = expert, blockIdx.y splits that expert's padding rows.
 __global__ void __launch_bounds__(kThreads) pad_zero_kernel(const int32_t *__restrict__ group_offsets,
                                                             const int32_t *__restrict__ group_counts,
                                                             int E, int d, int64_t rows_cap,
@@ -161,11 +162,15 @@ __global__ void __launch_bounds__(kThreads) pad_zero_kernel(const int32_t *__res
   const int r1 = int(min((long long)group_offsets[e + 1], (long long)rows_cap));
   const int nv = d / 8;
   const uint4 z = make_uint4(0, 0, 0, 0);
-  for (int64_t i = threadIdx.x; i < int64_t(r1 - r0) * nv; i += kThreads) {
+  const int64_t n = int64_t(r1 - r0) * nv;
+  for (int64_t i = int64_t(blockIdx.y) * kThreads + threadIdx.x; i < n;
+       i += int64_t(gridDim.y) * kThreads) {
     const int64_t r = r0 + i / nv, c = i % nv;
     stg_v4(buf + size_t(r) * d + c * 8, z);
   }
 }
+
+constexpr int kPadSplit = 8;  // blocks per expert in pad_zero_kernel
 
 // y[t] = sum_j g[t,j] * out_perm[row(t,j)]  (fp32 sum, one bf16 rounding)
 __global__ void __launch_bounds__(kThreads) combine_kernel(
@@ -370,7 +375,7 @@ int moe_permute(const uint16_t *x, const int32_t *topk_idx, const int32_t *count
                                                          x_perm));
     if (int st = moe::launch_status("moe_permute: gather")) return st;
   }
-  MOE_LAUNCH("pad_zero", s, pad_zero_kernel<<<E, kThreads, 0, s>>>(group_offsets, group_counts, E, d, rows_cap, x_perm));
+  MOE_LAUNCH("pad_zero", s, pad_zero_kernel<<<dim3(E, kPadSplit), kThreads, 0, s>>>(group_offsets, group_counts, E, d, rows_cap, x_perm));
   return moe::launch_status("moe_permute: pad");
 }
 
@@ -407,7 +412,7 @@ int moe_unpermute_combine_bwd(const uint16_t *dy, const uint16_t *out_perm,
                                                          T, d, k, rows_cap, d_out_perm, d_gate));
     if (int st = moe::launch_status("moe_unpermute_combine_bwd: launch")) return st;
   }
-  MOE_LAUNCH("pad_zero", s, pad_zero_kernel<<<E, kThreads, 0, s>>>(group_offsets, group_counts, E, d, rows_cap, d_out_perm));
+  MOE_LAUNCH("pad_zero", s, pad_zero_kernel<<<dim3(E, kPadSplit), kThreads, 0, s>>>(group_offsets, group_counts, E, d, rows_cap, d_out_perm));
   return moe::launch_status("moe_unpermute_combine_bwd: pad");
 }
 
@@ -522,7 +527,7 @@ extern "C" int moe_permute_noalloc(const uint16_t *x, const int32_t *topk_idx,
                                      x, row_of_assignment, T, d, k, rows_cap, x_perm));
     if (int st = moe::launch_status("moe_permute_noalloc: gather")) return st;
   }
-  MOE_LAUNCH("pad_zero", s, pad_zero_kernel<<<E, kThreads, 0, s>>>(group_offsets, group_counts, E,
+  MOE_LAUNCH("pad_zero", s, pad_zero_kernel<<<dim3(E, kPadSplit), kThreads, 0, s>>>(group_offsets, group_counts, E,
                                                                     d, rows_cap, x_perm));
   return moe::launch_status("moe_permute_noalloc: pad");
 }

@@ -384,11 +384,12 @@ int moe_route(const uint16_t *x, const float *w_router, const float *bias,
   if (E < 1 || E > 256) return moe::set_error(MOE_ERR_UNSUPPORTED, "moe_route: E=%d not in [1,256]", E);
   if (k < 1 || k > 8 || k > E) return moe::set_error(MOE_ERR_UNSUPPORTED, "moe_route: k=%d", k);
   if (T < 0 || d <= 0 || d % 8) return moe::set_error(MOE_ERR_ARG, "moe_route: T=%d d=%d", T, d);
-  if (!topk_idx || !topk_gate) return moe::set_error(MOE_ERR_ARG, "moe_route: null output");
-  if (!logits_in && (!x || !w_router)) return moe::set_error(MOE_ERR_ARG, "moe_route: null x/w_router");
+  if (T > 0 && (!topk_idx || !topk_gate)) return moe::set_error(MOE_ERR_ARG, "moe_route: null output");
+  if (T > 0 && !logits_in && (!x || !w_router))
+    return moe::set_error(MOE_ERR_ARG, "moe_route: null x/w_router");
   if (x && !moe::aligned16(x)) return moe::set_error(MOE_ERR_ARG, "moe_route: x not 16-byte aligned");
   float *partial = nullptr;
-  if (!logits_in) {
+  if (!logits_in && T > 0) {
     const moe::WsLayout L = moe::ws_layout(T, d, E, k, 0);
     if (!ws || ws_bytes < L.total) return moe::set_error(MOE_ERR_WORKSPACE, "moe_route: workspace");
     if (!moe::aligned16(ws)) return moe::set_error(MOE_ERR_ARG, "moe_route: ws alignment");
@@ -432,8 +433,8 @@ int moe_route_bwd(const uint16_t *x_perm, const int32_t *topk_idx, const float *
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   if (E < 1 || E > 256 || k < 1 || k > 8 || T < 0 || d <= 0 || d % 8)
     return moe::set_error(MOE_ERR_ARG, "moe_route_bwd: sizes");
-  if (!x_perm || !topk_gate || !d_gate || !row_of_assignment || !group_offsets ||
-      !group_counts || !d_logits || !dw_router || !ws)
+  if (!x_perm || !group_offsets || !group_counts || !dw_router || !ws ||
+      (T > 0 && (!topk_gate || !d_gate || !row_of_assignment || !d_logits)))
     return moe::set_error(MOE_ERR_ARG, "moe_route_bwd: null pointer");
   if (rows_cap < moe_perm_rows_max(T, k, E))
     return moe::set_error(MOE_ERR_ARG, "moe_route_bwd: rows_cap too small");

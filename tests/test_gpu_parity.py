@@ -171,6 +171,9 @@ def test_permute_flags_count_mismatch():
 LAYER_CASES = [
     # T, d, E, k, F, bias, n_masked
     (512, 256, 16, 2, 512, "none", 0),        # the tiny workload
+    (300, 128, 1, 1, 128, "none", 0),         # one expert, k=1: a dense SwiGLU MLP; N=128 tiles,
+                                              # a weight-gradient pair with one row block
+    (1, 256, 4, 2, 256, "zipf", 0),           # a single token
     (1500, 384, 12, 4, 640, "zipf", 3),       # ragged groups, BN=128 paths, empty groups
     (700, 512, 8, 8, 256, "zipf", 0),         # k = number of experts
     (2100, 256, 32, 2, 384, "loguniform", 0), # volatile load, several empty experts
@@ -266,3 +269,43 @@ def test_etn_history_recorded_on_device_drives_algorithm_1():
     m, n = L.laep_prune_layers(got, T, k, alphas, 0.1)
     om, on = O.prune_layers(etn_ref, T, k, alphas, 0.1)
     assert (m == om).all() and (n == on).all()
+
+
+def test_layer_all_tokens_to_one_expert():
+    """A bias that sends every token to one expert: one group, seven empty ones."""
+    T, d, E, k, F = 900, 256, 8, 1, 256
+    inp = case_inputs(T, d, E, k, F, bias="none", seed=77)
+    inp["bias"][3] = 30.0
+    o = oracle_inputs(inp)
+    z = O.router_logits(o["x"], o["w_router"], o["bias"])
+    ref = O.moe_layer(o["x"], o["w_router"], o["bias"], None, k, o["w_gate_up"], o["w_down"],
+                      dy=o["dy"], logits32=z)
+    assert (ref["topk_idx"] == 3).all()
+    b = run_gpu_layer(inp, E, k, logits_in=z)
+    assert (b.topk_idx.cpu().numpy() == 3).all()
+    assert_close("y", to_np(b.y), ref["y"])
+    assert_close("dx", to_np(b.dx), ref["dx"])
+    assert_close("dw_gate_up", to_np(b.dw_gate_up), ref["dw_gate_up"])
+    assert_close("dw_down", to_np(b.dw_down), ref["dw_down"])
+    for e in range(E):
+        if e != 3:
+            assert not b.dw_gate_up[e].any() and not b.dw_down[e].any()
+
+
+def test_layer_without_tokens():
+    """T = 0: nothing is routed; every weight gradient is exactly zero."""
+    T, d, E, k, F = 0, 256, 4, 2, 256
+    inp = case_inputs(1, d, E, k, F, seed=3)
+    inp["x"] = inp["x"][:0].contiguous()
+    inp["dy"] = inp["dy"][:0].contiguous()
+    dev = "cuda"
+    g = {n: v.to(dev) for n, v in inp.items()}
+    b = layer.MoELayerBuffers(layer.LayerShape(T, d, E, k, F), dev)
+    b.dw_gate_up.fill_(1.0)
+    b.dw_down.fill_(1.0)
+    b.dw_router.fill_(1.0)
+    layer.forward(b, g["x"], g["w_router"], g["bias"], g["w_gate_up"], g["w_down"])
+    layer.backward(b, g["dy"], g["w_router"], g["w_gate_up"], g["w_down"])
+    torch.cuda.synchronize()
+    assert (b.group_offsets.cpu() == 0).all()
+    assert not b.dw_gate_up.any() and not b.dw_down.any() and not b.dw_router.any()

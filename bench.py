@@ -314,17 +314,47 @@ def timed_steps(wl, steps, world, local, per_kernel_timing=True):
     return max_over_ranks(ev0.elapsed_time(ev1), world), per_kernel, clk
 
 
+def group_bound_seconds(shape, counts, peaks):
+    """Per GEMM: the sum over experts of max(FLOPs_e / tensor peak, bytes_e / HBM peak),
+    each expert's group taken alone at full machine speed. Under skewed loads a light
+    expert's GEMM is bound by its weight (or weight-gradient) bytes, not its FLOPs, and a
+    pruned expert's weight gradients are still written (zeros), so this, not the FLOP
+    roofline, is what a grouped GEMM can reach on these loads."""
+    d, F = shape.d, shape.F
+    P = peaks["bf16_tflops_sustained"] * 1e12
+    BW = peaks["hbm_gbs"] * 1e9
+    out = dict.fromkeys(["gemm_gate_up", "gemm_down", "gemm_dgrad_down", "gemm_dgrad_gate_up",
+                         "gemm_wgrad_down", "gemm_wgrad_gate_up"], 0.0)
+    for m in counts:
+        m = int(m)
+        fl = {  # FLOPs, bytes (activations read/written, weights or weight gradients)
+            "gemm_gate_up": (4 * m * d * F, 2 * m * d + 4 * F * d + 4 * m * F + 2 * m * F),
+            "gemm_down": (2 * m * F * d, 2 * m * F + 2 * d * F + 2 * m * d),
+            "gemm_dgrad_down": (2 * m * d * F, 2 * m * d + 2 * d * F + 8 * m * F),
+            "gemm_dgrad_gate_up": (4 * m * F * d, 4 * m * F + 4 * F * d + 2 * m * d),
+            "gemm_wgrad_down": (2 * m * d * F, 2 * m * d + 2 * m * F + 2 * d * F),
+            "gemm_wgrad_gate_up": (4 * m * F * d, 4 * m * F + 2 * m * d + 4 * F * d),
+        }
+        for n, (f, b) in fl.items():
+            if m == 0 and not n.startswith("gemm_wgrad"):
+                continue  # no rows: no tile (weight gradients are still written)
+            out[n] += max(f / P, b / BW)
+    return out
+
+
 def kernel_report(wl, per_kernel, steps, peaks):
     """Per-kernel live CUDA-event times with achieved rates against the roofline."""
     s = wl.shape
     A = s.T * s.k
     flops = wl.gemm_flops()
+    bound = group_bound_seconds(s, wl.bufs.counts.cpu().tolist(), peaks)
     hbm = {  # algorithmic bytes per launch of the HBM-bound kernels
         "perm_gather": 2 * s.T * s.d + 2 * A * s.d,
         "combine": 2 * A * s.d + 2 * s.T * s.d,
         "combine_bwd": 2 * s.T * s.d + 4 * A * s.d,
         "permute_bwd": 2 * A * s.d + 2 * s.T * s.d,
         "route_bwd_partial": 2 * A * s.d,
+        "route_logits": 2 * s.T * s.d + 4 * s.d * s.E + 4 * s.T * s.E,
     }
     tot = sum(v[1] for v in per_kernel.values())
     out = {}
@@ -333,13 +363,11 @@ def kernel_report(wl, per_kernel, steps, peaks):
         per_launch_s = ms / c / 1e3
         if n in flops:
             tf = flops[n] / per_launch_s / 1e12
-            e.update(tflops=round(tf, 1), frac=round(tf / peaks["bf16_tflops_sustained"], 4))
+            e.update(tflops=round(tf, 1), frac=round(tf / peaks["bf16_tflops_sustained"], 4),
+                     group_bound_frac=round(bound[n] / per_launch_s, 4))
         elif n in hbm:
             gbs = hbm[n] / per_launch_s / 1e9
             e.update(gbs=round(gbs, 1), frac=round(gbs / peaks["hbm_gbs"], 4))
-        elif n == "route":
-            tf = 2.0 * s.T * s.d * s.E / per_launch_s / 1e12
-            e.update(fp32_tflops=round(tf, 2))
         out[n] = e
     return out
 
@@ -416,6 +444,8 @@ def run_ours(args):
     all_gemm_tflops = sum(flops.values()) / (all_gemm_ms / 1e3) / 1e12
     peak = peaks["bf16_tflops_sustained"]
     kernel_table = kernel_report(wl, per_kernel, args.steps, peaks)
+    gb = group_bound_seconds(wl.shape, wl.bufs.counts.cpu().tolist(), peaks)
+    gemm_bound_frac = sum(gb[n] for n in gemm_ms) / (all_gemm_ms / 1e3)
     laep = None
     if (wl.cfg.compact and args.tokens is None and args.experts is None and not args.no_prune
             and args.bias is None):
@@ -525,7 +555,11 @@ def run_ours(args):
         "grouped_gemm": {"tflops": round(all_gemm_tflops, 1),
                          "frac_of_peak": round(all_gemm_tflops / peak, 4),
                          "peak_tflops": peak, "peak": f"bf16 sustained, {peaks['source']}",
-                         "ms_per_step": round(all_gemm_ms, 4)},
+                         "ms_per_step": round(all_gemm_ms, 4),
+                         "group_bound_frac": round(gemm_bound_frac, 4),
+                         "group_bound": "sum over experts of max(FLOPs/tensor peak, bytes/HBM "
+                                        "peak) over the measured time (pruned experts' zero "
+                                        "weight gradients included)"},
         "roofline": {"kernel": dom, "bound": "tensor", "achieved": round(dom_tflops, 1),
                      "peak": peak, "unit": "TFLOP/s", "frac": round(dom_tflops / peak, 4),
                      "traffic": (committed_traffic(dom) if wl.cfg_id == 2 and args.tokens is None

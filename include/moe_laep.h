@@ -100,7 +100,7 @@ size_t moe_workspace_size(int T, int d, int E, int k, int F);
  * Sec. 3.2 defines the routing indicator E[i,j,l] (token j of layer l sent to
  * expert i) and Sec. 4 / Table 5 require pruned experts to receive no token;
  * the router itself is an fp32 linear layer with a fixed bias.
- *   z[t,e] = sum_i x[t,i] * w_router[i,e] + bias[e]     (fp32 FFMA)
+ *   z[t,e] = sum_i x[t,i] * w_router[i,e] + bias[e]     (fp32 accumulation)
  *   z[t,e] = -inf where active_mask[e] == 0
  *   topk_idx[t,0..k-1] = the k largest z (descending, ties to lower index)
  *   topk_gate[t,j]     = softmax over the k selected z (fp32)
@@ -111,8 +111,11 @@ size_t moe_workspace_size(int T, int d, int E, int k, int F);
  * still applied); logits_out [T,E] fp32 or NULL receives the masked z;
  * topk_idx [T,k] int32; topk_gate [T,k] fp32; counts [E] int32 or NULL;
  * ws, ws_bytes: workspace (moe_workspace_size; may be NULL with logits_in),
- * it holds the partial logits of the split reduction over d. The logits are
- * summed in a fixed order, so the routing is deterministic.
+ * it holds w_router as three bf16 terms (hi + mid + lo, which together keep
+ * every bit of an fp32 weight) for the tensor cores, whose bf16 products are
+ * exact and accumulate in fp32, and the partial logits of the split reduction
+ * over d. The partials are summed in a fixed order and every launch shape is a
+ * function of (T, d, E), so the routing is deterministic.
  * Limits: 1 <= E <= 256, 1 <= k <= min(E, 8), d % 8 == 0, T >= 0.
  * A token with fewer than k live experts sets MOE_DEV_TOO_FEW_LIVE.
  */

@@ -115,6 +115,8 @@ WsLayout ws_layout(int T, int d, int E, int k, int F) {
   off += align256(size_t(E) * d * 4);
   w.route_partial = off;
   off += align256(route_partial_bytes(T, d, E));
+  w.route_w3 = off;
+  off += align256(route_w3_bytes(d, E));
   w.total = off;
   return w;
 }

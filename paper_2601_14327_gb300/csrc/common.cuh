@@ -31,10 +31,12 @@ struct WsLayout {
   size_t rb_partial;    // fp32  [rows_cap/128, d] moe_route_bwd per-tile partial sums
   size_t w_router_t;    // fp32  [E, d]            moe_permute_bwd transposed router
   size_t route_partial; // fp32  [splits, T, NE]   moe_route split-reduction partial logits
+  size_t route_w3;      // bf16  [3, NP, d]        moe_route router weight as three bf16 terms
   size_t total;
 };
 WsLayout ws_layout(int T, int d, int E, int k, int F);
 size_t route_partial_bytes(int T, int d, int E);
+size_t route_w3_bytes(int d, int E);
 constexpr int kPermChunk = 4096;  // assignments per block in the permutation
 constexpr int kGroupPad = 128;    // rows per group are padded to this
 

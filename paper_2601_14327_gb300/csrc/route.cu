@@ -7,41 +7,14 @@
 #include <math.h>
 
 #include "common.cuh"
+#include "tc_ptx.cuh"
+#include "tmap.cuh"
 
 MOE_DEV_ERR_DECL
 
 namespace {
 
 constexpr int kRouteThreads = 256;
-constexpr int kRouteBK = 16;            // reduction chunk of the logit contraction
-constexpr int kRouteTargetCtas = 304;   // split the reduction until about this many CTAs
-
-// Logits kernel shape for the padded expert count NE (multiple of 64). Thread
-// (eg, tg) owns 8 tokens (tg*8 ..) and 8 experts {j*4*EG + eg*4 + q : j < 2,
-// q < 4}: per k it reads 8 x values and 8 W values as float4s (0.5-1 byte of
-// shared memory per FFMA; the float4 reads of one W row are contiguous across
-// eg) and keeps 64 accumulators, so two CTAs fit on an SM (<= 128 registers).
-template <int NE> struct RouteShape {
-  static constexpr int EG = NE / 8;                       // threads along the experts
-  static constexpr int THREADS = NE == 192 ? 384 : 256;
-  static constexpr int TN = 8;                            // experts per thread
-  static constexpr int TG = THREADS / EG;                 // threads along the tokens
-  static constexpr int TM = 8;                            // tokens per thread
-  static constexpr int BM = TG * TM;                      // tokens per CTA
-  static constexpr int MIN_BLOCKS = NE == 192 ? 1 : 2;
-  static constexpr size_t kStage = size_t(kRouteBK) * BM * 4 + size_t(kRouteBK) * NE * 4;
-  static constexpr size_t kSmem = 2 * kStage;
-};
-
-// Reduction split so that T/BM token tiles give about kRouteTargetCtas CTAs (at
-// most 8, never more CTAs than that target); fixed by (T, NE) alone, so the
-// workspace size is too.
-template <int NE> int route_splits(int T, int d) {
-  const int tiles = (T + RouteShape<NE>::BM - 1) / RouteShape<NE>::BM;
-  const int chunks = (d + kRouteBK - 1) / kRouteBK;
-  const int s = kRouteTargetCtas / std::max(tiles, 1);
-  return std::max(1, std::min({s, 8, chunks}));
-}
 int padded_experts(int E) { return E <= 64 ? 64 : (E <= 128 ? 128 : (E <= 192 ? 192 : 256)); }
 
 __device__ __forceinline__ bool better(float v, int e, float bv, int be) {
@@ -52,108 +25,231 @@ __global__ void zero_i32_kernel(int32_t *p, int n) {
   for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < n; i += gridDim.x * blockDim.x) p[i] = 0;
 }
 
-// partial[split][t][e] = sum over this split's k range of x[t,k] * W_r[k,e]
-// (fp32 FFMA, x converted from bf16 exactly; columns e >= E are zero). The next
-// k-chunk is loaded into registers while the current one is multiplied.
-template <int NE>
-__global__ void __launch_bounds__(RouteShape<NE>::THREADS, RouteShape<NE>::MIN_BLOCKS)
-    route_logits_kernel(
-    const uint16_t *__restrict__ x, const float *__restrict__ w_router, int T, int d, int E,
-    int k_per_split, float *__restrict__ partial) {
-  using S = RouteShape<NE>;
-  constexpr int TM = S::TM, TN = S::TN, EG = S::EG, BM = S::BM, BK = kRouteBK, NT = S::THREADS;
-  constexpr int XN = BM * BK / 8;             // 16-byte x loads per chunk
-  constexpr int XV = (XN + NT - 1) / NT;      // ... per thread
-  constexpr int WV = BK * NE / NT;            // W values per thread per chunk
-  extern __shared__ __align__(16) float smem[];
-  const int tid = threadIdx.x;
-  const int eg = tid % EG, tg = tid / EG;
-  const int t0 = blockIdx.x * BM;
-  const int kb = blockIdx.y * k_per_split, ke = min(d, kb + k_per_split);
+// ---- logits on the tensor cores ----------------------------------------------
+// The fp32 router weight is split into three bf16 terms, W = W_hi + W_mid + W_lo,
+// each the bf16 rounding of what the earlier terms leave (the bf16x3 scheme of
+// Henry, Tang and Heinecke, "Leveraging the bfloat16 artificial intelligence
+// datatype for higher-precision computations", 2019). Three 8-bit significands
+// cover the 24 of a normal fp32 weight, every bf16 x bf16 product is exact in
+// fp32, and the three MMAs of each k-step accumulate into one fp32 accumulator
+// in tensor memory, so the logits carry fp32 accumulation error only.
+//
+// One CTA = one 128-token tile x one range of k-blocks (a split of the
+// reduction over d when there are fewer tiles than SMs). Warp 0 issues the TMA
+// loads (x tile + the three weight terms per k-block), warp 1 owns TMEM and
+// issues the MMAs, then all four warps read the accumulator (one TMEM lane
+// quarter each) and write the partial logits partial[split][t][0..NP).
+constexpr int kRtBM = 128;       // tokens per tile (TMEM lanes)
+constexpr int kRtBK = 64;        // k-block: 64 bf16 = one 128-byte swizzle row
+constexpr int kRtThreads = 128;
+constexpr int kRtTargetCtas = 152;
+constexpr int kRtMaxSplits = 8;
+constexpr uint32_t kRtABytes = kRtBM * kRtBK * 2;
+constexpr int kRtMaxSmem = 232448;  // opt-in dynamic shared memory per CTA
+constexpr uint64_t kRtWaitNs = 2000000000ull;
 
-  float acc[TM][TN];
-#pragma unroll
-  for (int i = 0; i < TM; ++i)
-#pragma unroll
-    for (int j = 0; j < TN; ++j) acc[i][j] = 0.f;
-  float xr[XV][8], wr[WV];
-  auto load_chunk = [&](int k0) {
-#pragma unroll
-    for (int i = 0; i < XV; ++i) {
-      const int v = tid + i * NT;
-      const int row = v / (BK / 8), col = (v % (BK / 8)) * 8;
-      if (v < XN && t0 + row < T && k0 + col < ke) {
-        unpack8(ldg_nc_v4(x + size_t(t0 + row) * d + k0 + col), xr[i]);
-      } else {
-#pragma unroll
-        for (int q = 0; q < 8; ++q) xr[i][q] = 0.f;
-      }
-    }
-#pragma unroll
-    for (int i = 0; i < WV; ++i) {
-      const int v = tid + i * NT;
-      const int kk = v / NE, e = v % NE;
-      wr[i] = (e < E && k0 + kk < ke) ? __ldg(w_router + size_t(k0 + kk) * E + e) : 0.f;
-    }
-  };
-  auto store_chunk = [&](int buf) {
-    float *Xs = smem + buf * (S::kStage / 4);  // [BK][BM]
-    float *Ws = Xs + BK * BM;                  // [BK][NE]
-#pragma unroll
-    for (int i = 0; i < XV; ++i) {
-      const int v = tid + i * NT;
-      const int row = v / (BK / 8), col = (v % (BK / 8)) * 8;
-      if (v < XN) {
-#pragma unroll
-        for (int q = 0; q < 8; ++q) Xs[(col + q) * BM + row] = xr[i][q];
-      }
-    }
-#pragma unroll
-    for (int i = 0; i < WV; ++i) Ws[tid + i * NT] = wr[i];
-  };
-  const int nchunks = (ke - kb + BK - 1) / BK;
-  if (nchunks > 0) {
-    load_chunk(kb);
-    store_chunk(0);
+struct RouteTcParams {
+  int T;             // tokens
+  int kb_per_split;  // k-blocks of one split
+  int nkb;           // k-blocks in d
+  int NP;            // MMA N: experts rounded up to 16
+  int NE;            // row stride of the partial logits
+  int stages;        // shared-memory ring depth
+  uint32_t tmem_cols;
+  float *partial;
+};
+
+// Experts rounded up to the MMA's N granularity, and the matching TMEM allocation.
+int route_tc_np(int E) { return (E + 15) / 16 * 16; }
+uint32_t route_tc_tmem_cols(int NP) { return NP <= 32 ? 32u : (NP <= 64 ? 64u : (NP <= 128 ? 128u : 256u)); }
+uint32_t route_tc_stage_bytes(int NP) { return kRtABytes + 3u * uint32_t(NP) * 128u; }
+int route_tc_stages(int NP) {
+  return std::min(8, int((kRtMaxSmem - 2048) / route_tc_stage_bytes(NP)));
+}
+size_t route_tc_smem(int NP, int stages) {
+  return 1024 + size_t(stages) * route_tc_stage_bytes(NP) + size_t(2 * stages + 1) * 8 + 16;
+}
+// Splits of the reduction: enough CTAs to cover the SMs when T gives few tiles.
+// A function of (T, d) alone, so the workspace size is too.
+void route_tc_split(int T, int d, int *splits, int *kb_per_split) {
+  const int tiles = std::max(1, (T + kRtBM - 1) / kRtBM);
+  const int nkb = (d + kRtBK - 1) / kRtBK;
+  int s = std::max(1, std::min({kRtTargetCtas / tiles, kRtMaxSplits, nkb}));
+  const int per = (nkb + s - 1) / s;
+  *kb_per_split = per;
+  *splits = (nkb + per - 1) / per;  // every split gets at least one k-block
+}
+
+// W [d, E] fp32 -> W3 [3][NP][d] bf16 (hi, mid, lo; rows e >= E are zero), by
+// 32 x 32 tiles transposed through shared memory.
+__global__ void route_split_w_kernel(const float *__restrict__ w, int d, int E, int NP,
+                                     uint16_t *__restrict__ w3) {
+  __shared__ float tile[32][33];
+  const int k0 = blockIdx.x * 32, e0 = blockIdx.y * 32;
+  const int tx = threadIdx.x, ty = threadIdx.y;
+  for (int i = ty; i < 32; i += 8) {
+    const int k = k0 + i, e = e0 + tx;
+    tile[i][tx] = (k < d && e < E) ? w[size_t(k) * E + e] : 0.f;
   }
   __syncthreads();
-  for (int ch = 0; ch < nchunks; ++ch) {
-    if (ch + 1 < nchunks) load_chunk(kb + (ch + 1) * BK);
-    const float *Xs = smem + (ch & 1) * (S::kStage / 4);
-    const float *Ws = Xs + BK * BM;
-#pragma unroll
-    for (int kk = 0; kk < BK; ++kk) {
-      const float4 x0 = *reinterpret_cast<const float4 *>(&Xs[kk * BM + tg * TM]);
-      const float4 x1 = *reinterpret_cast<const float4 *>(&Xs[kk * BM + tg * TM + 4]);
-      const float xs[8] = {x0.x, x0.y, x0.z, x0.w, x1.x, x1.y, x1.z, x1.w};
-#pragma unroll
-      for (int j4 = 0; j4 < TN / 4; ++j4) {
-        const float4 wv = *reinterpret_cast<const float4 *>(&Ws[kk * NE + j4 * 4 * EG + eg * 4]);
-        const float ws[4] = {wv.x, wv.y, wv.z, wv.w};
-#pragma unroll
-        for (int i = 0; i < TM; ++i)
-#pragma unroll
-          for (int q = 0; q < 4; ++q) acc[i][j4 * 4 + q] = fmaf(xs[i], ws[q], acc[i][j4 * 4 + q]);
-      }
+  for (int i = ty; i < 32; i += 8) {
+    const int e = e0 + i, k = k0 + tx;
+    if (e < NP && k < d) {
+      const float v = tile[tx][i];
+      const __nv_bfloat16 hi = __float2bfloat16_rn(v);
+      const float r1 = v - __bfloat162float(hi);
+      const __nv_bfloat16 mid = __float2bfloat16_rn(r1);
+      const float r2 = r1 - __bfloat162float(mid);
+      const __nv_bfloat16 lo = __float2bfloat16_rn(r2);
+      const size_t plane = size_t(NP) * d, at = size_t(e) * d + k;
+      w3[at] = __bfloat16_as_ushort(hi);
+      w3[plane + at] = __bfloat16_as_ushort(mid);
+      w3[2 * plane + at] = __bfloat16_as_ushort(lo);
     }
-    if (ch + 1 < nchunks) store_chunk((ch + 1) & 1);
-    __syncthreads();
-  }
-  float *out = partial + size_t(blockIdx.y) * T * NE;
-#pragma unroll
-  for (int i = 0; i < TM; ++i) {
-    const int t = t0 + tg * TM + i;
-    if (t >= T) break;
-#pragma unroll
-    for (int j4 = 0; j4 < TN / 4; ++j4)
-      *reinterpret_cast<float4 *>(out + size_t(t) * NE + j4 * 4 * EG + eg * 4) =
-          make_float4(acc[i][j4 * 4], acc[i][j4 * 4 + 1], acc[i][j4 * 4 + 2], acc[i][j4 * 4 + 3]);
   }
 }
 
-// One warp per token: logits = sum of the split partials (fixed order) + bias,
-// pruned experts -inf, k rounds of a warp arg-max (ties to the lower index),
-// softmax over the selected logits, per-expert histogram.
+__global__ void __launch_bounds__(kRtThreads, 1)
+    route_logits_tc_kernel(const __grid_constant__ CUtensorMap tmX,
+                           const __grid_constant__ CUtensorMap tmW, const RouteTcParams p) {
+  extern __shared__ uint8_t smem_raw[];
+  const uint32_t raw = tc::smem_u32(smem_raw);
+  const uint32_t pad = (1024u - (raw & 1023u)) & 1023u;
+  const uint32_t b_bytes = uint32_t(p.NP) * 128u;
+  const uint32_t stage_bytes = kRtABytes + 3u * b_bytes;
+  const int S = p.stages;
+  const uint32_t s0 = raw + pad;
+  uint64_t *bars = reinterpret_cast<uint64_t *>(smem_raw + pad + size_t(S) * stage_bytes);
+  int *misc = reinterpret_cast<int *>(bars + 2 * S + 1);
+  volatile int *abort_flag = misc + 1;
+  volatile int no_abort = 0;
+  const uint32_t bar0 = tc::smem_u32(bars);
+  auto full_bar = [&](int s) { return bar0 + 8u * s; };
+  auto empty_bar = [&](int s) { return bar0 + 8u * (S + s); };
+  const uint32_t done_bar = bar0 + 8u * (2 * S);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int mt = blockIdx.x, split = blockIdx.y;
+  const int kb0 = split * p.kb_per_split, kb1 = min(p.nkb, kb0 + p.kb_per_split);
+  const uint32_t idesc = tc::idesc_bf16_f32(kRtBM, p.NP, false, false);
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < S; ++s) {
+      tc::mbar_init(full_bar(s), 1);
+      tc::mbar_init(empty_bar(s), 1);
+    }
+    tc::mbar_init(done_bar, 1);
+    tc::fence_mbar_init();
+    misc[1] = 0;
+  }
+  if (warp == 0 && lane == 0) {
+    tc::tma_prefetch_desc(&tmX);
+    tc::tma_prefetch_desc(&tmW);
+  }
+  if (warp == 1) {
+    tc::tmem_alloc(tc::smem_u32(misc), p.tmem_cols);
+    tc::tmem_relinquish();
+  }
+  tc::fence_before_sync();
+  __syncthreads();
+  tc::fence_after_sync();
+  const uint32_t tmem_base = static_cast<uint32_t>(misc[0]);
+
+  if (warp == 0 && lane == 0) {
+    // ---- TMA producer ----
+    uint32_t it = 0;
+    for (int kb = kb0; kb < kb1; ++kb, ++it) {
+      const int s = it % S;
+      const uint32_t ph = (it / S) & 1u;
+      if (!tc::mbar_wait(empty_bar(s), ph ^ 1u, kRtWaitNs, abort_flag)) {
+        dev_flag(&g_dev_err, MOE_DEV_WAIT_TIMEOUT);
+        *abort_flag = 1;
+        break;
+      }
+      tc::mbar_arrive_expect_tx(full_bar(s), stage_bytes);
+      const uint32_t dst = s0 + s * stage_bytes;
+      const int k0 = kb * kRtBK;
+      tc::tma_load_2d(dst, &tmX, full_bar(s), k0, mt * kRtBM);
+#pragma unroll
+      for (int j = 0; j < 3; ++j)
+        tc::tma_load_2d(dst + kRtABytes + j * b_bytes, &tmW, full_bar(s), k0, j * p.NP);
+    }
+    // every issued load lands before the CTA may exit (also after an abort)
+    for (int s = 0; s < S; ++s) {
+      if (it > uint32_t(s)) {
+        const uint32_t n = (it - 1 - s) / S;
+        if (!tc::mbar_wait(full_bar(s), n & 1u, kRtWaitNs, &no_abort))
+          dev_flag(&g_dev_err, MOE_DEV_WAIT_TIMEOUT);
+      }
+    }
+  } else if (warp == 1 && lane == 0) {
+    // ---- MMA issuer ----
+    uint32_t it = 0;
+    bool issued = false;
+    for (int kb = kb0; kb < kb1; ++kb, ++it) {
+      const int s = it % S;
+      const uint32_t ph = (it / S) & 1u;
+      if (!tc::mbar_wait(full_bar(s), ph, kRtWaitNs, abort_flag)) {
+        dev_flag(&g_dev_err, MOE_DEV_WAIT_TIMEOUT);
+        *abort_flag = 1;
+        break;
+      }
+      tc::fence_after_sync();
+      const uint32_t a_s = s0 + s * stage_bytes, b_s = a_s + kRtABytes;
+#pragma unroll
+      for (int kk = 0; kk < kRtBK / 16; ++kk) {
+        const uint64_t ad = tc::smem_desc_sw128(a_s + kk * 32, 16, 1024);
+#pragma unroll
+        for (int j = 0; j < 3; ++j) {
+          const uint64_t bd = tc::smem_desc_sw128(b_s + j * b_bytes + kk * 32, 16, 1024);
+          tc::mma_bf16(tmem_base, ad, bd, idesc, (kb != kb0 || kk != 0 || j != 0) ? 1u : 0u);
+        }
+      }
+      tc::mma_commit(empty_bar(s));
+      issued = true;
+    }
+    if (issued) tc::mma_commit(done_bar);
+    else *abort_flag = 1;  // nothing to wait for: the epilogue must not wait either
+  }
+  __syncwarp();
+
+  // ---- epilogue: TMEM lane quarter `warp` -> 32 tokens x NP partial logits ----
+  int ok = 0;
+  if (lane == 0) {
+    ok = tc::mbar_wait(done_bar, 0, kRtWaitNs, abort_flag) ? 1 : 0;
+    if (!ok && !*abort_flag) {
+      dev_flag(&g_dev_err, MOE_DEV_WAIT_TIMEOUT);
+      *abort_flag = 1;
+    }
+  }
+  ok = __shfl_sync(0xffffffffu, ok, 0);
+  if (ok) {
+    tc::fence_after_sync();
+    const int t = mt * kRtBM + warp * 32 + lane;
+    float *dst = p.partial + (size_t(split) * p.T + t) * p.NE;
+    for (int c0 = 0; c0 < p.NP; c0 += 32) {
+      uint32_t r[32];
+      tc::tmem_ld_32x32b_x32(tmem_base + (uint32_t(warp * 32) << 16) + uint32_t(c0), r);
+      tc::tmem_ld_wait();
+      if (t < p.T) {
+#pragma unroll
+        for (int q = 0; q < 8; ++q)
+          stg_v4(dst + c0 + 4 * q, make_uint4(r[4 * q], r[4 * q + 1], r[4 * q + 2], r[4 * q + 3]));
+      }
+    }
+  }
+  tc::fence_before_sync();
+  __syncthreads();
+  if (warp == 1) {
+    tc::fence_after_sync();
+    tc::tmem_dealloc(tmem_base, p.tmem_cols);
+  }
+}
+
+// One warp per token: logits = sum of the split
+// partials (fixed order) + bias, pruned experts -inf, k rounds of a warp arg-max
+// (ties to the lower index), softmax over the selected logits, per-expert
+// histogram (shared per block, then one global add per expert and block).
 template <int NE>
 __global__ void __launch_bounds__(kRouteThreads) route_topk_kernel(
     const float *__restrict__ partial, int splits, const float *__restrict__ logits_in,
@@ -165,8 +261,8 @@ __global__ void __launch_bounds__(kRouteThreads) route_topk_kernel(
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   for (int e = tid; e < NE; e += kRouteThreads) hist[e] = 0;
   __syncthreads();
-  const int t = blockIdx.x * (kRouteThreads / 32) + warp;
-  if (t < T) {
+  for (int t = blockIdx.x * (kRouteThreads / 32) + warp; t < T;
+       t += gridDim.x * (kRouteThreads / 32)) {
     float v[TK];
 #pragma unroll
     for (int j = 0; j < TK; ++j) {
@@ -327,28 +423,52 @@ __global__ void route_bwd_reduce_kernel(const float *__restrict__ partial,
   dw_router[size_t(i) * E + e] = s;
 }
 
+// Tensor-core logits: splits W into its three bf16 terms (w3), then one CTA per
+// (token tile, split). Returns the number of partial planes written in *splits.
+int launch_route_tc(const uint16_t *x, const float *w, int T, int d, int E, int NE, uint16_t *w3,
+                    float *partial, int *splits_out, cudaStream_t s) {
+  const int NP = route_tc_np(E);
+  const int stages = route_tc_stages(NP);
+  const size_t smem = route_tc_smem(NP, stages);
+  static bool attr_set = false;
+  if (!attr_set) {
+    cudaError_t e = cudaFuncSetAttribute(route_logits_tc_kernel,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, kRtMaxSmem);
+    if (e != cudaSuccess) return moe::cuda_status(e, "moe_route: set smem attribute");
+    attr_set = true;
+  }
+  dim3 sgrid((d + 31) / 32, (NP + 31) / 32);
+  MOE_LAUNCH("route_split_w", s, route_split_w_kernel<<<sgrid, dim3(32, 8), 0, s>>>(w, d, E, NP, w3));
+  if (int st = moe::launch_status("moe_route: split router weight")) return st;
+  CUtensorMap mx, mw;
+  int st;
+  if ((st = moe::make_map(&mx, x, uint64_t(T), uint64_t(d), kRtBK, kRtBM, "router x"))) return st;
+  if ((st = moe::make_map(&mw, w3, uint64_t(3 * NP), uint64_t(d), kRtBK, uint32_t(NP), "router w")))
+    return st;
+  int splits = 1, per = 1;
+  route_tc_split(T, d, &splits, &per);
+  RouteTcParams p;
+  p.T = T;
+  p.kb_per_split = per;
+  p.nkb = (d + kRtBK - 1) / kRtBK;
+  p.NP = NP;
+  p.NE = NE;
+  p.stages = stages;
+  p.tmem_cols = route_tc_tmem_cols(NP);
+  p.partial = partial;
+  dim3 grid((T + kRtBM - 1) / kRtBM, splits);
+  MOE_LAUNCH("route_logits", s, route_logits_tc_kernel<<<grid, kRtThreads, smem, s>>>(mx, mw, p));
+  *splits_out = splits;
+  return moe::launch_status("moe_route: logits");
+}
+
 template <int NE>
 int launch_route(const uint16_t *x, const float *w, const float *b, const uint8_t *mask, int T,
                  int d, int E, int k, const float *lin, float *lout, int32_t *idx, float *gate,
-                 int32_t *counts, float *partial, cudaStream_t s) {
-  using S = RouteShape<NE>;
+                 int32_t *counts, float *partial, uint16_t *w3, cudaStream_t s) {
   int splits = 0;
-  if (lin == nullptr) {
-    static bool attr_set = false;
-    if (!attr_set) {
-      cudaError_t e = cudaFuncSetAttribute(route_logits_kernel<NE>,
-                                           cudaFuncAttributeMaxDynamicSharedMemorySize, int(S::kSmem));
-      if (e != cudaSuccess) return moe::cuda_status(e, "moe_route: set smem attribute");
-      attr_set = true;
-    }
-    splits = route_splits<NE>(T, d);
-    const int chunks = (d + kRouteBK - 1) / kRouteBK;
-    const int k_per_split = ((chunks + splits - 1) / splits) * kRouteBK;
-    dim3 grid((T + S::BM - 1) / S::BM, splits);
-    MOE_LAUNCH("route_logits", s, route_logits_kernel<NE><<<grid, S::THREADS, S::kSmem, s>>>(
-                                      x, w, T, d, E, k_per_split, partial));
-    if (int st = moe::launch_status("moe_route: logits")) return st;
-  }
+  if (lin == nullptr)
+    if (int st = launch_route_tc(x, w, T, d, E, NE, w3, partial, &splits, s)) return st;
   const int grid2 = (T + kRouteThreads / 32 - 1) / (kRouteThreads / 32);
   MOE_LAUNCH("route_topk", s, route_topk_kernel<NE><<<grid2, kRouteThreads, 0, s>>>(
                                   partial, splits, lin, b, mask, T, E, k, lout, idx, gate, counts));
@@ -362,17 +482,12 @@ MOE_DEV_ERR_DEFINE_READER(route_dev_error)
 
 size_t route_partial_bytes(int T, int d, int E) {
   if (T <= 0) return 0;
-  const int NE = padded_experts(E);
-  int splits = 1;
-  switch (NE) {
-    case 64: splits = route_splits<64>(T, d); break;
-    case 128: splits = route_splits<128>(T, d); break;
-    case 192: splits = route_splits<192>(T, d); break;
-    default: splits = route_splits<256>(T, d); break;
-  }
-  return size_t(splits) * size_t(T) * size_t(NE) * 4;
+  int splits = 1, per = 1;
+  route_tc_split(T, d, &splits, &per);
+  return size_t(splits) * size_t(T) * size_t(padded_experts(E)) * 4;
 }
-}
+size_t route_w3_bytes(int d, int E) { return size_t(3) * route_tc_np(E) * size_t(d) * 2; }
+}  // namespace moe
 
 extern "C" {
 
@@ -389,11 +504,13 @@ int moe_route(const uint16_t *x, const float *w_router, const float *bias,
     return moe::set_error(MOE_ERR_ARG, "moe_route: null x/w_router");
   if (x && !moe::aligned16(x)) return moe::set_error(MOE_ERR_ARG, "moe_route: x not 16-byte aligned");
   float *partial = nullptr;
+  uint16_t *w3 = nullptr;
   if (!logits_in && T > 0) {
     const moe::WsLayout L = moe::ws_layout(T, d, E, k, 0);
     if (!ws || ws_bytes < L.total) return moe::set_error(MOE_ERR_WORKSPACE, "moe_route: workspace");
     if (!moe::aligned16(ws)) return moe::set_error(MOE_ERR_ARG, "moe_route: ws alignment");
     partial = reinterpret_cast<float *>(static_cast<char *>(ws) + L.route_partial);
+    w3 = reinterpret_cast<uint16_t *>(static_cast<char *>(ws) + L.route_w3);
   }
   if (counts) {
     MOE_LAUNCH("zero_counts", s, zero_i32_kernel<<<1, 256, 0, s>>>(counts, E));
@@ -401,10 +518,10 @@ int moe_route(const uint16_t *x, const float *w_router, const float *bias,
   }
   if (T == 0) return MOE_OK;
   switch (padded_experts(E)) {
-    case 64: return launch_route<64>(x, w_router, bias, active_mask, T, d, E, k, logits_in, logits_out, topk_idx, topk_gate, counts, partial, s);
-    case 128: return launch_route<128>(x, w_router, bias, active_mask, T, d, E, k, logits_in, logits_out, topk_idx, topk_gate, counts, partial, s);
-    case 192: return launch_route<192>(x, w_router, bias, active_mask, T, d, E, k, logits_in, logits_out, topk_idx, topk_gate, counts, partial, s);
-    default: return launch_route<256>(x, w_router, bias, active_mask, T, d, E, k, logits_in, logits_out, topk_idx, topk_gate, counts, partial, s);
+    case 64: return launch_route<64>(x, w_router, bias, active_mask, T, d, E, k, logits_in, logits_out, topk_idx, topk_gate, counts, partial, w3, s);
+    case 128: return launch_route<128>(x, w_router, bias, active_mask, T, d, E, k, logits_in, logits_out, topk_idx, topk_gate, counts, partial, w3, s);
+    case 192: return launch_route<192>(x, w_router, bias, active_mask, T, d, E, k, logits_in, logits_out, topk_idx, topk_gate, counts, partial, w3, s);
+    default: return launch_route<256>(x, w_router, bias, active_mask, T, d, E, k, logits_in, logits_out, topk_idx, topk_gate, counts, partial, w3, s);
   }
 }
 

@@ -60,7 +60,8 @@ def main():
     out = {"call": a.call, "T": T, "d": d, "E": E, "k": k}
     if a.call == "route":
         ms = _time(route, a.iters, a.warmup)
-        out.update(ms=round(ms, 4), fp32_tflops=round(2.0 * T * d * E / (ms / 1e3) / 1e12, 2))
+        nbytes = 2 * T * d + 4 * d * E + 8 * T * k  # x, router weight, indices and gates
+        out.update(ms=round(ms, 4), gbs=round(nbytes / (ms / 1e3) / 1e9, 1))
     else:
         route()
         R = L.moe_perm_rows_max(T, k, E)

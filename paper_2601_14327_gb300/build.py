@@ -18,7 +18,7 @@ CSRC = os.path.join(HERE, "csrc")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(BUILD, "libmoe_laep.so")
 SOURCES = ["api.cu", "laep.cu", "route.cu", "permute.cu", "gemm.cu"]
-HEADERS = ["common.cuh", "tc_ptx.cuh"]
+HEADERS = ["common.cuh", "tc_ptx.cuh", "tmap.cuh"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

@@ -92,7 +92,11 @@ __device__ __forceinline__ void fail(volatile int *abort_flag) {
   *abort_flag = 1;
 }
 
-__device__ __forceinline__ float silu_f(float a) { return a / (1.f + __expf(-a)); }
+// sigmoid(a) = 1 / (1 + e^-a) with the fast reciprocal-based divide (2 ulp; the
+// results are rounded to bf16). For very negative a, e^-a overflows to +inf and
+// the quotient is 0, the limit of the function.
+__device__ __forceinline__ float sigmoid_f(float a) { return __fdividef(1.f, 1.f + __expf(-a)); }
+__device__ __forceinline__ float silu_f(float a) { return a * sigmoid_f(a); }
 
 // Saved pre-activations [A|B] are stored in 32-row blocks: element (r, c) of the
 // [rows, 2F] matrix lives at ((r/32)*(2F/8) + c/8)*256 + (r%32)*8 + c%8, so the
@@ -202,7 +206,7 @@ __device__ __forceinline__ void epilogue_tile(const GemmParams &p, const CUtenso
 #pragma unroll
         for (int i = 0; i < 8; ++i) {
           const float dh = __uint_as_float(r[v * 8 + i]);
-          const float sg = 1.f / (1.f + __expf(-fa[i]));
+          const float sg = sigmoid_f(fa[i]);
           da[i] = dh * fb[i] * (sg * (1.f + fa[i] * (1.f - sg)));
           db[i] = dh * fa[i] * sg;
         }

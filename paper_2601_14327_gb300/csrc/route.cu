@@ -130,7 +130,10 @@ __global__ void __launch_bounds__(kRtThreads, 1)
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int mt = blockIdx.x, split = blockIdx.y;
-  const int kb0 = split * p.kb_per_split, kb1 = min(p.nkb, kb0 + p.kb_per_split);
+  const int kb0 = split * p.kb_per_split, nk = min(p.nkb, kb0 + p.kb_per_split) - kb0;
+  // Each tile starts its k-loop at its own offset, so that the CTAs do not all read
+  // the same weight tile from L2 at the same time (the order is fixed per tile).
+  const int rot = nk > 0 ? int((mt * 7u) % uint32_t(nk)) : 0;
   const uint32_t idesc = tc::idesc_bf16_f32(kRtBM, p.NP, false, false);
 
   if (threadIdx.x == 0) {
@@ -158,7 +161,8 @@ __global__ void __launch_bounds__(kRtThreads, 1)
   if (warp == 0 && lane == 0) {
     // ---- TMA producer ----
     uint32_t it = 0;
-    for (int kb = kb0; kb < kb1; ++kb, ++it) {
+    for (; int(it) < nk; ++it) {
+      const int kb = kb0 + (int(it) + rot) % nk;
       const int s = it % S;
       const uint32_t ph = (it / S) & 1u;
       if (!tc::mbar_wait(empty_bar(s), ph ^ 1u, kRtWaitNs, abort_flag)) {
@@ -186,7 +190,7 @@ __global__ void __launch_bounds__(kRtThreads, 1)
     // ---- MMA issuer ----
     uint32_t it = 0;
     bool issued = false;
-    for (int kb = kb0; kb < kb1; ++kb, ++it) {
+    for (; int(it) < nk; ++it) {
       const int s = it % S;
       const uint32_t ph = (it / S) & 1u;
       if (!tc::mbar_wait(full_bar(s), ph, kRtWaitNs, abort_flag)) {
@@ -202,7 +206,7 @@ __global__ void __launch_bounds__(kRtThreads, 1)
 #pragma unroll
         for (int j = 0; j < 3; ++j) {
           const uint64_t bd = tc::smem_desc_sw128(b_s + j * b_bytes + kk * 32, 16, 1024);
-          tc::mma_bf16(tmem_base, ad, bd, idesc, (kb != kb0 || kk != 0 || j != 0) ? 1u : 0u);
+          tc::mma_bf16(tmem_base, ad, bd, idesc, (it != 0 || kk != 0 || j != 0) ? 1u : 0u);
         }
       }
       tc::mma_commit(empty_bar(s));

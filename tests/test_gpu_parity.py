@@ -64,7 +64,10 @@ def test_route_ties_go_to_lower_index():
     np.testing.assert_allclose(g, og, rtol=0, atol=2e-6)
 
 
-@pytest.mark.parametrize("T,d,E", [(777, 512, 64), (300, 1024, 171), (129, 256, 256)])
+@pytest.mark.parametrize("T,d,E", [(777, 512, 64), (300, 1024, 171), (129, 256, 256),
+                                   # d not a multiple of the 64-wide k-block (zero-filled tail),
+                                   # few experts (MMA N = 16), one token, the smallest d
+                                   (333, 200, 13), (1, 72, 256), (64, 8, 5), (50, 136, 2)])
 def test_route_logits_fp32(T, d, E):
     inp = case_inputs(T, d, E, 2, 128, seed=5)
     o = oracle_inputs(inp)

@@ -141,7 +141,7 @@ class Workload:
     """Inputs, the one-time LAEP prune, and the buffers of one layer step."""
 
     def __init__(self, cfg_id: int, device: str, compact_override=None, tokens=None,
-                 experts=None, no_prune=False, bias=None):
+                 experts=None, no_prune=False, bias=None, gather=False):
         c = synth.CONFIGS[cfg_id]
         if tokens or experts or no_prune or bias:  # a variant of the workload (profiling)
             import dataclasses
@@ -182,7 +182,7 @@ class Workload:
                 self.mask = mask.to(device)
         self.shape = layer.LayerShape(T, d, E, k, F)
         self.E_live = E - (self.n_pruned if self.mask is not None else 0)
-        self.bufs = layer.MoELayerBuffers(self.shape, device, backward=True)
+        self.bufs = layer.MoELayerBuffers(self.shape, device, backward=True, gather=gather)
 
         self.graph = None
 
@@ -387,7 +387,7 @@ def laep_comparison(args, world, local, pruned_tps, wl_pruned):
     saved = wl_pruned.bufs
     wl_pruned.bufs = None
     torch.cuda.empty_cache()
-    wl_u = Workload(args.config, "cuda", no_prune=True)
+    wl_u = Workload(args.config, "cuda", no_prune=True, gather=bool(args.gather))
     for _ in range(args.warmup):
         wl_u.step()
     if args.graph:
@@ -413,7 +413,7 @@ def run_ours(args):
     L.load()
     peaks = measured_peaks()
     wl = Workload(args.config, "cuda", tokens=args.tokens, experts=args.experts,
-                  no_prune=args.no_prune, bias=args.bias)
+                  no_prune=args.no_prune, bias=args.bias, gather=bool(args.gather))
     s = wl.shape
     torch.cuda.synchronize()
     for _ in range(args.warmup):
@@ -551,7 +551,9 @@ def run_ours(args):
         "config": {"workload": c.name, "T": s.T, "d_model": s.d, "experts": c.E,
                    "experts_live": wl.E_live, "top_k": s.k, "d_ff": s.F, "gate_bias": c.bias,
                    "pruned": wl.n_pruned, "l2": "working set far above L2 (x 134 MB, expert "
-                   "weights GBs); no flush", "parallelism": "replicas" if world > 1 else "1 GPU"},
+                   "weights GBs); no flush", "parallelism": "replicas" if world > 1 else "1 GPU",
+                   "dispatch": ("TMA gathers from x (X_perm not materialized)" if args.gather
+                                else "materialized X_perm")},
         "grouped_gemm": {"tflops": round(all_gemm_tflops, 1),
                          "frac_of_peak": round(all_gemm_tflops / peak, 4),
                          "peak_tflops": peak, "peak": f"bf16 sustained, {peaks['source']}",
@@ -635,6 +637,9 @@ def main():
     ap.add_argument("--ref-tokens", type=int, default=64)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--gather", type=int, default=0,
+                    help="dispatch through a materialized X_perm (0), or by 4-row TMA gathers "
+                         "from x with X_perm never written (1; same results, slower GEMMs)")
     ap.add_argument("--graph", type=int, default=1,
                     help="time replays of a CUDA graph of the whole step (1) or eager steps (0)")
     # smaller cases of the same kernels, for profiler captures

@@ -253,6 +253,50 @@ int moe_grouped_ffn_fwd(const uint16_t *x_perm, const int32_t *group_offsets, in
                         uint16_t *out_perm, void *ws, size_t ws_bytes, moe_stream_t stream);
 
 /*
+ * Gathered form of the dispatch (no X_perm in memory). The grouped operand X_perm
+ * of the forward GEMM and of the dW_gate_up GEMM, and the rows the router
+ * backward reads, are taken from x itself through a row -> token map: grouped
+ * row r is x[token_of_row[r], :]. The GEMMs load those rows with 4-row TMA
+ * gathers (one token row of d_model per gathered row, 128 bytes at a time), so
+ * the (T*k + padding) x d copy that moe_permute writes is never materialized.
+ * Results are the same as with moe_permute's X_perm, bit for bit, on every real
+ * row and in every gradient: a padding row reads token 0 instead of zeros, and
+ * every consumer multiplies padding rows by zero (d_out_perm's padding rows are
+ * zero, and the router backward reads real rows only); on padding rows the
+ * forward's ab_saved, h and out_perm hold finite values instead of zeros.
+ * Cost on GB300: the two GEMMs that read X_perm run ~3.3x longer with 4-row
+ * gathers than with tile loads of a materialized X_perm, far more than the
+ * copy saves; moe_permute + the plain entry points are the fast path.
+ */
+
+/*
+ * moe_permute_map - the grouped layout of moe_permute without the row copy:
+ * group_offsets [E+1], group_counts [E], row_of_assignment [T,k] exactly as
+ * moe_permute computes them, and token_of_row [rows_cap] int32 (out): the token
+ * of each grouped row (real rows: the t of its assignment; padding rows: 0;
+ * rows at or past group_offsets[E] are not written). ws: the workspace of
+ * moe_permute (only its first region, the per-block histograms, is used).
+ * Limits as in moe_permute; token_of_row 16-byte aligned.
+ */
+int moe_permute_map(const int32_t *topk_idx, const int32_t *counts, int T, int E, int k,
+                    int64_t rows_cap, int32_t *group_offsets, int32_t *group_counts,
+                    int32_t *row_of_assignment, int32_t *token_of_row, void *ws, size_t ws_bytes,
+                    moe_stream_t stream);
+
+/*
+ * moe_grouped_ffn_fwd_gather - moe_grouped_ffn_fwd with X_perm read from
+ * x [T,d] bf16 through token_of_row (from moe_permute_map). Other arguments,
+ * outputs and limits as in moe_grouped_ffn_fwd; needs the CTA-pair GEMM kernel
+ * (the default; MOE_ERR_UNSUPPORTED under MOE_GEMM_1SM=1).
+ */
+int moe_grouped_ffn_fwd_gather(const uint16_t *x, const int32_t *token_of_row, int T,
+                               const int32_t *group_offsets, int E, int d, int F,
+                               int64_t rows_cap, const uint16_t *w_gate_up,
+                               const uint16_t *w_down, uint16_t *ab_saved, uint16_t *h,
+                               uint16_t *out_perm, void *ws, size_t ws_bytes,
+                               moe_stream_t stream);
+
+/*
  * moe_unpermute_combine - gate-weighted combine back to token order:
  *   y[t,:] = sum_j topk_gate[t,j] * out_perm[row_of_assignment[t,j], :]
  * summed in fp32, rounded once to bf16. out_perm [rows_cap,d] bf16;
@@ -311,6 +355,17 @@ int moe_grouped_ffn_bwd_wgrad(const uint16_t *d_out_perm, const uint16_t *x_perm
                               uint16_t *dw_gate_up, uint16_t *dw_down, moe_stream_t stream);
 
 /*
+ * moe_grouped_ffn_bwd_wgrad_gather - moe_grouped_ffn_bwd_wgrad with X_e read
+ * from x [T,d] bf16 through token_of_row (moe_permute_map). Other arguments
+ * and limits as in moe_grouped_ffn_bwd_wgrad (CTA-pair kernel only).
+ */
+int moe_grouped_ffn_bwd_wgrad_gather(const uint16_t *d_out_perm, const uint16_t *x,
+                                     const int32_t *token_of_row, int T, const uint16_t *h,
+                                     const uint16_t *d_ab, const int32_t *group_offsets, int E,
+                                     int d, int F, int64_t rows_cap, uint16_t *dw_gate_up,
+                                     uint16_t *dw_down, moe_stream_t stream);
+
+/*
  * moe_route_bwd - backward of the router's softmax over the selected experts:
  *   d_logits[t,j] = g[t,j] * (d_gate[t,j] - sum_i g[t,i] * d_gate[t,i])
  *   dw_router[:, e] = sum over assignments (t,j) to e of d_logits[t,j] * x[t,:]
@@ -323,6 +378,17 @@ int moe_route_bwd(const uint16_t *x_perm, const int32_t *topk_idx, const float *
                   const int32_t *group_offsets, const int32_t *group_counts, int T, int d,
                   int E, int k, int64_t rows_cap, float *d_logits, float *dw_router, void *ws,
                   size_t ws_bytes, moe_stream_t stream);
+
+/*
+ * moe_route_bwd_gather - moe_route_bwd with the rows of x read through
+ * token_of_row (moe_permute_map) instead of from x_perm. Arguments as in
+ * moe_route_bwd, with x [T,d] bf16 in place of x_perm.
+ */
+int moe_route_bwd_gather(const uint16_t *x, const int32_t *token_of_row, const float *topk_gate,
+                         const float *d_gate, const int32_t *row_of_assignment,
+                         const int32_t *group_offsets, const int32_t *group_counts, int T, int d,
+                         int E, int k, int64_t rows_cap, float *d_logits, float *dw_router,
+                         void *ws, size_t ws_bytes, moe_stream_t stream);
 
 /*
  * moe_permute_bwd - gradient of the layer input:

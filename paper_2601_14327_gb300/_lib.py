@@ -59,6 +59,10 @@ _SIGS = {
     "moe_grouped_ffn_bwd_wgrad": (I, [P, P, P, P, P, I, I, I, I64, P, P, P]),
     "moe_route_bwd": (I, [P, P, P, P, P, P, P, I, I, I, I, I64, P, P, P, SZ, P]),
     "moe_permute_bwd": (I, [P, P, P, P, P, I, I, I, I, P, P, SZ, P]),
+    "moe_permute_map": (I, [P, P, I, I, I, I64, P, P, P, P, P, SZ, P]),
+    "moe_grouped_ffn_fwd_gather": (I, [P, P, I, P, I, I, I, I64, P, P, P, P, P, P, SZ, P]),
+    "moe_grouped_ffn_bwd_wgrad_gather": (I, [P, P, P, I, P, P, P, I, I, I, I64, P, P, P]),
+    "moe_route_bwd_gather": (I, [P, P, P, P, P, P, P, I, I, I, I, I64, P, P, P, SZ, P]),
 }
 
 
@@ -265,6 +269,37 @@ def moe_route_bwd(x_perm, topk_idx, topk_gate, d_gate, row_of_assignment, group_
                   stream=None):
     _check("moe_route_bwd", load().moe_route_bwd(
         _ptr(x_perm), _ptr(topk_idx), _ptr(topk_gate), _ptr(d_gate), _ptr(row_of_assignment),
+        _ptr(group_offsets), _ptr(group_counts), T, d, E, k, rows_cap, _ptr(d_logits),
+        _ptr(dw_router), _ptr(ws), ws_bytes, _stream(stream)))
+
+
+def moe_permute_map(topk_idx, counts, T, E, k, rows_cap, group_offsets, group_counts,
+                    row_of_assignment, token_of_row, ws, ws_bytes, stream=None):
+    _check("moe_permute_map", load().moe_permute_map(
+        _ptr(topk_idx), _ptr(counts), T, E, k, rows_cap, _ptr(group_offsets), _ptr(group_counts),
+        _ptr(row_of_assignment), _ptr(token_of_row), _ptr(ws), ws_bytes, _stream(stream)))
+
+
+def moe_grouped_ffn_fwd_gather(x, token_of_row, T, group_offsets, E, d, F, rows_cap, w_gate_up,
+                               w_down, ab_saved, h, out_perm, ws, ws_bytes, stream=None):
+    _check("moe_grouped_ffn_fwd_gather", load().moe_grouped_ffn_fwd_gather(
+        _ptr(x), _ptr(token_of_row), T, _ptr(group_offsets), E, d, F, rows_cap, _ptr(w_gate_up),
+        _ptr(w_down), _ptr(ab_saved), _ptr(h), _ptr(out_perm), _ptr(ws), ws_bytes,
+        _stream(stream)))
+
+
+def moe_grouped_ffn_bwd_wgrad_gather(d_out_perm, x, token_of_row, T, h, d_ab, group_offsets, E,
+                                     d, F, rows_cap, dw_gate_up, dw_down, stream=None):
+    _check("moe_grouped_ffn_bwd_wgrad_gather", load().moe_grouped_ffn_bwd_wgrad_gather(
+        _ptr(d_out_perm), _ptr(x), _ptr(token_of_row), T, _ptr(h), _ptr(d_ab),
+        _ptr(group_offsets), E, d, F, rows_cap, _ptr(dw_gate_up), _ptr(dw_down), _stream(stream)))
+
+
+def moe_route_bwd_gather(x, token_of_row, topk_gate, d_gate, row_of_assignment, group_offsets,
+                         group_counts, T, d, E, k, rows_cap, d_logits, dw_router, ws, ws_bytes,
+                         stream=None):
+    _check("moe_route_bwd_gather", load().moe_route_bwd_gather(
+        _ptr(x), _ptr(token_of_row), _ptr(topk_gate), _ptr(d_gate), _ptr(row_of_assignment),
         _ptr(group_offsets), _ptr(group_counts), T, d, E, k, rows_cap, _ptr(d_logits),
         _ptr(dw_router), _ptr(ws), ws_bytes, _stream(stream)))
 

@@ -81,6 +81,9 @@ struct GemmParams {
   uint16_t *out;   // primary output
   uint16_t *out2;  // kGateUp: pre-activations [A|B] (32-row blocked, see ab_block_index)
   const uint16_t *aux;  // kDgradDown: saved pre-activations [rows, 2F]
+  // Gathered operand (kGateUp: A, kWgradGateUp: B): grouped row r reads row
+  // token_of_row[r] of x [T, d] instead of row r of X_perm (nullptr: X_perm).
+  const int32_t *token_of_row;
 };
 
 struct Tile {
@@ -525,7 +528,19 @@ struct PairTile {
   int e, goff, mp, nt, nkb, mtiles;
 };
 
-template <int MODE, int BN>
+__device__ __forceinline__ int4 ld_rows4(const int32_t *p) {
+  return __ldg(reinterpret_cast<const int4 *>(p));
+}
+
+// GATHER (kGateUp, kWgradGateUp): the X_perm operand is read from x through
+// token_of_row with 4-row TMA gathers, so X_perm is never materialized. The whole
+// producer warp issues them, one gather of 4 rows per lane and k-block: the 128
+// A rows of the tile (kGateUp), or 2 x 64 k-rows of B (kWgradGateUp, whose row
+// indices change every k-block and are loaded one k-block ahead). Measured on
+// GB300 at T=16384, d=4096, 48 live experts: both GEMMs take ~3.3x as long as with
+// X_perm tile loads (each k-block needs 32 gathers of 4 x 128 bytes where one tile
+// load moves 128 rows; the per-instruction cost of the gathers sets the pace).
+template <int MODE, int BN, bool GATHER>
 __global__ void __launch_bounds__(kThreads, 1)
     grouped_gemm_pair_kernel(const __grid_constant__ CUtensorMap tmA,
                              const __grid_constant__ CUtensorMap tmB,
@@ -640,7 +655,69 @@ __global__ void __launch_bounds__(kThreads, 1)
     return t;
   };
 
-  if (warp == 0) {
+  if (warp == 0 && GATHER) {
+    // ============ TMA producer, gathered operand (the whole warp in each CTA) ============
+    const uint32_t full_leader = tc::mapa(full_bar(0), 0);
+    const int box = lane >> 4, grp = lane & 15;  // kWgradGateUp: B box and 4-row group
+    uint32_t it = 0;
+    bool ok = true;
+    for (int tile = cluster; tile < total && ok; tile += nclusters) {
+      const PairTile t = decode(tile);
+      const int mt = 2 * t.mp + int(rank);
+      int4 rows4 = make_int4(0, 0, 0, 0), nxt = make_int4(0, 0, 0, 0);
+      // kGateUp: this lane's 4 rows of the tile (token 0 for the row block past an
+      // odd group end, which is computed but not stored)
+      if (MODE == kGateUp && mt < t.mtiles) rows4 = ld_rows4(p.token_of_row + t.goff + mt * BM + 4 * lane);
+      if (MODE == kWgradGateUp && t.nkb > 0) nxt = ld_rows4(p.token_of_row + t.goff + 4 * grp);
+      for (int kb = 0; kb < t.nkb; ++kb, ++it) {
+        const int s = it % STAGES;
+        const uint32_t ph = (it / STAGES) & 1u;
+        if (MODE == kWgradGateUp) {
+          rows4 = nxt;
+          if (kb + 1 < t.nkb) nxt = ld_rows4(p.token_of_row + t.goff + (kb + 1) * BK + 4 * grp);
+        }
+        int w_ok = 1;
+        if (lane == 0) w_ok = tc::mbar_wait(empty_bar(s), ph ^ 1u, kWaitLimitNs, abort_flag) ? 1 : 0;
+        w_ok = __shfl_sync(0xffffffffu, w_ok, 0);
+        if (!w_ok) {
+          if (lane == 0) fail(abort_flag);
+          ok = false;
+          break;
+        }
+        const uint32_t a_dst = sA0 + s * Sh::A_BYTES, b_dst = sB0 + s * Sh::B_BYTES;
+        const uint32_t fb = full_leader + 8u * s;
+        const int k0 = kb * BK;
+        if (lane == 0) {
+          if (leader) tc::mbar_arrive_expect_tx(full_bar(s), 2 * Sh::STAGE_BYTES);
+          if (MODE == kGateUp) {  // even CTA: gate rows, odd CTA: up rows
+            tc::tma_load_2d_pair(b_dst, &tmB, fb, k0, t.e * 2 * p.F + int(rank) * p.F + t.nt * 128);
+          } else {  // A = [dA | dB] of the group, MN-major
+            const int krow = t.goff + k0;
+#pragma unroll
+            for (int i = 0; i < BM / 64; ++i)
+              tc::tma_load_2d_pair(a_dst + i * 64 * 128, &tmA, fb, mt * BM + i * 64, krow);
+          }
+        }
+        if (MODE == kGateUp) {
+          tc::tma_gather4_pair(a_dst + uint32_t(lane) * 512u, &tmA, fb, k0, rows4.x, rows4.y,
+                               rows4.z, rows4.w);
+        } else if (box < BNH / 64) {
+          tc::tma_gather4_pair(b_dst + uint32_t(box) * 64u * 128u + uint32_t(grp) * 512u, &tmB, fb,
+                               t.nt * BN + int(rank) * BNH + box * 64, rows4.x, rows4.y, rows4.z,
+                               rows4.w);
+        }
+      }
+    }
+    // Drain (even CTA): its full barriers count the loads of both CTAs.
+    if (leader && lane == 0) {
+      for (int s = 0; s < STAGES; ++s) {
+        if (it > uint32_t(s)) {
+          const uint32_t n = (it - 1 - s) / STAGES;
+          if (!tc::mbar_wait(full_bar(s), n & 1u, kWaitLimitNs, &no_abort)) fail(abort_flag);
+        }
+      }
+    }
+  } else if (warp == 0) {
     // ============ TMA producer (one thread in each CTA) ============
     if (lane == 0) {
       const uint32_t full_leader = tc::mapa(full_bar(0), 0);
@@ -806,11 +883,11 @@ int launch_one(const CUtensorMap &a, const CUtensorMap &b, const CUtensorMap &o,
   return moe::launch_status(what);
 }
 
-template <int MODE, int BN>
+template <int MODE, int BN, bool GATHER>
 int launch_pair(const CUtensorMap &a, const CUtensorMap &b, const CUtensorMap &o,
                 const GemmParams &p, cudaStream_t s, const char *what) {
   using Sh = PairShape<BN>;
-  auto kern = grouped_gemm_pair_kernel<MODE, BN>;
+  auto kern = grouped_gemm_pair_kernel<MODE, BN, GATHER>;
   cudaLaunchAttribute at[1];
   at[0].id = cudaLaunchAttributeClusterDimension;
   at[0].val.clusterDim.x = 2;
@@ -849,20 +926,34 @@ int run_gemm(int N, const void *a_base, uint64_t a_rows, uint64_t a_cols, const 
   const bool pair = use_pair<MODE>();
   const int BN = (MODE == kGateUp || N % 256 == 0) ? 256 : 128;
   p.n_tiles = (MODE == kGateUp) ? N / 256 : N / BN;
+  const bool gather = p.token_of_row != nullptr;
+  if (gather && MODE != kGateUp && MODE != kWgradGateUp)
+    return moe::set_error(MOE_ERR_UNSUPPORTED, "%s: no gathered operand in this GEMM", what);
+  if (gather && !pair)
+    return moe::set_error(MOE_ERR_UNSUPPORTED, "%s: the gathered operand needs the CTA-pair kernel", what);
+  // the gathered operand's map is over x [T, d] with a one-row box (4-row gathers)
+  const bool gather_a = gather && MODE == kGateUp, gather_b = gather && MODE == kWgradGateUp;
   CUtensorMap ma, mb;
   int st;
-  if ((st = Tr::A_MN ? make_map(&ma, a_base, a_rows, a_cols, 64, BK, what)
-                     : make_map(&ma, a_base, a_rows, a_cols, BK, BM, what)))
+  if ((st = gather_a  ? make_map(&ma, a_base, a_rows, a_cols, BK, 1, what)
+            : Tr::A_MN ? make_map(&ma, a_base, a_rows, a_cols, 64, BK, what)
+                       : make_map(&ma, a_base, a_rows, a_cols, BK, BM, what)))
     return st;
   const uint32_t b_box_rows = pair ? uint32_t(BN / 2) : 128u;
-  if ((st = Tr::B_MN ? make_map(&mb, b_base, b_rows, b_cols, 64, BK, what)
-                     : make_map(&mb, b_base, b_rows, b_cols, BK, b_box_rows, what)))
+  if ((st = gather_b  ? make_map(&mb, b_base, b_rows, b_cols, 64, 1, what)
+            : Tr::B_MN ? make_map(&mb, b_base, b_rows, b_cols, 64, BK, what)
+                       : make_map(&mb, b_base, b_rows, b_cols, BK, b_box_rows, what)))
     return st;
   CUtensorMap mo;  // the epilogue's output, in 32 x 32 chunks
   if ((st = make_map(&mo, p.out, o_rows, o_cols, 32, 32, what, CU_TENSOR_MAP_SWIZZLE_64B))) return st;
   if (pair) {
-    return BN == 256 ? launch_pair<MODE, 256>(ma, mb, mo, p, s, what)
-                     : launch_pair<MODE, 128>(ma, mb, mo, p, s, what);
+    if constexpr (MODE == kGateUp || MODE == kWgradGateUp) {
+      if (gather)
+        return BN == 256 ? launch_pair<MODE, 256, true>(ma, mb, mo, p, s, what)
+                         : launch_pair<MODE, 128, true>(ma, mb, mo, p, s, what);
+    }
+    return BN == 256 ? launch_pair<MODE, 256, false>(ma, mb, mo, p, s, what)
+                     : launch_pair<MODE, 128, false>(ma, mb, mo, p, s, what);
   }
   return BN == 256 ? launch_one<MODE, 256>(ma, mb, mo, p, s, what)
                    : launch_one<MODE, 128>(ma, mb, mo, p, s, what);
@@ -917,6 +1008,45 @@ int moe_grouped_ffn_fwd(const uint16_t *x_perm, const int32_t *group_offsets, in
   q.out = out_perm;
   return run_gemm<kDown>(d, h, R, F, w_down, uint64_t(E) * d, F, R, d, q, s,
                          "moe_grouped_ffn_fwd: down GEMM");
+}
+
+int moe_grouped_ffn_fwd_gather(const uint16_t *x, const int32_t *token_of_row, int T,
+                               const int32_t *group_offsets, int E, int d, int F,
+                               int64_t rows_cap, const uint16_t *w_gate_up,
+                               const uint16_t *w_down, uint16_t *ab_saved, uint16_t *h,
+                               uint16_t *out_perm, void *ws, size_t ws_bytes, moe_stream_t stream) {
+  (void)ws;
+  (void)ws_bytes;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if (int st = check_common(E, d, F, rows_cap, "moe_grouped_ffn_fwd_gather")) return st;
+  if (T < 0) return moe::set_error(MOE_ERR_ARG, "moe_grouped_ffn_fwd_gather: T=%d", T);
+  const void *ptrs[] = {token_of_row, group_offsets, w_gate_up, w_down, ab_saved, h, out_perm};
+  for (const void *q : ptrs)
+    if (!q || !moe::aligned16(q))
+      return moe::set_error(MOE_ERR_ARG, "moe_grouped_ffn_fwd_gather: null or unaligned pointer");
+  if (T > 0 && (!x || !moe::aligned16(x)))
+    return moe::set_error(MOE_ERR_ARG, "moe_grouped_ffn_fwd_gather: null or unaligned x");
+  const uint64_t R = uint64_t(rows_cap);
+  GemmParams p{};
+  p.group_offsets = group_offsets;
+  p.E = E; p.d = d; p.F = F;
+  p.nkb = d / BK;
+  p.out = h;
+  p.out2 = ab_saved;
+  p.token_of_row = token_of_row;
+  // no tokens: no tile reads x; the map needs some valid base
+  const void *xa = T > 0 ? static_cast<const void *>(x) : static_cast<const void *>(h);
+  if (int st = run_gemm<kGateUp>(2 * F, xa, uint64_t(std::max(T, 1)), d, w_gate_up,
+                                 uint64_t(E) * 2 * F, d, R, F, p, s,
+                                 "moe_grouped_ffn_fwd_gather: gate/up GEMM"))
+    return st;
+  GemmParams q{};
+  q.group_offsets = group_offsets;
+  q.E = E; q.d = d; q.F = F;
+  q.nkb = F / BK;
+  q.out = out_perm;
+  return run_gemm<kDown>(d, h, R, F, w_down, uint64_t(E) * d, F, R, d, q, s,
+                         "moe_grouped_ffn_fwd_gather: down GEMM");
 }
 
 int moe_grouped_ffn_bwd_dgrad(const uint16_t *d_out_perm, const uint16_t *ab_saved,
@@ -974,6 +1104,40 @@ int moe_grouped_ffn_bwd_wgrad(const uint16_t *d_out_perm, const uint16_t *x_perm
   p.out = dw_gate_up;
   return run_gemm<kWgradGateUp>(d, d_ab, R, 2 * F, x_perm, R, d, uint64_t(E) * 2 * F, d, p, s,
                                 "moe_grouped_ffn_bwd: dW_gate_up GEMM");
+}
+
+int moe_grouped_ffn_bwd_wgrad_gather(const uint16_t *d_out_perm, const uint16_t *x,
+                                     const int32_t *token_of_row, int T, const uint16_t *h,
+                                     const uint16_t *d_ab, const int32_t *group_offsets, int E,
+                                     int d, int F, int64_t rows_cap, uint16_t *dw_gate_up,
+                                     uint16_t *dw_down, moe_stream_t stream) {
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if (int st = check_common(E, d, F, rows_cap, "moe_grouped_ffn_bwd_wgrad_gather")) return st;
+  if (T < 0) return moe::set_error(MOE_ERR_ARG, "moe_grouped_ffn_bwd_wgrad_gather: T=%d", T);
+  const void *ptrs[] = {d_out_perm, token_of_row, h, d_ab, group_offsets, dw_gate_up, dw_down};
+  for (const void *q : ptrs)
+    if (!q || !moe::aligned16(q))
+      return moe::set_error(MOE_ERR_ARG, "moe_grouped_ffn_bwd_wgrad_gather: null or unaligned pointer");
+  if (T > 0 && (!x || !moe::aligned16(x)))
+    return moe::set_error(MOE_ERR_ARG, "moe_grouped_ffn_bwd_wgrad_gather: null or unaligned x");
+  const uint64_t R = uint64_t(rows_cap);
+  int st;
+  GemmParams p{};
+  p.group_offsets = group_offsets;
+  p.E = E; p.d = d; p.F = F;
+  p.nkb = 0;
+  p.m_tiles_w = d / BM;
+  p.out = dw_down;
+  if ((st = run_gemm<kWgradDown>(F, d_out_perm, R, d, h, R, F, uint64_t(E) * d, F, p, s,
+                                 "moe_grouped_ffn_bwd_wgrad_gather: dW_down GEMM")))
+    return st;
+  p.m_tiles_w = 2 * F / BM;
+  p.out = dw_gate_up;
+  p.token_of_row = token_of_row;
+  const void *xb = T > 0 ? static_cast<const void *>(x) : static_cast<const void *>(dw_gate_up);
+  return run_gemm<kWgradGateUp>(d, d_ab, R, 2 * F, xb, uint64_t(std::max(T, 1)), d,
+                                uint64_t(E) * 2 * F, d, p, s,
+                                "moe_grouped_ffn_bwd_wgrad_gather: dW_gate_up GEMM");
 }
 
 int moe_grouped_ffn_bwd(const uint16_t *d_out_perm, const uint16_t *x_perm,

@@ -84,7 +84,8 @@ __global__ void __launch_bounds__(1024) perm_scan_kernel(
 __global__ void __launch_bounds__(kThreads) perm_rank_kernel(
     const int32_t *__restrict__ idx, int64_t A, int E, int nblk,
     const int32_t *__restrict__ hist_prefix, const int32_t *__restrict__ group_offsets,
-    int64_t rows_cap, int32_t *__restrict__ row_of_assignment) {
+    int64_t rows_cap, int32_t *__restrict__ row_of_assignment, int k,
+    int32_t *__restrict__ token_of_row) {
   __shared__ int wh[kWarps][256];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   for (int i = threadIdx.x; i < kWarps * 256; i += kThreads) (&wh[0][0])[i] = 0;
@@ -126,7 +127,20 @@ __global__ void __launch_bounds__(kThreads) perm_rank_kernel(
     if (e >= 0 && lane == leader) wh[warp][e] += __popc(peers);
     __syncwarp();
     if (a < A) row_of_assignment[a] = (e >= 0 && !overflow) ? row : -1;
+    if (token_of_row != nullptr && a < A && e >= 0 && !overflow) token_of_row[row] = int(a / k);
   }
+}
+
+// Pad rows of every group read token 0 (their products are multiplied by zero
+// downstream: the pad rows of d_out_perm and of the router's d_logits are zero).
+__global__ void __launch_bounds__(kThreads) pad_token_kernel(const int32_t *__restrict__ group_offsets,
+                                                             const int32_t *__restrict__ group_counts,
+                                                             int E, int64_t rows_cap,
+                                                             int32_t *__restrict__ token_of_row) {
+  const int e = blockIdx.x;
+  const int r0 = group_offsets[e] + group_counts[e];
+  const int r1 = int(min((long long)group_offsets[e + 1], (long long)rows_cap));
+  for (int r = r0 + threadIdx.x; r < r1; r += kThreads) token_of_row[r] = 0;
 }
 
 // One warp per token: read x[t,:] once, write it to its k grouped rows.
@@ -369,7 +383,7 @@ int moe_permute(const uint16_t *x, const int32_t *topk_idx, const int32_t *count
   if (int st = moe::launch_status("moe_permute: scan")) return st;
   if (A > 0) {
     MOE_LAUNCH("perm_rank", s, perm_rank_kernel<<<nblk, kThreads, 0, s>>>(topk_idx, A, E, nblk, hist, group_offsets, rows_cap,
-                                               row_of_assignment));
+                                               row_of_assignment, k, nullptr));
     if (int st = moe::launch_status("moe_permute: rank")) return st;
     MOE_LAUNCH("perm_gather", s, perm_gather_kernel<<<warp_grid(T), kThreads, 0, s>>>(x, row_of_assignment, T, d, k, rows_cap,
                                                          x_perm));
@@ -377,6 +391,40 @@ int moe_permute(const uint16_t *x, const int32_t *topk_idx, const int32_t *count
   }
   MOE_LAUNCH("pad_zero", s, pad_zero_kernel<<<dim3(E, kPadSplit), kThreads, 0, s>>>(group_offsets, group_counts, E, d, rows_cap, x_perm));
   return moe::launch_status("moe_permute: pad");
+}
+
+int moe_permute_map(const int32_t *topk_idx, const int32_t *counts, int T, int E, int k,
+                    int64_t rows_cap, int32_t *group_offsets, int32_t *group_counts,
+                    int32_t *row_of_assignment, int32_t *token_of_row, void *ws, size_t ws_bytes,
+                    moe_stream_t stream) {
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if (E < 1 || E > 256 || k < 1 || k > 8 || T < 0)
+    return moe::set_error(MOE_ERR_ARG, "moe_permute_map: sizes T=%d E=%d k=%d", T, E, k);
+  if (!group_offsets || !group_counts || !ws || !token_of_row ||
+      (T > 0 && (!topk_idx || !row_of_assignment)))
+    return moe::set_error(MOE_ERR_ARG, "moe_permute_map: null pointer");
+  if (rows_cap < moe_perm_rows_max(T, k, E))
+    return moe::set_error(MOE_ERR_ARG, "moe_permute_map: rows_cap %lld < %lld", (long long)rows_cap,
+                          (long long)moe_perm_rows_max(T, k, E));
+  if (rows_cap >= (int64_t(1) << 31))
+    return moe::set_error(MOE_ERR_UNSUPPORTED, "moe_permute_map: rows_cap >= 2^31");
+  const moe::WsLayout L = moe::ws_layout(T, 8, E, k, 0);
+  if (ws_bytes < L.perm_hist + size_t(E) * std::max<int64_t>(1, (int64_t(T) * k + kChunk - 1) / kChunk) * 4)
+    return moe::set_error(MOE_ERR_WORKSPACE, "moe_permute_map: workspace");
+  const int64_t A = int64_t(T) * k;
+  const int nblk = int(std::max<int64_t>(1, (A + kChunk - 1) / kChunk));
+  int32_t *hist = reinterpret_cast<int32_t *>(static_cast<char *>(ws) + L.perm_hist);
+  MOE_LAUNCH("perm_hist", s, perm_hist_kernel<<<nblk, kThreads, 0, s>>>(topk_idx, A, E, nblk, hist));
+  if (int st = moe::launch_status("moe_permute_map: hist")) return st;
+  MOE_LAUNCH("perm_scan", s, perm_scan_kernel<<<1, 1024, 0, s>>>(hist, E, nblk, counts, rows_cap, group_offsets, group_counts));
+  if (int st = moe::launch_status("moe_permute_map: scan")) return st;
+  if (A > 0) {
+    MOE_LAUNCH("perm_rank", s, perm_rank_kernel<<<nblk, kThreads, 0, s>>>(topk_idx, A, E, nblk, hist, group_offsets, rows_cap,
+                                               row_of_assignment, k, token_of_row));
+    if (int st = moe::launch_status("moe_permute_map: rank")) return st;
+  }
+  MOE_LAUNCH("pad_token", s, pad_token_kernel<<<E, kThreads, 0, s>>>(group_offsets, group_counts, E, rows_cap, token_of_row));
+  return moe::launch_status("moe_permute_map: pad");
 }
 
 int moe_unpermute_combine(const uint16_t *out_perm, const int32_t *row_of_assignment,
@@ -521,7 +569,7 @@ extern "C" int moe_permute_noalloc(const uint16_t *x, const int32_t *topk_idx,
   if (A > 0) {
     MOE_LAUNCH("perm_rank", s, perm_rank_kernel<<<nblk, kThreads, 0, s>>>(
                                    topk_idx, A, E, nblk, hist, group_offsets, rows_cap,
-                                   row_of_assignment));
+                                   row_of_assignment, k, nullptr));
     if (int st = moe::launch_status("moe_permute_noalloc: rank")) return st;
     MOE_LAUNCH("perm_gather", s, perm_gather_kernel<<<warp_grid(T), kThreads, 0, s>>>(
                                      x, row_of_assignment, T, d, k, rows_cap, x_perm));

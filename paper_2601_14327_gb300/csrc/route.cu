@@ -381,11 +381,12 @@ __global__ void route_bwd_dz_kernel(const float *__restrict__ gate, const float 
 }
 
 // One CTA per 128-row tile of the grouped layout: partial[tile, :] =
-// sum over the tile's real rows of dz_perm[r] * x_perm[r, :].
+// sum over the tile's real rows of dz_perm[r] * X_perm[r, :], where X_perm row r is
+// x_src row r, or x_src row token_of_row[r] when token_of_row is given (x itself).
 __global__ void __launch_bounds__(256) route_bwd_partial_kernel(
-    const uint16_t *__restrict__ x_perm, const float *__restrict__ dz_perm,
-    const int32_t *__restrict__ group_offsets, const int32_t *__restrict__ group_counts, int E,
-    int d, float *__restrict__ partial) {
+    const uint16_t *__restrict__ x_src, const int32_t *__restrict__ token_of_row,
+    const float *__restrict__ dz_perm, const int32_t *__restrict__ group_offsets,
+    const int32_t *__restrict__ group_counts, int E, int d, float *__restrict__ partial) {
   const int tile = blockIdx.x;
   const int row0 = tile * moe::kGroupPad;
   if (row0 >= group_offsets[E]) return;
@@ -403,8 +404,9 @@ __global__ void __launch_bounds__(256) route_bwd_partial_kernel(
     for (int q = 0; q < 8; ++q) acc[q] = 0.f;
     for (int r = row0; r < row_end; ++r) {
       const float w = dz_perm[r];
+      const size_t src = token_of_row != nullptr ? size_t(token_of_row[r]) : size_t(r);
       float f[8];
-      unpack8(ldg_nc_v4(x_perm + size_t(r) * d + c8 * 8), f);
+      unpack8(ldg_nc_v4(x_src + src * d + c8 * 8), f);
 #pragma unroll
       for (int q = 0; q < 8; ++q) acc[q] = fmaf(w, f[q], acc[q]);
     }
@@ -545,24 +547,24 @@ int moe_load_stats(const int32_t *topk_idx, int T, int k, int E, int32_t *counts
   return moe::launch_status("moe_load_stats: launch");
 }
 
-int moe_route_bwd(const uint16_t *x_perm, const int32_t *topk_idx, const float *topk_gate,
-                  const float *d_gate, const int32_t *row_of_assignment,
-                  const int32_t *group_offsets, const int32_t *group_counts, int T, int d, int E,
-                  int k, int64_t rows_cap, float *d_logits, float *dw_router, void *ws,
-                  size_t ws_bytes, moe_stream_t stream) {
-  (void)topk_idx;
-  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+}  // extern "C"
+
+namespace {
+int route_bwd_impl(const char *fn, const uint16_t *x_src, const int32_t *token_of_row,
+                   const float *topk_gate, const float *d_gate, const int32_t *row_of_assignment,
+                   const int32_t *group_offsets, const int32_t *group_counts, int T, int d, int E,
+                   int k, int64_t rows_cap, float *d_logits, float *dw_router, void *ws,
+                   size_t ws_bytes, cudaStream_t s) {
   if (E < 1 || E > 256 || k < 1 || k > 8 || T < 0 || d <= 0 || d % 8)
-    return moe::set_error(MOE_ERR_ARG, "moe_route_bwd: sizes");
-  if (!x_perm || !group_offsets || !group_counts || !dw_router || !ws ||
-      (T > 0 && (!topk_gate || !d_gate || !row_of_assignment || !d_logits)))
-    return moe::set_error(MOE_ERR_ARG, "moe_route_bwd: null pointer");
-  if (rows_cap < moe_perm_rows_max(T, k, E))
-    return moe::set_error(MOE_ERR_ARG, "moe_route_bwd: rows_cap too small");
-  if (!moe::aligned16(x_perm) || !moe::aligned16(ws))
-    return moe::set_error(MOE_ERR_ARG, "moe_route_bwd: alignment");
+    return moe::set_error(MOE_ERR_ARG, "%s: sizes", fn);
+  if (!group_offsets || !group_counts || !dw_router || !ws ||
+      (T > 0 && (!x_src || !topk_gate || !d_gate || !row_of_assignment || !d_logits)))
+    return moe::set_error(MOE_ERR_ARG, "%s: null pointer", fn);
+  if (rows_cap < moe_perm_rows_max(T, k, E)) return moe::set_error(MOE_ERR_ARG, "%s: rows_cap too small", fn);
+  if ((x_src && !moe::aligned16(x_src)) || !moe::aligned16(ws))
+    return moe::set_error(MOE_ERR_ARG, "%s: alignment", fn);
   const moe::WsLayout L = moe::ws_layout(T, d, E, k, 0);
-  if (ws_bytes < L.total) return moe::set_error(MOE_ERR_WORKSPACE, "moe_route_bwd: workspace");
+  if (ws_bytes < L.total) return moe::set_error(MOE_ERR_WORKSPACE, "%s: workspace", fn);
   float *dz_perm = reinterpret_cast<float *>(static_cast<char *>(ws) + L.dz_perm);
   float *partial = reinterpret_cast<float *>(static_cast<char *>(ws) + L.rb_partial);
   if (T > 0) {
@@ -570,13 +572,40 @@ int moe_route_bwd(const uint16_t *x_perm, const int32_t *topk_idx, const float *
                                                         rows_cap, d_logits, dz_perm));
     if (int st = moe::launch_status("moe_route_bwd: dz")) return st;
     const int tiles = int(rows_cap / moe::kGroupPad);
-    MOE_LAUNCH("route_bwd_partial", s, route_bwd_partial_kernel<<<tiles, 256, 0, s>>>(x_perm, dz_perm, group_offsets, group_counts, E,
-                                                   d, partial));
+    MOE_LAUNCH("route_bwd_partial", s, route_bwd_partial_kernel<<<tiles, 256, 0, s>>>(
+                                           x_src, token_of_row, dz_perm, group_offsets,
+                                           group_counts, E, d, partial));
     if (int st = moe::launch_status("moe_route_bwd: partial")) return st;
   }
   dim3 grid((d + 255) / 256, E);
   MOE_LAUNCH("route_bwd_reduce", s, route_bwd_reduce_kernel<<<grid, 256, 0, s>>>(partial, group_offsets, E, d, dw_router));
   return moe::launch_status("moe_route_bwd: reduce");
+}
+}  // namespace
+
+extern "C" {
+
+int moe_route_bwd(const uint16_t *x_perm, const int32_t *topk_idx, const float *topk_gate,
+                  const float *d_gate, const int32_t *row_of_assignment,
+                  const int32_t *group_offsets, const int32_t *group_counts, int T, int d, int E,
+                  int k, int64_t rows_cap, float *d_logits, float *dw_router, void *ws,
+                  size_t ws_bytes, moe_stream_t stream) {
+  (void)topk_idx;
+  if (!x_perm) return moe::set_error(MOE_ERR_ARG, "moe_route_bwd: null x_perm");
+  return route_bwd_impl("moe_route_bwd", x_perm, nullptr, topk_gate, d_gate, row_of_assignment,
+                        group_offsets, group_counts, T, d, E, k, rows_cap, d_logits, dw_router,
+                        ws, ws_bytes, reinterpret_cast<cudaStream_t>(stream));
+}
+
+int moe_route_bwd_gather(const uint16_t *x, const int32_t *token_of_row, const float *topk_gate,
+                         const float *d_gate, const int32_t *row_of_assignment,
+                         const int32_t *group_offsets, const int32_t *group_counts, int T, int d,
+                         int E, int k, int64_t rows_cap, float *d_logits, float *dw_router,
+                         void *ws, size_t ws_bytes, moe_stream_t stream) {
+  if (T > 0 && !token_of_row) return moe::set_error(MOE_ERR_ARG, "moe_route_bwd_gather: null token_of_row");
+  return route_bwd_impl("moe_route_bwd_gather", x, token_of_row, topk_gate, d_gate,
+                        row_of_assignment, group_offsets, group_counts, T, d, E, k, rows_cap,
+                        d_logits, dw_router, ws, ws_bytes, reinterpret_cast<cudaStream_t>(stream));
 }
 
 }  // extern "C"

@@ -144,6 +144,21 @@ __device__ __forceinline__ void tma_load_2d_pair(uint32_t dst, const void *map, 
       : "memory");
 }
 
+// Gathers four rows (r0..r3) of a 2-D tensor whose map has a one-row box, from
+// column c0 on, into four consecutive rows of this CTA's shared-memory tile at
+// `dst` (512 bytes for 128-byte rows; the map's swizzle applies by destination
+// address, as for a tile load); completion counted on an mbarrier of either CTA
+// of the pair (cluster address).
+__device__ __forceinline__ void tma_gather4_pair(uint32_t dst, const void *map, uint32_t bar_cluster,
+                                                 int c0, int r0, int r1, int r2, int r3) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.tile::gather4.mbarrier::complete_tx::bytes"
+      ".cta_group::2 [%0], [%1, {%3, %4, %5, %6, %7}], [%2];" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(bar_cluster), "r"(c0), "r"(r0), "r"(r1), "r"(r2),
+      "r"(r3)
+      : "memory");
+}
+
 // ---- tcgen05 ------------------------------------------------------------------
 __device__ __forceinline__ void tmem_alloc(uint32_t dst_smem, uint32_t ncols) {
   asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(dst_smem),

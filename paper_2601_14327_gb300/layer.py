@@ -27,11 +27,21 @@ class LayerShape:
 
 
 class MoELayerBuffers:
-    """Device buffers of one layer step (activations, grouped layout, grads)."""
+    """Device buffers of one layer step (activations, grouped layout, grads).
 
-    def __init__(self, shape: LayerShape, device="cuda", backward: bool = True):
+    gather=False (default): moe_permute writes X_perm and the GEMMs read it with tile
+    loads. gather=True: the grouped operand is read from x through token_of_row by the
+    GEMMs' 4-row TMA gathers (moe_permute_map and the *_gather calls), so X_perm is not
+    allocated; the results are identical, but on GB300 the gathers make the two GEMMs
+    that read X_perm about 3.3x slower (32 gathers of 4 x 128 bytes per 128-row k-block
+    against one tile load), far more than the separate gather pass costs."""
+
+    def __init__(self, shape: LayerShape, device="cuda", backward: bool = True,
+                 gather: bool = False):
         s = shape
         self.shape = s
+        self.gather = gather
+        self.x = None  # the forward's input, kept for the backward in gather mode
         R = s.rows_cap
         dev = torch.device(device)
         bf16, f32, i32 = torch.bfloat16, torch.float32, torch.int32
@@ -44,7 +54,12 @@ class MoELayerBuffers:
         self.group_offsets = torch.empty(s.E + 1, dtype=i32, device=dev)
         self.group_counts = torch.empty(s.E, dtype=i32, device=dev)
         self.row_of_assignment = torch.empty(s.T, s.k, dtype=i32, device=dev)
-        self.x_perm = torch.empty(R, s.d, dtype=bf16, device=dev)
+        if gather:
+            self.token_of_row = torch.empty(R, dtype=i32, device=dev)
+            self.x_perm = None
+        else:
+            self.token_of_row = None
+            self.x_perm = torch.empty(R, s.d, dtype=bf16, device=dev)
         self.ab = torch.empty(R, 2 * s.F, dtype=bf16, device=dev)
         self.h = torch.empty(R, s.F, dtype=bf16, device=dev)
         self.out_perm = torch.empty(R, s.d, dtype=bf16, device=dev)
@@ -78,10 +93,19 @@ def forward(b: MoELayerBuffers, x, w_router, bias, w_gate_up, w_down, active_mas
     s = b.shape
     R = s.rows_cap
     route(b, x, w_router, bias, active_mask, logits_in, keep_logits, stream)
-    L.moe_permute(x, b.topk_idx, b.counts, s.T, s.d, s.E, s.k, R, b.group_offsets,
-                  b.group_counts, b.row_of_assignment, b.x_perm, b.ws, b.ws_bytes, stream)
-    L.moe_grouped_ffn_fwd(b.x_perm, b.group_offsets, s.E, s.d, s.F, R, w_gate_up, w_down, b.ab,
-                          b.h, b.out_perm, b.ws, b.ws_bytes, stream)
+    if b.gather:
+        b.x = x
+        L.moe_permute_map(b.topk_idx, b.counts, s.T, s.E, s.k, R, b.group_offsets,
+                          b.group_counts, b.row_of_assignment, b.token_of_row, b.ws, b.ws_bytes,
+                          stream)
+        L.moe_grouped_ffn_fwd_gather(x, b.token_of_row, s.T, b.group_offsets, s.E, s.d, s.F, R,
+                                     w_gate_up, w_down, b.ab, b.h, b.out_perm, b.ws, b.ws_bytes,
+                                     stream)
+    else:
+        L.moe_permute(x, b.topk_idx, b.counts, s.T, s.d, s.E, s.k, R, b.group_offsets,
+                      b.group_counts, b.row_of_assignment, b.x_perm, b.ws, b.ws_bytes, stream)
+        L.moe_grouped_ffn_fwd(b.x_perm, b.group_offsets, s.E, s.d, s.F, R, w_gate_up, w_down,
+                              b.ab, b.h, b.out_perm, b.ws, b.ws_bytes, stream)
     L.moe_unpermute_combine(b.out_perm, b.row_of_assignment, b.topk_gate, s.T, s.d, s.k, b.y,
                             stream)
     return b.y
@@ -106,9 +130,14 @@ def backward(b: MoELayerBuffers, dy, w_router, w_gate_up, w_down, stream=None,
         ev = torch.cuda.Event()
         ev.record(main)
         side.wait_event(ev)
-    L.moe_route_bwd(b.x_perm, b.topk_idx, b.topk_gate, b.d_gate, b.row_of_assignment,
-                    b.group_offsets, b.group_counts, s.T, s.d, s.E, s.k, R, b.d_logits,
-                    b.dw_router, b.ws, b.ws_bytes, side)
+    if b.gather:
+        L.moe_route_bwd_gather(b.x, b.token_of_row, b.topk_gate, b.d_gate, b.row_of_assignment,
+                               b.group_offsets, b.group_counts, s.T, s.d, s.E, s.k, R,
+                               b.d_logits, b.dw_router, b.ws, b.ws_bytes, side)
+    else:
+        L.moe_route_bwd(b.x_perm, b.topk_idx, b.topk_gate, b.d_gate, b.row_of_assignment,
+                        b.group_offsets, b.group_counts, s.T, s.d, s.E, s.k, R, b.d_logits,
+                        b.dw_router, b.ws, b.ws_bytes, side)
     L.moe_grouped_ffn_bwd_dgrad(b.d_out_perm, b.ab, b.group_offsets, s.E, s.d, s.F, R,
                                 w_gate_up, w_down, b.d_ab, b.dx_perm, main)
     if overlap:
@@ -117,8 +146,13 @@ def backward(b: MoELayerBuffers, dy, w_router, w_gate_up, w_down, stream=None,
         side.wait_event(ev)
     L.moe_permute_bwd(b.dx_perm, b.row_of_assignment, b.topk_idx, b.d_logits, w_router, s.T,
                       s.d, s.E, s.k, b.dx, b.ws, b.ws_bytes, side)
-    L.moe_grouped_ffn_bwd_wgrad(b.d_out_perm, b.x_perm, b.h, b.d_ab, b.group_offsets, s.E, s.d,
-                                s.F, R, b.dw_gate_up, b.dw_down, main)
+    if b.gather:
+        L.moe_grouped_ffn_bwd_wgrad_gather(b.d_out_perm, b.x, b.token_of_row, s.T, b.h, b.d_ab,
+                                           b.group_offsets, s.E, s.d, s.F, R, b.dw_gate_up,
+                                           b.dw_down, main)
+    else:
+        L.moe_grouped_ffn_bwd_wgrad(b.d_out_perm, b.x_perm, b.h, b.d_ab, b.group_offsets, s.E,
+                                    s.d, s.F, R, b.dw_gate_up, b.dw_down, main)
     if overlap:
         ev = torch.cuda.Event()
         ev.record(side)

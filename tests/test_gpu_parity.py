@@ -312,3 +312,75 @@ def test_layer_without_tokens():
     torch.cuda.synchronize()
     assert (b.group_offsets.cpu() == 0).all()
     assert not b.dw_gate_up.any() and not b.dw_down.any() and not b.dw_router.any()
+
+
+# ---------------------------------------------------------------- gathered dispatch
+
+@pytest.mark.parametrize("T,E,k", [(3000, 64, 6), (1000, 128, 8), (257, 16, 2)])
+def test_permute_map_bit_exact(T, E, k):
+    """moe_permute_map: the grouped layout of the oracle, and the token of every row."""
+    dev = "cuda"
+    rng = np.random.default_rng(T)
+    oidx = np.stack([rng.choice(E, size=k, replace=False) for _ in range(T)]).astype(np.int32)
+    R = L.moe_perm_rows_max(T, k, E)
+    ws_bytes = L.moe_workspace_size(T, 128, E, k, 128)
+    ws = torch.empty(ws_bytes, dtype=torch.uint8, device=dev)
+    goff = torch.empty(E + 1, dtype=torch.int32, device=dev)
+    gcnt = torch.empty(E, dtype=torch.int32, device=dev)
+    row = torch.empty(T, k, dtype=torch.int32, device=dev)
+    tok = torch.full((R,), -7, dtype=torch.int32, device=dev)
+    L.moe_permute_map(torch.from_numpy(oidx).to(dev), None, T, E, k, R, goff, gcnt, row, tok, ws,
+                      ws_bytes)
+    torch.cuda.synchronize()
+    ooff, ocnt, orow = O.permutation(oidx, E, 128)
+    assert (goff.cpu().numpy() == ooff).all() and (gcnt.cpu().numpy() == ocnt).all()
+    assert (row.cpu().numpy() == orow).all()
+    tk = tok.cpu().numpy()
+    assert (tk[orow.reshape(-1)] == np.repeat(np.arange(T), k)).all()
+    for e in range(E):
+        assert (tk[ooff[e] + ocnt[e]:ooff[e + 1]] == 0).all()
+    assert (tk[ooff[E]:] == -7).all()  # rows past the layout are not written
+
+
+def _layer_both_ways(inp, E, k, mask=None):
+    dev = "cuda"
+    T, d = inp["x"].shape
+    F = inp["w_down"].shape[2]
+    g = {n: v.to(dev) for n, v in inp.items()}
+    m = None if mask is None else torch.as_tensor(mask, dtype=torch.uint8).to(dev)
+    out = []
+    for gather in (False, True):
+        b = layer.MoELayerBuffers(layer.LayerShape(T, d, E, k, F), dev, backward=True,
+                                  gather=gather)
+        layer.forward(b, g["x"], g["w_router"], g["bias"], g["w_gate_up"], g["w_down"], m)
+        layer.backward(b, g["dy"], g["w_router"], g["w_gate_up"], g["w_down"])
+        torch.cuda.synchronize()
+        out.append(b)
+    return out
+
+
+@pytest.mark.parametrize("T,d,E,k,F,n_masked", [(1500, 256, 16, 4, 256, 0),
+                                                (777, 384, 24, 8, 128, 5),
+                                                (1, 128, 8, 2, 128, 0),
+                                                (0, 128, 4, 2, 128, 0),
+                                                (2048, 256, 8, 1, 384, 3)])
+def test_gathered_layer_equals_materialized(T, d, E, k, F, n_masked):
+    """The gathered dispatch (X_perm never written) gives the materialized path's results
+    bit for bit: outputs, every gradient, and the saved activations on real rows."""
+    inp = case_inputs(T, d, E, k, F, seed=T + 3)
+    mask = None
+    if n_masked:
+        mask = np.ones(E, np.uint8)
+        mask[np.random.default_rng(E).choice(E, n_masked, replace=False)] = 0
+    a, b = _layer_both_ways(inp, E, k, mask)
+    assert torch.equal(a.row_of_assignment, b.row_of_assignment)
+    assert torch.equal(a.group_offsets, b.group_offsets)
+    for name in ["y", "dx", "dw_gate_up", "dw_down", "dw_router", "d_logits", "d_gate"]:
+        assert torch.equal(getattr(a, name), getattr(b, name)), name
+    rows = a.row_of_assignment.reshape(-1).long()
+    for name in ["h", "out_perm", "dx_perm"]:
+        assert torch.equal(getattr(a, name)[rows], getattr(b, name)[rows]), name
+    rr = rows.cpu().numpy()
+    ua = unblock_ab(a.ab.view(torch.int16).cpu().numpy(), F)
+    ub = unblock_ab(b.ab.view(torch.int16).cpu().numpy(), F)
+    assert (ua[rr] == ub[rr]).all()

@@ -141,7 +141,7 @@ class Workload:
     """Inputs, the one-time LAEP prune, and the buffers of one layer step."""
 
     def __init__(self, cfg_id: int, device: str, compact_override=None, tokens=None,
-                 experts=None, no_prune=False, bias=None, gather=False):
+                 experts=None, no_prune=False, bias=None, gather=False, overlap=True):
         c = synth.CONFIGS[cfg_id]
         if tokens or experts or no_prune or bias:  # a variant of the workload (profiling)
             import dataclasses
@@ -185,6 +185,7 @@ class Workload:
         self.bufs = layer.MoELayerBuffers(self.shape, device, backward=True, gather=gather)
 
         self.graph = None
+        self.overlap = overlap
 
     def step(self, x=None, dy=None):
         if self.graph is not None and x is None and dy is None:
@@ -197,7 +198,7 @@ class Workload:
         layer.forward(b, i["x"] if x is None else x, i["w_router"], i["bias"], i["w_gate_up"],
                       i["w_down"], self.mask)
         layer.backward(b, i["dy"] if dy is None else dy, i["w_router"], i["w_gate_up"],
-                       i["w_down"])
+                       i["w_down"], overlap=self.overlap)
 
     def make_graph(self, x=None, dy=None):
         """A CUDA graph of one whole step (both streams) on inputs x, dy. The library's calls
@@ -387,7 +388,8 @@ def laep_comparison(args, world, local, pruned_tps, wl_pruned):
     saved = wl_pruned.bufs
     wl_pruned.bufs = None
     torch.cuda.empty_cache()
-    wl_u = Workload(args.config, "cuda", no_prune=True, gather=bool(args.gather))
+    wl_u = Workload(args.config, "cuda", no_prune=True, gather=bool(args.gather),
+                    overlap=bool(args.overlap))
     for _ in range(args.warmup):
         wl_u.step()
     if args.graph:
@@ -413,7 +415,8 @@ def run_ours(args):
     L.load()
     peaks = measured_peaks()
     wl = Workload(args.config, "cuda", tokens=args.tokens, experts=args.experts,
-                  no_prune=args.no_prune, bias=args.bias, gather=bool(args.gather))
+                  no_prune=args.no_prune, bias=args.bias, gather=bool(args.gather),
+                  overlap=bool(args.overlap))
     s = wl.shape
     torch.cuda.synchronize()
     for _ in range(args.warmup):
@@ -640,6 +643,9 @@ def main():
     ap.add_argument("--gather", type=int, default=0,
                     help="dispatch through a materialized X_perm (0), or by 4-row TMA gathers "
                          "from x with X_perm never written (1; same results, slower GEMMs)")
+    ap.add_argument("--overlap", type=int, default=1,
+                    help="router backward and unpermute-sum on a second stream beside the "
+                         "GEMMs (1) or on the main stream after them (0)")
     ap.add_argument("--graph", type=int, default=1,
                     help="time replays of a CUDA graph of the whole step (1) or eager steps (0)")
     # smaller cases of the same kernels, for profiler captures

@@ -402,7 +402,26 @@ __global__ void __launch_bounds__(256) route_bwd_partial_kernel(
     float acc[8];
 #pragma unroll
     for (int q = 0; q < 8; ++q) acc[q] = 0.f;
-    for (int r = row0; r < row_end; ++r) {
+    int r = row0;
+    // eight rows per step: eight independent 16-byte loads in flight per thread
+    for (; r + 8 <= row_end; r += 8) {
+      uint4 v[8];
+      float w[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        w[u] = dz_perm[r + u];
+        const size_t src = token_of_row != nullptr ? size_t(token_of_row[r + u]) : size_t(r + u);
+        v[u] = ldg_nc_v4(x_src + src * d + c8 * 8);
+      }
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        float f[8];
+        unpack8(v[u], f);
+#pragma unroll
+        for (int q = 0; q < 8; ++q) acc[q] = fmaf(w[u], f[q], acc[q]);
+      }
+    }
+    for (; r < row_end; ++r) {
       const float w = dz_perm[r];
       const size_t src = token_of_row != nullptr ? size_t(token_of_row[r]) : size_t(r);
       float f[8];

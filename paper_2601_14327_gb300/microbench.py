@@ -33,7 +33,8 @@ def _time(fn, iters, warmup):
 
 def main():
     ap = argparse.ArgumentParser()
-    ap.add_argument("call", choices=["route", "permute", "combine"])
+    ap.add_argument("call", choices=["route", "permute", "combine", "permute_bwd",
+                                     "permute_bwd_norouter", "route_bwd"])
     ap.add_argument("--T", type=int, default=16384)
     ap.add_argument("--d", type=int, default=4096)
     ap.add_argument("--E", type=int, default=64)
@@ -76,6 +77,23 @@ def main():
         if a.call == "permute":
             ms = _time(permute, a.iters, a.warmup)
             nbytes = 2 * T * d + 2 * T * k * d
+        elif a.call.startswith("permute_bwd"):
+            permute()
+            dl = torch.randn(T, k, generator=gen, device=dev) * 0.1
+            dx = torch.empty(T, d, dtype=torch.bfloat16, device=dev)
+            router = a.call == "permute_bwd"
+            ms = _time(lambda: L.moe_permute_bwd(xp, row, idx, dl if router else None,
+                                                 w if router else None, T, d, E, k, dx, ws,
+                                                 ws_bytes), a.iters, a.warmup)
+            nbytes = 2 * T * k * d + 2 * T * d
+        elif a.call == "route_bwd":
+            permute()
+            dg = torch.randn(T, k, generator=gen, device=dev)
+            dl = torch.empty(T, k, dtype=torch.float32, device=dev)
+            dw = torch.empty(d, E, dtype=torch.float32, device=dev)
+            ms = _time(lambda: L.moe_route_bwd(xp, idx, gate, dg, row, goff, gcnt, T, d, E, k, R,
+                                               dl, dw, ws, ws_bytes), a.iters, a.warmup)
+            nbytes = 2 * T * k * d
         else:
             permute()
             y = torch.empty(T, d, dtype=torch.bfloat16, device=dev)

@@ -9,8 +9,9 @@
 // the expert loads, and empty groups produce no tile. In the weight-gradient
 // GEMMs (reduction over a group's rows, so tile cost ~ group size) the
 // experts are ordered heaviest first, the longest-processing-time order that
-// Algorithm 2's greedy balancing also uses; experts without rows come last (their
-// tiles are zero stores only).
+// Algorithm 2's greedy balancing also uses; experts without rows get no tile: the
+// epilogue warps store their zero gradients up front, while the first tiles' MMAs
+// run (CTA-pair kernel; the one-SM kernel stores them as tiles at the end).
 //
 // Warps: 0 issues TMA loads, 1 owns TMEM and issues the MMAs, 2..9 are the epilogue
 // (two per TMEM lane quarter, each taking half of the tile's columns).
@@ -237,6 +238,26 @@ __device__ __forceinline__ void epilogue_tile(const GemmParams &p, const CUtenso
       stage_and_store(tmO, stage, lane, v, nt * BN + c, trow);
     }
   }
+}
+
+// Zeroes this warp's 2 KB staging chunk (after its earlier stores have read it).
+__device__ __forceinline__ void zero_fill_stage(uint32_t stage, int lane) {
+  if (lane == 0) tc::bulk_wait_read0();
+  __syncwarp();
+  const uint4 z = make_uint4(0, 0, 0, 0);
+#pragma unroll
+  for (uint32_t c = 0; c < 4; ++c) st_shared_v4(stage + uint32_t(lane) * 64u + c * 16u, z);
+  tc::fence_proxy_async_smem();
+  __syncwarp();
+}
+// One lane: stores the staging chunk to every 32-column chunk of this warp's column
+// half of output tile (trow, nt), as one bulk group.
+template <int BN>
+__device__ __forceinline__ void store_chunks_from(const CUtensorMap *tmO, uint32_t stage, int trow,
+                                                  int nt, int half) {
+  for (int c = half * (BN / 2); c < (half + 1) * (BN / 2); c += 32)
+    tc::tma_store_2d(tmO, stage, nt * BN + c, trow);
+  tc::bulk_commit();
 }
 
 // Zero weight gradient of an expert without rows: this warp's 32 rows and column half.
@@ -621,14 +642,23 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
   __syncthreads();
   if (threadIdx.x == 0) {
-    int acc = 0;
+    // Weight gradients: experts without rows get no tile in the list (they come last
+    // in the heaviest-first order); their zero gradients are stored by the epilogue
+    // warps up front instead, while the first tiles' MMAs run (misc[2] = their count).
+    int acc = 0, n_empty = 0;
     for (int i = 0; i < E; ++i) {
       s_prefix[i] = acc;
       const int e = s_order[i];
-      const int mt = Tr::WGRAD ? p.m_tiles_w : (s_goff[e + 1] - s_goff[e]) / BM;
+      const int rows = s_goff[e + 1] - s_goff[e];
+      if (Tr::WGRAD && rows == 0) {
+        ++n_empty;
+        continue;
+      }
+      const int mt = Tr::WGRAD ? p.m_tiles_w : rows / BM;
       acc += ((mt + 1) / 2) * p.n_tiles;
     }
     s_prefix[E] = acc;
+    misc[2] = n_empty;
   }
   tc::fence_before_sync();
   __syncthreads();
@@ -812,18 +842,28 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t stage = stage_base + uint32_t(warp - 2) * kStageBytes;
     const int r_in_tile = q * 32 + lane;
     const uint32_t tempty_leader = tc::mapa(tempty_bar(0), 0);
+    if (Tr::WGRAD) {
+      // Experts without rows: their weight gradient is exactly zero. Units of 128 rows
+      // x BN columns, spread over all CTAs; every store reads the same zeroed chunk.
+      const int n_empty = misc[2];
+      const int per_e = p.m_tiles_w * p.n_tiles;
+      const int units = n_empty * per_e;
+      if (int(blockIdx.x) < units) {
+        const int M_out = p.m_tiles_w * BM;
+        zero_fill_stage(stage, lane);
+        for (int u = int(blockIdx.x); u < units; u += int(gridDim.x)) {
+          const int e = s_order[E - n_empty + u / per_e];
+          const int rem = u % per_e;
+          const int mb = rem / p.n_tiles, nt = rem - mb * p.n_tiles;
+          if (lane == 0) store_chunks_from<BN>(&tmO, stage, e * M_out + mb * BM + q * 32, nt, half);
+        }
+      }
+    }
     uint32_t tcount = 0;
     for (int tile = cluster; tile < total; tile += nclusters) {
       const PairTile t = decode(tile);
       const int mt = 2 * t.mp + int(rank);
       const bool mine = mt < t.mtiles;  // this CTA's row block exists
-      if (Tr::WGRAD && t.nkb == 0) {
-        if (mine) {  // empty group: its weight gradient is exactly zero
-          const int M_out = p.m_tiles_w * BM;
-          zero_tile_store<BN>(&tmO, stage, lane, t.e * M_out + mt * BM + q * 32, t.nt, half);
-        }
-        continue;
-      }
       const uint32_t a = tcount & 1u, aph = (tcount >> 1) & 1u;
       const bool ok = tc::mbar_wait(tfull_bar(a), aph, kWaitLimitNs, abort_flag);
       __syncwarp();

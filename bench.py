@@ -182,7 +182,9 @@ class Workload:
                 self.mask = mask.to(device)
         self.shape = layer.LayerShape(T, d, E, k, F)
         self.E_live = E - (self.n_pruned if self.mask is not None else 0)
-        self.bufs = layer.MoELayerBuffers(self.shape, device, backward=True, gather=gather)
+        self.backward = c.backward  # the forward-only workloads time the forward pass
+        self.bufs = layer.MoELayerBuffers(self.shape, device, backward=self.backward,
+                                          gather=gather)
 
         self.graph = None
         self.overlap = overlap
@@ -197,8 +199,9 @@ class Workload:
         i, b = self.inp, self.bufs
         layer.forward(b, i["x"] if x is None else x, i["w_router"], i["bias"], i["w_gate_up"],
                       i["w_down"], self.mask)
-        layer.backward(b, i["dy"] if dy is None else dy, i["w_router"], i["w_gate_up"],
-                       i["w_down"], overlap=self.overlap)
+        if self.backward:
+            layer.backward(b, i["dy"] if dy is None else dy, i["w_router"], i["w_gate_up"],
+                           i["w_down"], overlap=self.overlap)
 
     def make_graph(self, x=None, dy=None):
         """A CUDA graph of one whole step (both streams) on inputs x, dy. The library's calls
@@ -268,13 +271,14 @@ def replica_throughput(world, tokens_per_rank, steps, ms_max):
     return world * tokens_per_rank * steps / (ms_max / 1e3)
 
 
-def oracle_sample(wl_inputs_host, mask_host, k, n_tok):
-    """Runs the CPU oracle over the first n_tok tokens; returns (seconds, threads)."""
+def oracle_sample(wl_inputs_host, mask_host, k, n_tok, backward=True):
+    """Runs the CPU oracle over the first n_tok tokens (forward, and backward unless the
+    workload is forward-only); returns the seconds it took."""
     from oracle import moe_oracle as O
     h = wl_inputs_host
     t0 = time.perf_counter()
     O.moe_layer(h["x"][:n_tok], h["w_router"], h["bias"], mask_host, k, h["w_gate_up"],
-                h["w_down"], dy=h["dy"][:n_tok])
+                h["w_down"], dy=h["dy"][:n_tok] if backward else None)
     return time.perf_counter() - t0
 
 
@@ -290,29 +294,39 @@ def host_inputs(inp, n_tok):
     return out
 
 
-def timed_steps(wl, steps, world, local, per_kernel_timing=True):
+def timed_steps(wl, steps, world, local, per_kernel_timing=True, flush=None):
     """K timed steps between barrier+synchronize; returns (max-over-ranks ms, per-kernel
-    CUDA-event table, clock samples)."""
+    CUDA-event table, clock samples). With `flush` (a buffer larger than L2) the buffer is
+    rewritten before every step and only the steps are timed (an event pair per step)."""
     stream = torch.cuda.current_stream()
     clocks = ClockSampler(local)
     L.moe_timing_enable(per_kernel_timing)
     L.moe_timing_read(reset=True)
-    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(steps if flush is not None else 1)]
     barrier(world)
     torch.cuda.synchronize()
     clocks.start()
     time.sleep(0.3)  # let the sampler start
-    ev0.record(stream)
-    for _ in range(steps):
-        wl.step()
-    ev1.record(stream)
+    if flush is None:
+        ev[0][0].record(stream)
+        for _ in range(steps):
+            wl.step()
+        ev[0][1].record(stream)
+    else:
+        for i in range(steps):
+            flush.zero_()
+            ev[i][0].record(stream)
+            wl.step()
+            ev[i][1].record(stream)
     torch.cuda.synchronize()
     barrier(world)
     clk = clocks.stop()
     L.moe_timing_enable(False)
     per_kernel = L.moe_timing_read(reset=True)
     assert L.moe_device_error(clear=True) == 0, "device error during the timed steps"
-    return max_over_ranks(ev0.elapsed_time(ev1), world), per_kernel, clk
+    ms = sum(a.elapsed_time(b) for a, b in ev)
+    return max_over_ranks(ms, world), per_kernel, clk
 
 
 def group_bound_seconds(shape, counts, peaks):
@@ -425,15 +439,20 @@ def run_ours(args):
     assert L.moe_device_error(clear=True) == 0, "device error during warm-up"
 
     stream = torch.cuda.current_stream()
+    # a 256 MB buffer rewritten before every timed step evicts the step's data from L2
+    flush = (torch.empty(256 << 20, dtype=torch.uint8, device="cuda") if args.flush_l2
+             else None)
     if args.graph:
         # per-kernel CUDA-event table from eager steps, the timed steps replay a graph
-        _, per_kernel, _ = timed_steps(wl, args.steps, world, local, per_kernel_timing=True)
+        _, per_kernel, _ = timed_steps(wl, args.steps, world, local, per_kernel_timing=True,
+                                       flush=flush)
         wl.capture()
         for _ in range(args.warmup):
             wl.step()
-        ms_total, _, clk = timed_steps(wl, args.steps, world, local, per_kernel_timing=False)
+        ms_total, _, clk = timed_steps(wl, args.steps, world, local, per_kernel_timing=False,
+                                       flush=flush)
     else:
-        ms_total, per_kernel, clk = timed_steps(wl, args.steps, world, local)
+        ms_total, per_kernel, clk = timed_steps(wl, args.steps, world, local, flush=flush)
     ms_step = ms_total / args.steps
     tokens_per_s = replica_throughput(world, s.T, args.steps, ms_total)
     launches = sum(n for n, _ in per_kernel.values())
@@ -444,7 +463,7 @@ def run_ours(args):
     dom = max(gemm_ms, key=lambda n: per_kernel[n][1])
     dom_tflops = flops[dom] / (gemm_ms[dom] / 1e3) / 1e12
     all_gemm_ms = sum(per_kernel[n][1] for n in gemm_ms) / args.steps
-    all_gemm_tflops = sum(flops.values()) / (all_gemm_ms / 1e3) / 1e12
+    all_gemm_tflops = sum(flops[n] for n in gemm_ms) / (all_gemm_ms / 1e3) / 1e12
     peak = peaks["bf16_tflops_sustained"]
     kernel_table = kernel_report(wl, per_kernel, args.steps, peaks)
     gb = group_bound_seconds(wl.shape, wl.bufs.counts.cpu().tolist(), peaks)
@@ -455,31 +474,36 @@ def run_ours(args):
         laep = laep_comparison(args, world, local, tokens_per_s, wl)
 
     # end to end through the public API: every step uploads its inputs from pinned host
-    # memory and downloads its results (y, dx). A copy stream and two input slots pipeline
-    # the copies with the compute: step i+2's inputs and step i's results move while
-    # step i+1 computes; the first uploads and the last download are inside the timed region.
+    # memory and downloads its results (x, dy in; y, dx out; forward-only workloads: x in,
+    # y out). A copy stream and two device slots pipeline the copies with the compute:
+    # step i+2's inputs and step i's results move while step i+1 computes; the first
+    # uploads and the last downloads are inside the timed region.
     e2e = None
     if not args.no_e2e:
-        x_h = wl.inp["x"].cpu().pin_memory()
-        dy_h = wl.inp["dy"].cpu().pin_memory()
-        y_h = [torch.empty_like(x_h).pin_memory() for _ in range(2)]
-        dx_h = [torch.empty_like(x_h).pin_memory() for _ in range(2)]
-        x_d = [torch.empty_like(wl.inp["x"]) for _ in range(2)]
-        dy_d = [torch.empty_like(wl.inp["dy"]) for _ in range(2)]
-        y_d = [wl.bufs.y, torch.empty_like(wl.bufs.y)]   # results alternate between two slots
-        dx_d = [wl.bufs.dx, torch.empty_like(wl.bufs.dx)]
+        in_names = ["x", "dy"] if wl.backward else ["x"]
+        out_names = ["y", "dx"] if wl.backward else ["y"]
+        host_in = {n: wl.inp[n].cpu().pin_memory() for n in in_names}
+        dev_in = [{n: torch.empty_like(wl.inp[n]) for n in in_names} for _ in range(2)]
+        dev_out = [{n: getattr(wl.bufs, n) for n in out_names},  # results alternate slots
+                   {n: torch.empty_like(getattr(wl.bufs, n)) for n in out_names}]
+        host_out = [{n: torch.empty_like(dev_out[0][n], device="cpu").pin_memory()
+                     for n in out_names} for _ in range(2)]
         for j in range(2):
-            x_d[j].copy_(x_h)
-            dy_d[j].copy_(dy_h)
+            for n in in_names:
+                dev_in[j][n].copy_(host_in[n])
 
         def use_slot(j):
-            wl.bufs.y, wl.bufs.dx = y_d[j], dx_d[j]
+            for n in out_names:
+                setattr(wl.bufs, n, dev_out[j][n])
+
+        def inputs(j):
+            return dev_in[j]["x"], dev_in[j].get("dy")
 
         graphs = []
         for j in range(2):
             use_slot(j)
-            wl.eager_step(x_d[j], dy_d[j])
-            graphs.append(wl.make_graph(x_d[j], dy_d[j]) if args.graph else None)
+            wl.eager_step(*inputs(j))
+            graphs.append(wl.make_graph(*inputs(j)) if args.graph else None)
         copy = torch.cuda.Stream()
         in_ready = [torch.cuda.Event() for _ in range(2)]
         step_done = [torch.cuda.Event() for _ in range(2)]
@@ -487,8 +511,8 @@ def run_ours(args):
 
         def upload(j):
             with torch.cuda.stream(copy):
-                x_d[j].copy_(x_h, non_blocking=True)
-                dy_d[j].copy_(dy_h, non_blocking=True)
+                for n in in_names:
+                    dev_in[j][n].copy_(host_in[n], non_blocking=True)
                 in_ready[j].record(copy)
 
         def run(i):
@@ -500,12 +524,12 @@ def run_ours(args):
                 graphs[j].replay()
             else:
                 use_slot(j)
-                wl.eager_step(x_d[j], dy_d[j])
+                wl.eager_step(*inputs(j))
             step_done[j].record(stream)
             with torch.cuda.stream(copy):
                 copy.wait_event(step_done[j])
-                y_h[j].copy_(y_d[j], non_blocking=True)
-                dx_h[j].copy_(dx_d[j], non_blocking=True)
+                for n in out_names:
+                    host_out[j][n].copy_(dev_out[j][n], non_blocking=True)
                 out_copied[j].record(copy)
             if i + 2 < args.steps:
                 upload(j)  # ordered after step i's downloads on the copy stream
@@ -527,19 +551,21 @@ def run_ours(args):
         barrier(world)
         use_slot(0)
         e_ms = max_over_ranks(ev0.elapsed_time(ev1), world)
-        nbytes = x_h.numel() * 2
+        nb = lambda ts: sum(t.numel() * t.element_size() for t in ts)
         e2e = {"value": round(replica_throughput(world, s.T, args.steps, e_ms), 1),
                "unit": "tokens/s",
-               "h2d_bytes_per_step": 2 * nbytes, "d2h_bytes_per_step": 2 * nbytes,
-               "note": "x, dy uploaded and y, dx downloaded every step on a copy stream, "
-                       "overlapped with the neighbouring steps' compute"}
+               "h2d_bytes_per_step": nb(host_in.values()),
+               "d2h_bytes_per_step": nb(host_out[0].values()),
+               "note": f"{', '.join(in_names)} uploaded and {', '.join(out_names)} downloaded "
+                       "every step on a copy stream, overlapped with the neighbouring steps' "
+                       "compute"}
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        n_tok = args.cpu_tokens
+        n_tok = min(args.cpu_tokens, s.T)
         hin = host_inputs(wl.inp, n_tok)
         mask_h = None if wl.mask is None else wl.mask.cpu().numpy()
-        secs = oracle_sample(hin, mask_h, s.k, n_tok)
+        secs = oracle_sample(hin, mask_h, s.k, n_tok, backward=wl.backward)
         cpu = {"value": round(n_tok / secs, 3), "unit": "tokens/s",
                "cores": int(os.environ.get("OPENBLAS_NUM_THREADS", NCPU)), "kind": "oracle",
                "sample": f"first {n_tok} of {s.T} tokens of the same layer step (all {s.E} experts, "
@@ -553,8 +579,11 @@ def run_ours(args):
         "data": "synthetic (seeded; random-init expert weights)",
         "config": {"workload": c.name, "T": s.T, "d_model": s.d, "experts": c.E,
                    "experts_live": wl.E_live, "top_k": s.k, "d_ff": s.F, "gate_bias": c.bias,
-                   "pruned": wl.n_pruned, "l2": "working set far above L2 (x 134 MB, expert "
-                   "weights GBs); no flush", "parallelism": "replicas" if world > 1 else "1 GPU",
+                   "pruned": wl.n_pruned, "pass": "forward+backward" if wl.backward else "forward",
+                   "l2": ("256 MB buffer rewritten before every timed step" if args.flush_l2
+                          else "no flush (working set: x %.0f MB, expert weights %.2f GB)"
+                          % (2 * s.T * s.d / 1e6, 6 * s.E * s.d * s.F / 1e9)),
+                   "parallelism": "replicas" if world > 1 else "1 GPU",
                    "dispatch": ("TMA gathers from x (X_perm not materialized)" if args.gather
                                 else "materialized X_perm")},
         "grouped_gemm": {"tflops": round(all_gemm_tflops, 1),
@@ -593,7 +622,7 @@ def run_reference(args):
     if rank != 0:
         return
     c = synth.CONFIGS[args.config]
-    n_tok = args.ref_tokens
+    n_tok = min(args.ref_tokens, c.T)
     dev = "cuda" if torch.cuda.is_available() else "cpu"
     inp = synth.make_config_inputs(args.config, device=dev)
     mask_h = None
@@ -608,14 +637,16 @@ def run_reference(args):
     hin = host_inputs(inp, n_tok)
     del inp
     for _ in range(args.warmup):
-        oracle_sample(hin, mask_h, c.k, n_tok)
+        oracle_sample(hin, mask_h, c.k, n_tok, backward=c.backward)
     secs = 0.0
     for _ in range(args.steps):
-        secs += oracle_sample(hin, mask_h, c.k, n_tok)
+        secs += oracle_sample(hin, mask_h, c.k, n_tok, backward=c.backward)
     v = n_tok * args.steps / secs
     cores = int(os.environ.get("OPENBLAS_NUM_THREADS", NCPU))
-    sample = (f"first {n_tok} of {c.T} tokens per step, full layer fwd+bwd over all {E} experts "
-              f"(16 least-loaded masked when the workload prunes), fp64 numpy oracle")
+    sample = (f"first {n_tok} of {c.T} tokens per step, full layer "
+              f"{'fwd+bwd' if c.backward else 'forward'} over all {E} experts"
+              + (f" ({c.prune_lowest} least-loaded masked)" if c.prune_lowest else "")
+              + ", fp64 numpy oracle")
     print(json.dumps({
         "impl": "reference", "metric": METRIC, "value": round(v, 3), "unit": "tokens/s",
         "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
@@ -646,6 +677,8 @@ def main():
     ap.add_argument("--overlap", type=int, default=1,
                     help="router backward and unpermute-sum on a second stream beside the "
                          "GEMMs (1) or on the main stream after them (0)")
+    ap.add_argument("--flush-l2", action="store_true",
+                    help="rewrite a 256 MB buffer before every timed step (time the steps only)")
     ap.add_argument("--graph", type=int, default=1,
                     help="time replays of a CUDA graph of the whole step (1) or eager steps (0)")
     # smaller cases of the same kernels, for profiler captures

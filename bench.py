@@ -141,7 +141,8 @@ class Workload:
     """Inputs, the one-time LAEP prune, and the buffers of one layer step."""
 
     def __init__(self, cfg_id: int, device: str, compact_override=None, tokens=None,
-                 experts=None, no_prune=False, bias=None, gather=False, overlap=True):
+                 experts=None, no_prune=False, bias=None, gather=False, overlap=True,
+                 backward=None):
         c = synth.CONFIGS[cfg_id]
         if tokens or experts or no_prune or bias:  # a variant of the workload (profiling)
             import dataclasses
@@ -182,7 +183,8 @@ class Workload:
                 self.mask = mask.to(device)
         self.shape = layer.LayerShape(T, d, E, k, F)
         self.E_live = E - (self.n_pruned if self.mask is not None else 0)
-        self.backward = c.backward  # the forward-only workloads time the forward pass
+        # the forward-only workloads time the forward pass (backward=True forces both)
+        self.backward = c.backward if backward is None else bool(backward)
         self.bufs = layer.MoELayerBuffers(self.shape, device, backward=self.backward,
                                           gather=gather)
 

@@ -401,6 +401,16 @@ int moe_permute_bwd(const uint16_t *dx_perm, const int32_t *row_of_assignment,
                     int T, int d, int E, int k, uint16_t *dx, void *ws, size_t ws_bytes,
                     moe_stream_t stream);
 
+/*
+ * moe_selftest_wait_timeout - failure-detection self-test (no counterpart in the
+ * paper). Launches one thread that waits, with the bounded pipeline wait the GEMM
+ * and router kernels use on their mbarriers, on an mbarrier nothing arrives on.
+ * After limit_ns nanoseconds (1e6 .. 2e9) the wait gives up, the kernel records
+ * MOE_DEV_WAIT_TIMEOUT in the device error word (read with moe_device_error) and
+ * returns; the context stays usable. Nothing else is touched.
+ */
+int moe_selftest_wait_timeout(int64_t limit_ns, moe_stream_t stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -63,6 +63,7 @@ _SIGS = {
     "moe_grouped_ffn_fwd_gather": (I, [P, P, I, P, I, I, I, I64, P, P, P, P, P, P, SZ, P]),
     "moe_grouped_ffn_bwd_wgrad_gather": (I, [P, P, P, I, P, P, P, I, I, I, I64, P, P, P]),
     "moe_route_bwd_gather": (I, [P, P, P, P, P, P, P, I, I, I, I, I64, P, P, P, SZ, P]),
+    "moe_selftest_wait_timeout": (I, [I64, P]),
 }
 
 
@@ -309,3 +310,7 @@ def moe_permute_bwd(dx_perm, row_of_assignment, topk_idx, d_logits, w_router, T,
     _check("moe_permute_bwd", load().moe_permute_bwd(
         _ptr(dx_perm), _ptr(row_of_assignment), _ptr(topk_idx), _ptr(d_logits), _ptr(w_router),
         T, d, E, k, _ptr(dx), _ptr(ws), ws_bytes, _stream(stream)))
+
+
+def moe_selftest_wait_timeout(limit_ns, stream=None):
+    _check("moe_selftest_wait_timeout", load().moe_selftest_wait_timeout(limit_ns, _stream(stream)))

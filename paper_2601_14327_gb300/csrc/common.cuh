@@ -8,6 +8,8 @@
 
 #include <algorithm>
 
+#include <nvtx3/nvToolsExt.h>
+
 #include "../../include/moe_laep.h"
 
 // ---------------------------------------------------------------- host side
@@ -54,12 +56,16 @@ int gemm_dev_error(int clear, int *code);
 }  // namespace moe
 
 // Launches a kernel (the variadic part is the launch statement) under the
-// timing registry, then checks the launch.
+// timing registry and inside an NVTX range named after it (a profiler can select
+// the library's launches by range; without a tool attached the range costs a
+// pointer test).
 #define MOE_LAUNCH(name, stream, ...)                        \
   do {                                                       \
+    nvtxRangePushA(name);                                    \
     cudaEvent_t moe_ev_ = moe::timing_begin(stream);         \
     __VA_ARGS__;                                             \
     moe::timing_end(name, moe_ev_, stream);                  \
+    nvtxRangePop();                                          \
   } while (0)
 
 // -------------------------------------------------------------- device side

@@ -1010,6 +1010,20 @@ int check_common(int E, int d, int F, int64_t rows_cap, const char *fn) {
   return MOE_OK;
 }
 
+// Self-test of the bounded pipeline wait of the tensor-core kernels: one thread
+// initializes an mbarrier that nothing will ever arrive on and waits for its first
+// phase with the same bounded wait; after limit_ns it gives up, records
+// MOE_DEV_WAIT_TIMEOUT and returns, leaving the context usable.
+__global__ void wait_timeout_selftest_kernel(uint64_t limit_ns) {
+  __shared__ uint64_t bar;
+  __shared__ int abort_word;
+  const uint32_t b = tc::smem_u32(&bar);
+  tc::mbar_init(b, 1);
+  tc::fence_mbar_init();
+  abort_word = 0;
+  if (!tc::mbar_wait(b, 0, limit_ns, &abort_word)) dev_flag(&g_dev_err, MOE_DEV_WAIT_TIMEOUT);
+}
+
 }  // namespace
 
 namespace moe {
@@ -1017,6 +1031,16 @@ MOE_DEV_ERR_DEFINE_READER(gemm_dev_error)
 }
 
 extern "C" {
+
+int moe_selftest_wait_timeout(int64_t limit_ns, moe_stream_t stream) {
+  if (limit_ns < 1000000 || limit_ns > 2000000000)
+    return moe::set_error(MOE_ERR_ARG, "moe_selftest_wait_timeout: limit_ns %lld not in [1e6, 2e9]",
+                          (long long)limit_ns);
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  MOE_LAUNCH("selftest_wait_timeout", s,
+             wait_timeout_selftest_kernel<<<1, 1, 0, s>>>(uint64_t(limit_ns)));
+  return moe::launch_status("moe_selftest_wait_timeout");
+}
 
 int moe_grouped_ffn_fwd(const uint16_t *x_perm, const int32_t *group_offsets, int E, int d, int F,
                         int64_t rows_cap, const uint16_t *w_gate_up, const uint16_t *w_down,

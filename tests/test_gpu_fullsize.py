@@ -55,7 +55,8 @@ def _rel(got, ref):
 @pytest.mark.parametrize("cfg_id", [0, 1, 2, 3, 4])
 def test_full_size_sampled_parity(cfg_id):
     L.moe_device_error(clear=True)
-    wl = bench.Workload(cfg_id, "cuda")
+    # the forward-only workloads run their backward too here (extra coverage at full size)
+    wl = bench.Workload(cfg_id, "cuda", backward=True)
     wl.step()
     torch.cuda.synchronize()
     assert L.moe_device_error(clear=True) == 0

@@ -4,6 +4,10 @@ Integer/index results (routing, counts, grouped layout) must be bit-exact
 when both sides route from the same fp32 logits; floating results must meet
 max|gpu - oracle| / max|oracle| <= 2e-2 (bf16 data, fp32 accumulation).
 """
+import os
+import subprocess
+import sys
+
 import numpy as np
 import pytest
 import torch
@@ -384,3 +388,32 @@ def test_gathered_layer_equals_materialized(T, d, E, k, F, n_masked):
     ua = unblock_ab(a.ab.view(torch.int16).cpu().numpy(), F)
     ub = unblock_ab(b.ab.view(torch.int16).cpu().numpy(), F)
     assert (ua[rr] == ub[rr]).all()
+
+
+def test_one_sm_gemm_kernel_against_oracle():
+    """The one-SM GEMM kernel (MOE_GEMM_1SM=1, kept for A/B measurements against the
+    CTA-pair kernel) on layer cases; the variable is read once per process, so the
+    cases run in a child process."""
+    env = dict(os.environ, MOE_GEMM_1SM="1")
+    script = os.path.join(os.path.dirname(os.path.abspath(__file__)), "gpu_one_sm_check.py")
+    r = subprocess.run([sys.executable, script], env=env, capture_output=True, text=True,
+                       timeout=900)
+    assert r.returncode == 0, r.stdout[-2000:] + r.stderr[-4000:]
+
+
+def test_bounded_wait_expires_and_reports():
+    """A pipeline wait that nothing satisfies (an mbarrier no one arrives on) gives up
+    after its limit: the kernel returns, the device error word reads
+    MOE_DEV_WAIT_TIMEOUT (4), and the context keeps running the library's kernels."""
+    import time
+    assert L.moe_device_error(clear=True) == 0
+    t0 = time.perf_counter()
+    L.moe_selftest_wait_timeout(50_000_000)  # 50 ms
+    code = L.moe_device_error(clear=True)    # synchronizes the device
+    dt = time.perf_counter() - t0
+    assert code == 4
+    assert 0.045 <= dt < 5.0
+    z = np.random.default_rng(3).standard_normal((300, 16)).astype(np.float32)
+    idx, g, cnt, _ = _route_only(300, 16, 2, z)
+    oidx, _ = O.route_topk(z, 2)
+    assert (idx == oidx).all() and cnt.sum() == 600

@@ -369,6 +369,8 @@ def kernel_report(wl, per_kernel, steps, peaks):
         "perm_gather": 2 * s.T * s.d + 2 * A * s.d,
         "combine": 2 * A * s.d + 2 * s.T * s.d,
         "combine_bwd": 2 * s.T * s.d + 4 * A * s.d,
+        "combine_bwd_dout": 2 * s.T * s.d + 2 * A * s.d,
+        "combine_bwd_dgate": 2 * s.T * s.d + 2 * A * s.d,
         "permute_bwd": 2 * A * s.d + 2 * s.T * s.d,
         "route_bwd_partial": 2 * A * s.d,
         "route_logits": 2 * s.T * s.d + 4 * s.d * s.E + 4 * s.T * s.E,

@@ -312,6 +312,11 @@ int moe_unpermute_combine(const uint16_t *out_perm, const int32_t *row_of_assign
  *   d_gate[t,j] = <dy[t,:], out_perm[row(t,j),:]>         (fp32)
  * and zeroes the padding rows of d_out_perm (group_offsets/group_counts from
  * moe_permute). dy [T,d] bf16; d_out_perm [rows_cap,d] bf16; d_gate [T,k].
+ * Either output may be NULL (not both, unless T == 0): that half is skipped. A
+ * caller whose router is frozen needs d_out_perm only, which never reads out_perm;
+ * out_perm is read for d_gate only, group_offsets / group_counts are used for
+ * d_out_perm only. (Running the d_gate half on a second stream beside the dH GEMM
+ * measured no faster on GB300 than the fused call: it slows the GEMM by as much.)
  */
 int moe_unpermute_combine_bwd(const uint16_t *dy, const uint16_t *out_perm,
                               const int32_t *row_of_assignment, const float *topk_gate,

@@ -224,6 +224,10 @@ __global__ void __launch_bounds__(kThreads) combine_kernel(
 }
 
 // d_out_perm[row(t,j)] = g[t,j] * dy[t];  d_gate[t,j] = <dy[t], out_perm[row(t,j)]>
+// DOUT: d_out_perm rows = g * dy[t]; DGATE: d_gate = <dy[t], out_perm rows>. The two
+// halves can run as separate launches (DGATE alone reads out_perm and writes nothing
+// large; DOUT alone never reads out_perm).
+template <bool DOUT, bool DGATE>
 __global__ void __launch_bounds__(kThreads) combine_bwd_kernel(
     const uint16_t *__restrict__ dy, const uint16_t *__restrict__ out_perm,
     const int32_t *__restrict__ row_of_assignment, const float *__restrict__ gate, int T, int d,
@@ -248,26 +252,32 @@ __global__ void __launch_bounds__(kThreads) combine_bwd_kernel(
     float fd[8];
     unpack8(ldg_nc_v4(dy + size_t(t) * d + c * 8), fd);
     uint4 v[8];
+    if (DGATE) {
 #pragma unroll
-    for (int j = 0; j < 8; ++j)
-      if (j < k && rows[j] >= 0) v[j] = ldg_nc_v4(out_perm + size_t(rows[j]) * d + c * 8);
+      for (int j = 0; j < 8; ++j)
+        if (j < k && rows[j] >= 0) v[j] = ldg_nc_v4(out_perm + size_t(rows[j]) * d + c * 8);
+    }
 #pragma unroll
     for (int j = 0; j < 8; ++j) {
       if (j < k && rows[j] >= 0) {
-        float f[8], o[8];
-        unpack8(v[j], f);
+        if (DGATE) {
+          float f[8];
+          unpack8(v[j], f);
 #pragma unroll
-        for (int q = 0; q < 8; ++q) {
-          dot[j] = fmaf(fd[q], f[q], dot[j]);
-          o[q] = g[j] * fd[q];
+          for (int q = 0; q < 8; ++q) dot[j] = fmaf(fd[q], f[q], dot[j]);
         }
-        stg_v4(d_out_perm + size_t(rows[j]) * d + c * 8, pack8(o));
+        if (DOUT) {
+          float o[8];
+#pragma unroll
+          for (int q = 0; q < 8; ++q) o[q] = g[j] * fd[q];
+          stg_v4(d_out_perm + size_t(rows[j]) * d + c * 8, pack8(o));
+        }
       }
     }
   }
 #pragma unroll
   for (int j = 0; j < 8; ++j) {
-    if (j < k) {
+    if (DGATE && j < k) {
       float s = dot[j];
 #pragma unroll
       for (int off = 16; off > 0; off >>= 1) s += __shfl_xor_sync(0xffffffffu, s, off);
@@ -449,17 +459,33 @@ int moe_unpermute_combine_bwd(const uint16_t *dy, const uint16_t *out_perm,
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   if (E < 1 || E > 256 || k < 1 || k > 8 || T < 0 || d <= 0 || d % 8)
     return moe::set_error(MOE_ERR_ARG, "moe_unpermute_combine_bwd: sizes");
-  if (!group_offsets || !group_counts || !d_out_perm ||
-      (T > 0 && (!dy || !out_perm || !row_of_assignment || !topk_gate || !d_gate)))
+  if (!d_out_perm && !d_gate && T > 0)  // (with no tokens d_gate is empty and may be NULL)
+    return moe::set_error(MOE_ERR_ARG, "moe_unpermute_combine_bwd: no output requested");
+  if ((d_out_perm && (!group_offsets || !group_counts)) ||
+      (T > 0 && (!dy || !row_of_assignment || !topk_gate || (d_gate && !out_perm))))
     return moe::set_error(MOE_ERR_ARG, "moe_unpermute_combine_bwd: null pointer");
-  if (!moe::aligned16(d_out_perm) || (dy && !moe::aligned16(dy)) || (out_perm && !moe::aligned16(out_perm)))
+  if ((d_out_perm && !moe::aligned16(d_out_perm)) || (dy && !moe::aligned16(dy)) ||
+      (out_perm && !moe::aligned16(out_perm)))
     return moe::set_error(MOE_ERR_ARG, "moe_unpermute_combine_bwd: alignment");
   const int64_t rows_cap = moe_perm_rows_max(T, k, E);
   if (T > 0) {
-    MOE_LAUNCH("combine_bwd", s, combine_bwd_kernel<<<warp_grid(T), kThreads, 0, s>>>(dy, out_perm, row_of_assignment, topk_gate,
-                                                         T, d, k, rows_cap, d_out_perm, d_gate));
+    const int grid = warp_grid(T);
+    if (d_out_perm && d_gate) {
+      MOE_LAUNCH("combine_bwd", s, (combine_bwd_kernel<true, true><<<grid, kThreads, 0, s>>>(
+                                       dy, out_perm, row_of_assignment, topk_gate, T, d, k,
+                                       rows_cap, d_out_perm, d_gate)));
+    } else if (d_out_perm) {
+      MOE_LAUNCH("combine_bwd_dout", s, (combine_bwd_kernel<true, false><<<grid, kThreads, 0, s>>>(
+                                            dy, out_perm, row_of_assignment, topk_gate, T, d, k,
+                                            rows_cap, d_out_perm, d_gate)));
+    } else {
+      MOE_LAUNCH("combine_bwd_dgate", s, (combine_bwd_kernel<false, true><<<grid, kThreads, 0, s>>>(
+                                             dy, out_perm, row_of_assignment, topk_gate, T, d, k,
+                                             rows_cap, d_out_perm, d_gate)));
+    }
     if (int st = moe::launch_status("moe_unpermute_combine_bwd: launch")) return st;
   }
+  if (!d_out_perm) return MOE_OK;
   MOE_LAUNCH("pad_zero", s, pad_zero_kernel<<<dim3(E, kPadSplit), kThreads, 0, s>>>(group_offsets, group_counts, E, d, rows_cap, d_out_perm));
   return moe::launch_status("moe_unpermute_combine_bwd: pad");
 }

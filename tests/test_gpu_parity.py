@@ -417,3 +417,29 @@ def test_bounded_wait_expires_and_reports():
     idx, g, cnt, _ = _route_only(300, 16, 2, z)
     oidx, _ = O.route_topk(z, 2)
     assert (idx == oidx).all() and cnt.sum() == 600
+
+
+def test_combine_bwd_halves_equal_fused():
+    """moe_unpermute_combine_bwd with one output NULL computes that half alone: the
+    d_out_perm half and the d_gate half equal the fused call bit for bit."""
+    T, d, E, k = 1000, 512, 16, 4
+    dev = "cuda"
+    inp = case_inputs(T, d, E, k, 128, seed=21)
+    b = layer.MoELayerBuffers(layer.LayerShape(T, d, E, k, 128), dev, backward=True)
+    g = {n: v.to(dev) for n, v in inp.items()}
+    layer.forward(b, g["x"], g["w_router"], g["bias"], g["w_gate_up"], g["w_down"])
+    args = (g["dy"], b.out_perm, b.row_of_assignment, b.topk_gate, b.group_offsets,
+            b.group_counts, T, d, E, k)
+    dop_f = torch.full_like(b.d_out_perm, float("nan"))
+    dg_f = torch.full_like(b.d_gate, float("nan"))
+    L.moe_unpermute_combine_bwd(*args, dop_f, dg_f)
+    dop_h = torch.full_like(b.d_out_perm, float("nan"))
+    dg_h = torch.full_like(b.d_gate, float("nan"))
+    L.moe_unpermute_combine_bwd(*args, dop_h, None)
+    L.moe_unpermute_combine_bwd(*args, None, dg_h)
+    torch.cuda.synchronize()
+    used = int(b.group_offsets[E].item())
+    assert torch.equal(dop_f[:used], dop_h[:used])
+    assert torch.equal(dg_f, dg_h)
+    with pytest.raises(L.MoEError):
+        L.moe_unpermute_combine_bwd(*args, None, None)

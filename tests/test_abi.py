@@ -128,3 +128,41 @@ def test_laep_algorithms_match_oracle_random(lib):
         order, group_of, gl = L.laep_rearrange(loads, ng)
         oo, og, ogl = O.rearrange(loads, ng)
         assert (order == oo).all() and (group_of == og).all() and (gl == ogl).all()
+
+
+def test_new_entry_points_validate_before_launch(lib):
+    """Fused-dispatch entry points, the combine-backward halves and the wait self-test
+    reject bad arguments on the host (no device work is queued)."""
+    R = L.moe_perm_rows_max(100, 2, 8)
+    with pytest.raises(L.MoEError) as e:  # no token_of_row
+        L.moe_permute_map(16, None, 100, 8, 2, R, 16, 16, 16, None, 16, 1 << 20, stream=0)
+    assert e.value.status == -1
+    with pytest.raises(L.MoEError) as e:  # rows_cap below T*k + 128*E
+        L.moe_permute_map(16, None, 100, 8, 2, 100, 16, 16, 16, 16, 16, 1 << 20, stream=0)
+    assert e.value.status == -1
+    with pytest.raises(L.MoEError) as e:  # workspace too small for the block histograms
+        L.moe_permute_map(16, None, 100, 8, 2, R, 16, 16, 16, 16, 16, 4, stream=0)
+    assert e.value.status == -6
+    with pytest.raises(L.MoEError) as e:  # d not a multiple of 128
+        L.moe_grouped_ffn_fwd_gather(16, 16, 10, 16, 8, 100, 256, R, 16, 16, 16, 16, 16, 16, 0,
+                                     stream=0)
+    assert e.value.status == -2
+    with pytest.raises(L.MoEError) as e:  # x missing with tokens present
+        L.moe_grouped_ffn_fwd_gather(None, 16, 10, 16, 8, 128, 256, R, 16, 16, 16, 16, 16, 16, 0,
+                                     stream=0)
+    assert e.value.status == -1
+    with pytest.raises(L.MoEError) as e:  # unaligned token_of_row
+        L.moe_grouped_ffn_bwd_wgrad_gather(16, 16, 20, 10, 16, 16, 16, 8, 128, 256, R, 16, 16,
+                                           stream=0)
+    assert e.value.status == -1
+    with pytest.raises(L.MoEError) as e:  # router backward through the map needs the map
+        L.moe_route_bwd_gather(16, None, 16, 16, 16, 16, 16, 10, 128, 8, 2, R, 16, 16, 16,
+                               1 << 20, stream=0)
+    assert e.value.status == -1
+    with pytest.raises(L.MoEError) as e:  # combine backward with neither output
+        L.moe_unpermute_combine_bwd(16, 16, 16, 16, 16, 16, 10, 128, 8, 2, None, None, stream=0)
+    assert e.value.status == -1
+    for bad in (0, 999_999, 2_000_000_001):
+        with pytest.raises(L.MoEError) as e:
+            L.moe_selftest_wait_timeout(bad, stream=0)
+        assert e.value.status == -1

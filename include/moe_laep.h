@@ -208,10 +208,10 @@ int moe_permute(const uint16_t *x, const int32_t *topk_idx, const int32_t *count
 /*
  * moe_permute_noalloc - moe_permute for callers that cannot allocate device
  * memory. The paper has no counterpart; this is a deployment variant.
- * Some callers may not call cudaMalloc or hand out a workspace, e.g. code
- * running inside an engine whose device memory is planned before it runs
- * (an inference plugin's enqueue) or while a stream is being captured into a
- * CUDA graph. This entry point computes exactly what moe_permute computes
+ * Some callers may not call cudaMalloc or hand out a workspace: code that
+ * runs inside an inference engine's plugin, for example, where the engine
+ * planned and owns all device memory before execution and passes the plugin
+ * only its input and output buffers. This entry point computes exactly what moe_permute computes
  * (same arguments minus ws/ws_bytes, same results) but keeps its per-block
  * histograms in a fixed 256 KiB array compiled into the library (65536
  * int32 entries) instead of a workspace; it allocates nothing.

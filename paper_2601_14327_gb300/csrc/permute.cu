@@ -522,9 +522,9 @@ int moe_permute_bwd(const uint16_t *dx_perm, const int32_t *row_of_assignment,
 
 // ---------------------------------------------------------------------------
 // moe_permute_noalloc: moe_permute for callers that cannot allocate device
-// memory (no cudaMalloc and no caller workspace), e.g. code running inside an
-// engine whose device memory is planned before execution (an inference
-// plugin's enqueue, a stream being captured into a CUDA graph). The
+// memory (no cudaMalloc and no caller workspace), e.g. an inference engine's
+// plugin, whose device memory the engine planned and owns before execution
+// and which receives only its input and output buffers. The
 // per-block histograms live in a fixed array compiled into the library
 // instead of the caller's workspace.
 //

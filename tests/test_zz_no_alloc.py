@@ -1,7 +1,7 @@
 """moe_permute_noalloc: the permutation for callers that cannot allocate.
 
-Some callers may not call cudaMalloc or pass a workspace (an engine that plans
-its device memory before running, a stream under CUDA-graph capture). For
+Some callers may not call cudaMalloc or pass a workspace (a plugin inside an
+inference engine that planned and owns all device memory before running). For
 them the library offers one entry point that keeps its scratch in a fixed
 array compiled into the library. This test checks, through the C ABI, that
 it returns exactly what the workspace-based moe_permute returns, on two

@@ -46,21 +46,22 @@ GEMMS = ["gemm_gate_up", "gemm_down", "gemm_dgrad_down", "gemm_dgrad_gate_up",
 
 
 def committed_traffic(kernel):
-    """DRAM bytes per launch of `kernel` from the committed ncu capture, or None when
-    the kernel sources changed since the counters were taken (or no capture exists)."""
+    """DRAM bytes per launch of `kernel` from the committed ncu capture, or None when the
+    sources that kernel is built from changed since the counters were taken (or no capture
+    exists)."""
     import hashlib
     path = os.path.join(ROOT, "profiles", "dram_traffic_laep_pruned_fwdbwd_T16384.json")
     if not os.path.exists(path):
         return None
     with open(path) as f:
-        rec = json.load(f)
+        rec = json.load(f).get("kernels", {}).get(kernel)
+    if rec is None:
+        return None
     h = hashlib.sha256()
     for src in rec["sources"]:
         with open(os.path.join(ROOT, src), "rb") as f:
             h.update(f.read())
-    if h.hexdigest() != rec["sources_sha256"]:
-        return None
-    return rec["dram_bytes_per_launch"].get(kernel)
+    return rec["bytes_per_launch"] if h.hexdigest() == rec["sources_sha256"] else None
 
 
 def measured_peaks():

@@ -157,11 +157,20 @@ __global__ void __launch_bounds__(kThreads) perm_gather_kernel(
   for (int j = 0; j < 8; ++j) rows[j] = __shfl_sync(0xffffffffu, my_row, j);
   const int nv = d / 8;
   const uint16_t *src = x + size_t(t) * d;
-  for (int c = lane; c < nv; c += 32) {
-    const uint4 v = ldg_nc_v4(src + c * 8);
+  // four 16-byte loads in flight per lane before their stores
+  for (int c0 = lane; c0 < nv; c0 += 128) {
+    uint4 v[4];
 #pragma unroll
-    for (int j = 0; j < 8; ++j)
-      if (j < k && rows[j] >= 0 && rows[j] < rows_cap) stg_v4(x_perm + size_t(rows[j]) * d + c * 8, v);
+    for (int u = 0; u < 4; ++u)
+      if (c0 + 32 * u < nv) v[u] = ldg_nc_v4(src + (c0 + 32 * u) * 8);
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int c = c0 + 32 * u;
+      if (c >= nv) break;
+#pragma unroll
+      for (int j = 0; j < 8; ++j)
+        if (j < k && rows[j] >= 0 && rows[j] < rows_cap) stg_v4(x_perm + size_t(rows[j]) * d + c * 8, v[u]);
+    }
   }
 }
 

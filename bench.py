@@ -401,7 +401,8 @@ PARAMS_NOTE = ("paper context (Table 5, 824 AI chips, BF16, expert parallelism):
 def laep_comparison(args, world, local, pruned_tps, wl_pruned):
     """Same workload without pruning (all experts live), timed the same way."""
     steps = max(3, min(args.steps, 10))
-    pruned_params = 3 * wl_pruned.shape.E * wl_pruned.shape.d * wl_pruned.shape.F
+    # live experts: the compacted count, or the unmasked ones when pruning is a mask
+    pruned_params = 3 * wl_pruned.E_live * wl_pruned.shape.d * wl_pruned.shape.F
     c = wl_pruned.cfg
     # free the pruned workload's activations while the unpruned one runs
     saved = wl_pruned.bufs
@@ -421,7 +422,10 @@ def laep_comparison(args, world, local, pruned_tps, wl_pruned):
     del wl_u
     torch.cuda.empty_cache()
     wl_pruned.bufs = saved
-    return {"experts_unpruned": c.E, "experts_pruned": wl_pruned.shape.E,
+    return {"experts_unpruned": c.E, "experts_pruned": wl_pruned.E_live,
+            "pruning": ("compacted (pruned experts' weights removed)" if wl_pruned.mask is None
+                        else "mask (pruned experts get no token; their weight gradients are "
+                             "still written, as zeros)"),
             "unpruned_tokens_per_s": round(tps_u, 1), "pruned_tokens_per_s": round(pruned_tps, 1),
             "speedup": round(pruned_tps / tps_u, 4),
             "expert_params_unpruned": unpruned_params, "expert_params_pruned": pruned_params,
@@ -474,7 +478,7 @@ def run_ours(args):
     gb = group_bound_seconds(wl.shape, wl.bufs.counts.cpu().tolist(), peaks)
     gemm_bound_frac = sum(gb[n] for n in gemm_ms) / (all_gemm_ms / 1e3)
     laep = None
-    if (wl.cfg.compact and args.tokens is None and args.experts is None and not args.no_prune
+    if (wl.cfg.prune_lowest and args.tokens is None and args.experts is None and not args.no_prune
             and args.bias is None):
         laep = laep_comparison(args, world, local, tokens_per_s, wl)
 

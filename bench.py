@@ -477,14 +477,11 @@ def run_ours(args):
     kernel_table = kernel_report(wl, per_kernel, args.steps, peaks)
     gb = group_bound_seconds(wl.shape, wl.bufs.counts.cpu().tolist(), peaks)
     gemm_bound_frac = sum(gb[n] for n in gemm_ms) / (all_gemm_ms / 1e3)
-    laep = None
-    if (wl.cfg.prune_lowest and args.tokens is None and args.experts is None and not args.no_prune
-            and args.bias is None):
-        laep = laep_comparison(args, world, local, tokens_per_s, wl)
 
     # end to end through the public API: every step uploads its inputs from pinned host
     # memory and downloads its results (x, dy in; y, dx out; forward-only workloads: x in,
-    # y out). A copy stream and two device slots pipeline the copies with the compute:
+    # y out). An upload stream, a download stream and two device slots pipeline the copies
+    # with the compute:
     # step i+2's inputs and step i's results move while step i+1 computes; the first
     # uploads and the last downloads are inside the timed region.
     e2e = None
@@ -513,16 +510,17 @@ def run_ours(args):
             use_slot(j)
             wl.eager_step(*inputs(j))
             graphs.append(wl.make_graph(*inputs(j)) if args.graph else None)
-        copy = torch.cuda.Stream()
+        # uploads and downloads on separate streams: the two directions overlap
+        up, down = torch.cuda.Stream(), torch.cuda.Stream()
         in_ready = [torch.cuda.Event() for _ in range(2)]
         step_done = [torch.cuda.Event() for _ in range(2)]
         out_copied = [torch.cuda.Event() for _ in range(2)]
 
         def upload(j):
-            with torch.cuda.stream(copy):
+            with torch.cuda.stream(up):
                 for n in in_names:
                     dev_in[j][n].copy_(host_in[n], non_blocking=True)
-                in_ready[j].record(copy)
+                in_ready[j].record(up)
 
         def run(i):
             j = i % 2
@@ -535,19 +533,21 @@ def run_ours(args):
                 use_slot(j)
                 wl.eager_step(*inputs(j))
             step_done[j].record(stream)
-            with torch.cuda.stream(copy):
-                copy.wait_event(step_done[j])
+            with torch.cuda.stream(down):
+                down.wait_event(step_done[j])
                 for n in out_names:
                     host_out[j][n].copy_(dev_out[j][n], non_blocking=True)
-                out_copied[j].record(copy)
+                out_copied[j].record(down)
             if i + 2 < args.steps:
-                upload(j)  # ordered after step i's downloads on the copy stream
+                up.wait_event(step_done[j])  # step i no longer reads slot j's inputs
+                upload(j)
 
         ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         barrier(world)
         torch.cuda.synchronize()
         ev0.record(stream)
-        copy.wait_event(ev0)
+        up.wait_event(ev0)
+        down.wait_event(ev0)
         upload(0)
         if args.steps > 1:
             upload(1)
@@ -566,8 +566,14 @@ def run_ours(args):
                "h2d_bytes_per_step": nb(host_in.values()),
                "d2h_bytes_per_step": nb(host_out[0].values()),
                "note": f"{', '.join(in_names)} uploaded and {', '.join(out_names)} downloaded "
-                       "every step on a copy stream, overlapped with the neighbouring steps' "
-                       "compute"}
+                       "every step (an upload and a download stream), overlapped with the "
+                       "neighbouring steps' compute"}
+
+    # pruned vs unpruned, after the end-to-end run (it allocates a second workload)
+    laep = None
+    if (wl.cfg.prune_lowest and args.tokens is None and args.experts is None and not args.no_prune
+            and args.bias is None):
+        laep = laep_comparison(args, world, local, tokens_per_s, wl)
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:

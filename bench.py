@@ -572,7 +572,7 @@ def run_ours(args):
     # pruned vs unpruned, after the end-to-end run (it allocates a second workload)
     laep = None
     if (wl.cfg.prune_lowest and args.tokens is None and args.experts is None and not args.no_prune
-            and args.bias is None):
+            and args.bias is None and not args.no_laep):
         laep = laep_comparison(args, world, local, tokens_per_s, wl)
 
     cpu = None
@@ -686,6 +686,8 @@ def main():
     ap.add_argument("--ref-tokens", type=int, default=64)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-laep", action="store_true",
+                    help="skip the pruned-vs-unpruned comparison (e.g. for profiler captures)")
     ap.add_argument("--gather", type=int, default=0,
                     help="dispatch through a materialized X_perm (0), or by 4-row TMA gathers "
                          "from x with X_perm never written (1; same results, slower GEMMs)")

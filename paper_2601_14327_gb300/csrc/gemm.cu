@@ -478,7 +478,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
     }
   } else {
-    // ===================== epilogue (warps 2..5) =====================
+    // ===================== epilogue (warps 2..9) =====================
     const int q = warp & 3;  // TMEM lane quarter this warp may access
     const int half = (warp - 2) / 4;  // column half this warp handles
     const uint32_t stage = stage_base + uint32_t(warp - 2) * kStageBytes;
@@ -836,7 +836,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
     }
   } else {
-    // ============ epilogue (warps 2..5 of each CTA) ============
+    // ============ epilogue (warps 2..9 of each CTA) ============
     const int q = warp & 3;
     const int half = (warp - 2) / 4;
     const uint32_t stage = stage_base + uint32_t(warp - 2) * kStageBytes;

@@ -184,6 +184,8 @@ LAYER_CASES = [
     (1500, 384, 12, 4, 640, "zipf", 3),       # ragged groups, BN=128 paths, empty groups
     (700, 512, 8, 8, 256, "zipf", 0),         # k = number of experts
     (2100, 256, 32, 2, 384, "loguniform", 0), # volatile load, several empty experts
+    (3000, 256, 256, 8, 256, "zipf", 40),     # the maximum expert count (schedule arrays full),
+                                              # many light and empty experts
 ]
 
 

@@ -445,3 +445,25 @@ def test_combine_bwd_halves_equal_fused():
     assert torch.equal(dg_f, dg_h)
     with pytest.raises(L.MoEError):
         L.moe_unpermute_combine_bwd(*args, None, None)
+
+
+def test_layer_is_deterministic_and_stream_layout_independent():
+    """Every reduction runs in a fixed order (split partials, router partial sums, combine
+    sums) and the only atomics are integer counts, so a step gives the same bits every
+    time, and the two-stream backward gives the same bits as the one-stream one."""
+    T, d, E, k, F = 2000, 256, 16, 4, 256
+    dev = "cuda"
+    inp = case_inputs(T, d, E, k, F, seed=77)
+    g = {n: v.to(dev) for n, v in inp.items()}
+    outs = []
+    for overlap in (True, True, False):
+        b = layer.MoELayerBuffers(layer.LayerShape(T, d, E, k, F), dev, backward=True)
+        layer.forward(b, g["x"], g["w_router"], g["bias"], g["w_gate_up"], g["w_down"])
+        layer.backward(b, g["dy"], g["w_router"], g["w_gate_up"], g["w_down"], overlap=overlap)
+        torch.cuda.synchronize()
+        outs.append(b)
+    names = ["topk_idx", "topk_gate", "counts", "row_of_assignment", "y", "dx", "dw_gate_up",
+             "dw_down", "dw_router", "d_logits"]
+    for other in outs[1:]:
+        for n in names:
+            assert torch.equal(getattr(outs[0], n), getattr(other, n)), n

@@ -64,6 +64,9 @@ def committed_traffic(kernel):
     return rec["bytes_per_launch"] if h.hexdigest() == rec["sources_sha256"] else None
 
 
+HBM_NOMINAL_GBS = 8000.0  # GB300 HBM3e, nominal (~8 TB/s); the measured copy peak is below it
+
+
 def measured_peaks():
     path = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(path):
@@ -387,7 +390,8 @@ def kernel_report(wl, per_kernel, steps, peaks):
                      group_bound_frac=round(bound[n] / per_launch_s, 4))
         elif n in hbm:
             gbs = hbm[n] / per_launch_s / 1e9
-            e.update(gbs=round(gbs, 1), frac=round(gbs / peaks["hbm_gbs"], 4))
+            e.update(gbs=round(gbs, 1), frac=round(gbs / peaks["hbm_gbs"], 4),
+                     frac_nominal=round(gbs / HBM_NOMINAL_GBS, 4))
         out[n] = e
     return out
 

@@ -271,16 +271,31 @@ def moe_backward(dy, x, topk_idx, gates, w_router, w_gate_up, w_down, fwd):
         dw_gate_up[e, :F] = dae.T @ xe
         dw_gate_up[e, F:] = dbe.T @ xe
 
-    dz = g * (d_gate - np.sum(g * d_gate, axis=1, keepdims=True))
-    dw_router = np.zeros((d, E))
-    for e in range(E):
-        t, j = _assignments_of(topk_idx, e)
-        if t.size:
-            dw_router[:, e] = x[t].T @ dz[t, j]
+    dz, dw_router = router_backward(x, topk_idx, g, d_gate, E)
     dx = dX.sum(axis=1) + np.einsum("tj,dtj->td", dz, wr[:, topk_idx])
     return {"d_o": d_o, "d_gate": d_gate, "dA": dA, "dB": dB, "dX": dX,
             "dw_gate_up": dw_gate_up, "dw_down": dw_down, "d_logits": dz,
             "dw_router": dw_router, "dx": dx}
+
+
+def router_backward(x, topk_idx, gates, d_gate, E):
+    """Router part of the backward, fp64: the softmax over the selected k
+    (reading R3) and the linear router's weight gradient.
+
+    dz[t,j] = g_j (d_gate_j - sum_i g_i d_gate_i)
+    dW_r[:, e] = sum over assignments (t,j) to e of dz[t,j] x[t]  (zero if none)
+    Returns (dz [T,k], dW_r [d,E]).
+    """
+    x = np.asarray(x, np.float64)
+    g = np.asarray(gates, np.float64)
+    d_gate = np.asarray(d_gate, np.float64)
+    dz = g * (d_gate - np.sum(g * d_gate, axis=1, keepdims=True))
+    dw_router = np.zeros((x.shape[1], E))
+    for e in range(E):
+        t, j = _assignments_of(topk_idx, e)
+        if t.size:
+            dw_router[:, e] = x[t].T @ dz[t, j]
+    return dz, dw_router
 
 
 def moe_layer(x, w_router, bias, active_mask, k, w_gate_up, w_down, dy=None,

@@ -376,7 +376,7 @@ def kernel_report(wl, per_kernel, steps, peaks):
         "combine_bwd_dout": 2 * s.T * s.d + 2 * A * s.d,
         "combine_bwd_dgate": 2 * s.T * s.d + 2 * A * s.d,
         "permute_bwd": 2 * A * s.d + 2 * s.T * s.d,
-        "route_bwd_partial": 2 * A * s.d,
+        "route_bwd_dw": 2 * s.T * s.d + 4 * s.d * s.E,
         "route_logits": 2 * s.T * s.d + 4 * s.d * s.E + 4 * s.T * s.E,
     }
     tot = sum(v[1] for v in per_kernel.values())

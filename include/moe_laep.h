@@ -254,15 +254,15 @@ int moe_grouped_ffn_fwd(const uint16_t *x_perm, const int32_t *group_offsets, in
 
 /*
  * Gathered form of the dispatch (no X_perm in memory). The grouped operand X_perm
- * of the forward GEMM and of the dW_gate_up GEMM, and the rows the router
- * backward reads, are taken from x itself through a row -> token map: grouped
+ * of the forward GEMM and of the dW_gate_up GEMM is taken from x itself through a
+ * row -> token map: grouped
  * row r is x[token_of_row[r], :]. The GEMMs load those rows with 4-row TMA
  * gathers (one token row of d_model per gathered row, 128 bytes at a time), so
  * the (T*k + padding) x d copy that moe_permute writes is never materialized.
  * Results are the same as with moe_permute's X_perm, bit for bit, on every real
  * row and in every gradient: a padding row reads token 0 instead of zeros, and
  * every consumer multiplies padding rows by zero (d_out_perm's padding rows are
- * zero, and the router backward reads real rows only); on padding rows the
+ * zero); on padding rows the
  * forward's ab_saved, h and out_perm hold finite values instead of zeros.
  * Cost on GB300: the two GEMMs that read X_perm run ~3.3x longer with 4-row
  * gathers than with tile loads of a materialized X_perm, far more than the
@@ -371,29 +371,22 @@ int moe_grouped_ffn_bwd_wgrad_gather(const uint16_t *d_out_perm, const uint16_t 
                                      uint16_t *dw_down, moe_stream_t stream);
 
 /*
- * moe_route_bwd - backward of the router's softmax over the selected experts:
+ * moe_route_bwd - backward of the router's softmax over the selected experts
+ * (the routing scores of Sec. 3.2 as a trainable linear router):
  *   d_logits[t,j] = g[t,j] * (d_gate[t,j] - sum_i g[t,i] * d_gate[t,i])
  *   dw_router[:, e] = sum over assignments (t,j) to e of d_logits[t,j] * x[t,:]
- * (the bias is fixed, unselected and pruned experts get zero). x_perm is the
- * grouped copy of x from moe_permute. d_logits [T,k] fp32 (out);
- * dw_router [d,E] fp32 (out, overwritten).
+ * (the bias is fixed; unselected and pruned experts get zero). x [T,d] bf16 is the
+ * layer input (16-byte aligned); topk_idx, topk_gate [T,k] as moe_route wrote them;
+ * d_gate [T,k] fp32 (from moe_unpermute_combine_bwd). d_logits [T,k] fp32 (out);
+ * dw_router [d,E] fp32 (out, overwritten; zero when T == 0).
+ * dw_router is the product x^T dZ on the tensor cores, dZ [T,E] split into three
+ * bf16 terms (bf16 x bf16 products are exact in fp32), accumulated in fp32 in a
+ * fixed order: bitwise reproducible from run to run. ws/ws_bytes: workspace of
+ * moe_workspace_size(T, d, E, k, F) bytes, 16-byte aligned.
  */
-int moe_route_bwd(const uint16_t *x_perm, const int32_t *topk_idx, const float *topk_gate,
-                  const float *d_gate, const int32_t *row_of_assignment,
-                  const int32_t *group_offsets, const int32_t *group_counts, int T, int d,
-                  int E, int k, int64_t rows_cap, float *d_logits, float *dw_router, void *ws,
-                  size_t ws_bytes, moe_stream_t stream);
-
-/*
- * moe_route_bwd_gather - moe_route_bwd with the rows of x read through
- * token_of_row (moe_permute_map) instead of from x_perm. Arguments as in
- * moe_route_bwd, with x [T,d] bf16 in place of x_perm.
- */
-int moe_route_bwd_gather(const uint16_t *x, const int32_t *token_of_row, const float *topk_gate,
-                         const float *d_gate, const int32_t *row_of_assignment,
-                         const int32_t *group_offsets, const int32_t *group_counts, int T, int d,
-                         int E, int k, int64_t rows_cap, float *d_logits, float *dw_router,
-                         void *ws, size_t ws_bytes, moe_stream_t stream);
+int moe_route_bwd(const uint16_t *x, const int32_t *topk_idx, const float *topk_gate,
+                  const float *d_gate, int T, int d, int E, int k, float *d_logits,
+                  float *dw_router, void *ws, size_t ws_bytes, moe_stream_t stream);
 
 /*
  * moe_permute_bwd - gradient of the layer input:

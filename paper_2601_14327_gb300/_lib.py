@@ -57,12 +57,11 @@ _SIGS = {
     "moe_grouped_ffn_bwd": (I, [P, P, P, P, P, I, I, I, I64, P, P, P, P, P, P, P, SZ, P]),
     "moe_grouped_ffn_bwd_dgrad": (I, [P, P, P, I, I, I, I64, P, P, P, P, P]),
     "moe_grouped_ffn_bwd_wgrad": (I, [P, P, P, P, P, I, I, I, I64, P, P, P]),
-    "moe_route_bwd": (I, [P, P, P, P, P, P, P, I, I, I, I, I64, P, P, P, SZ, P]),
+    "moe_route_bwd": (I, [P, P, P, P, I, I, I, I, P, P, P, SZ, P]),
     "moe_permute_bwd": (I, [P, P, P, P, P, I, I, I, I, P, P, SZ, P]),
     "moe_permute_map": (I, [P, P, I, I, I, I64, P, P, P, P, P, SZ, P]),
     "moe_grouped_ffn_fwd_gather": (I, [P, P, I, P, I, I, I, I64, P, P, P, P, P, P, SZ, P]),
     "moe_grouped_ffn_bwd_wgrad_gather": (I, [P, P, P, I, P, P, P, I, I, I, I64, P, P, P]),
-    "moe_route_bwd_gather": (I, [P, P, P, P, P, P, P, I, I, I, I, I64, P, P, P, SZ, P]),
     "moe_selftest_wait_timeout": (I, [I64, P]),
 }
 
@@ -265,12 +264,10 @@ def moe_grouped_ffn_bwd_wgrad(d_out_perm, x_perm, h, d_ab, group_offsets, E, d, 
         rows_cap, _ptr(dw_gate_up), _ptr(dw_down), _stream(stream)))
 
 
-def moe_route_bwd(x_perm, topk_idx, topk_gate, d_gate, row_of_assignment, group_offsets,
-                  group_counts, T, d, E, k, rows_cap, d_logits, dw_router, ws, ws_bytes,
+def moe_route_bwd(x, topk_idx, topk_gate, d_gate, T, d, E, k, d_logits, dw_router, ws, ws_bytes,
                   stream=None):
     _check("moe_route_bwd", load().moe_route_bwd(
-        _ptr(x_perm), _ptr(topk_idx), _ptr(topk_gate), _ptr(d_gate), _ptr(row_of_assignment),
-        _ptr(group_offsets), _ptr(group_counts), T, d, E, k, rows_cap, _ptr(d_logits),
+        _ptr(x), _ptr(topk_idx), _ptr(topk_gate), _ptr(d_gate), T, d, E, k, _ptr(d_logits),
         _ptr(dw_router), _ptr(ws), ws_bytes, _stream(stream)))
 
 
@@ -294,15 +291,6 @@ def moe_grouped_ffn_bwd_wgrad_gather(d_out_perm, x, token_of_row, T, h, d_ab, gr
     _check("moe_grouped_ffn_bwd_wgrad_gather", load().moe_grouped_ffn_bwd_wgrad_gather(
         _ptr(d_out_perm), _ptr(x), _ptr(token_of_row), T, _ptr(h), _ptr(d_ab),
         _ptr(group_offsets), E, d, F, rows_cap, _ptr(dw_gate_up), _ptr(dw_down), _stream(stream)))
-
-
-def moe_route_bwd_gather(x, token_of_row, topk_gate, d_gate, row_of_assignment, group_offsets,
-                         group_counts, T, d, E, k, rows_cap, d_logits, dw_router, ws, ws_bytes,
-                         stream=None):
-    _check("moe_route_bwd_gather", load().moe_route_bwd_gather(
-        _ptr(x), _ptr(token_of_row), _ptr(topk_gate), _ptr(d_gate), _ptr(row_of_assignment),
-        _ptr(group_offsets), _ptr(group_counts), T, d, E, k, rows_cap, _ptr(d_logits),
-        _ptr(dw_router), _ptr(ws), ws_bytes, _stream(stream)))
 
 
 def moe_permute_bwd(dx_perm, row_of_assignment, topk_idx, d_logits, w_router, T, d, E, k, dx,

@@ -103,14 +103,13 @@ WsLayout ws_layout(int T, int d, int E, int k, int F) {
   WsLayout w{};
   const int64_t A = int64_t(T) * k;
   const int64_t nblk = std::max<int64_t>(1, (A + kPermChunk - 1) / kPermChunk);
-  const int64_t rows = moe_perm_rows_max(T, k, E);
   size_t off = 0;
   w.perm_hist = off;
   off += align256(size_t(E) * nblk * 4);
-  w.dz_perm = off;
-  off += align256(size_t(rows) * 4);
-  w.rb_partial = off;
-  off += align256(size_t(rows / kGroupPad) * d * 4);
+  w.route_dz3 = off;
+  off += align256(route_dz3_bytes(T, E));
+  w.route_dw_partial = off;
+  off += align256(route_dw_partial_bytes(T, d, E));
   w.w_router_t = off;
   off += align256(size_t(E) * d * 4);
   w.route_partial = off;

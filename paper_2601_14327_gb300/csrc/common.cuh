@@ -29,8 +29,8 @@ int num_sms();
 // Workspace layout shared by the entry points (disjoint regions, 256-byte aligned).
 struct WsLayout {
   size_t perm_hist;     // int32 [E * nblk]        moe_permute block histograms
-  size_t dz_perm;       // fp32  [rows_cap]        moe_route_bwd per-row d_logits
-  size_t rb_partial;    // fp32  [rows_cap/128, d] moe_route_bwd per-tile partial sums
+  size_t route_dz3;     // bf16  [3, NP, Tp]       moe_route_bwd logit gradient as three bf16 terms
+  size_t route_dw_partial; // fp32 [splits, d, NE] moe_route_bwd split-reduction partial sums
   size_t w_router_t;    // fp32  [E, d]            moe_permute_bwd transposed router
   size_t route_partial; // fp32  [splits, T, NE]   moe_route split-reduction partial logits
   size_t route_w3;      // bf16  [3, NP, d]        moe_route router weight as three bf16 terms
@@ -39,6 +39,8 @@ struct WsLayout {
 WsLayout ws_layout(int T, int d, int E, int k, int F);
 size_t route_partial_bytes(int T, int d, int E);
 size_t route_w3_bytes(int d, int E);
+size_t route_dz3_bytes(int T, int E);
+size_t route_dw_partial_bytes(int T, int d, int E);
 constexpr int kPermChunk = 4096;  // assignments per block in the permutation
 constexpr int kGroupPad = 128;    // rows per group are padded to this
 

@@ -49,9 +49,9 @@ constexpr int kRtMaxSmem = 232448;  // opt-in dynamic shared memory per CTA
 constexpr uint64_t kRtWaitNs = 2000000000ull;
 
 struct RouteTcParams {
-  int T;             // tokens
+  int M;             // output rows: tokens (logits) or d_model (router weight gradient)
   int kb_per_split;  // k-blocks of one split
-  int nkb;           // k-blocks in d
+  int nkb;           // k-blocks of the reduction (over d, or over the padded tokens)
   int NP;            // MMA N: experts rounded up to 16
   int NE;            // row stride of the partial logits
   int stages;        // shared-memory ring depth
@@ -69,16 +69,22 @@ int route_tc_stages(int NP) {
 size_t route_tc_smem(int NP, int stages) {
   return 1024 + size_t(stages) * route_tc_stage_bytes(NP) + size_t(2 * stages + 1) * 8 + 16;
 }
-// Splits of the reduction: enough CTAs to cover the SMs when T gives few tiles.
-// A function of (T, d) alone, so the workspace size is too.
-void route_tc_split(int T, int d, int *splits, int *kb_per_split) {
-  const int tiles = std::max(1, (T + kRtBM - 1) / kRtBM);
-  const int nkb = (d + kRtBK - 1) / kRtBK;
+// Splits of the reduction: enough CTAs to cover the SMs when the M rows (tokens for
+// the logits, d_model for the weight gradient) give few tiles. A function of
+// (M, K) alone, so the workspace size is too. K > 0.
+void route_tc_split(int M, int K, int *splits, int *kb_per_split) {
+  const int tiles = std::max(1, (M + kRtBM - 1) / kRtBM);
+  const int nkb = (K + kRtBK - 1) / kRtBK;
   int s = std::max(1, std::min({kRtTargetCtas / tiles, kRtMaxSplits, nkb}));
   const int per = (nkb + s - 1) / s;
   *kb_per_split = per;
   *splits = (nkb + per - 1) / per;  // every split gets at least one k-block
 }
+
+// Router weight gradient: tokens padded to one k-block, and the row stride of its
+// partial sums (the epilogue writes 32 columns at a time).
+int route_tokens_padded(int T) { return (T + kRtBK - 1) / kRtBK * kRtBK; }
+int route_dw_stride(int E) { return (route_tc_np(E) + 31) / 32 * 32; }
 
 // W [d, E] fp32 -> W3 [3][NP][d] bf16 (hi, mid, lo; rows e >= E are zero), by
 // 32 x 32 tiles transposed through shared memory.
@@ -109,9 +115,14 @@ __global__ void route_split_w_kernel(const float *__restrict__ w, int d, int E, 
   }
 }
 
+// DW = false: the logits, partial[split][t][e] = x[t, k-range] . W3[e, k-range].
+// DW = true: the router weight gradient, partial[split][i][e] = sum over the split's
+// tokens t of x[t, i] * dZ[t, e] (A = x^T, read MN-major from x itself as two 64 x 64
+// boxes per k-block; B = dZ's three bf16 terms, K-major [3][NP][T padded to 64]).
+template <bool DW>
 __global__ void __launch_bounds__(kRtThreads, 1)
-    route_logits_tc_kernel(const __grid_constant__ CUtensorMap tmX,
-                           const __grid_constant__ CUtensorMap tmW, const RouteTcParams p) {
+    route_tc_kernel(const __grid_constant__ CUtensorMap tmX,
+                    const __grid_constant__ CUtensorMap tmW, const RouteTcParams p) {
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = tc::smem_u32(smem_raw);
   const uint32_t pad = (1024u - (raw & 1023u)) & 1023u;
@@ -134,7 +145,7 @@ __global__ void __launch_bounds__(kRtThreads, 1)
   // Each tile starts its k-loop at its own offset, so that the CTAs do not all read
   // the same weight tile from L2 at the same time (the order is fixed per tile).
   const int rot = nk > 0 ? int((mt * 7u) % uint32_t(nk)) : 0;
-  const uint32_t idesc = tc::idesc_bf16_f32(kRtBM, p.NP, false, false);
+  const uint32_t idesc = tc::idesc_bf16_f32(kRtBM, p.NP, DW, false);
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < S; ++s) {
@@ -173,7 +184,12 @@ __global__ void __launch_bounds__(kRtThreads, 1)
       tc::mbar_arrive_expect_tx(full_bar(s), stage_bytes);
       const uint32_t dst = s0 + s * stage_bytes;
       const int k0 = kb * kRtBK;
-      tc::tma_load_2d(dst, &tmX, full_bar(s), k0, mt * kRtBM);
+      if (DW) {  // x^T: features mt*128 .. +127 (two 64-wide boxes) x tokens k0 .. k0+63
+        tc::tma_load_2d(dst, &tmX, full_bar(s), mt * kRtBM, k0);
+        tc::tma_load_2d(dst + 64 * 128, &tmX, full_bar(s), mt * kRtBM + 64, k0);
+      } else {
+        tc::tma_load_2d(dst, &tmX, full_bar(s), k0, mt * kRtBM);
+      }
 #pragma unroll
       for (int j = 0; j < 3; ++j)
         tc::tma_load_2d(dst + kRtABytes + j * b_bytes, &tmW, full_bar(s), k0, j * p.NP);
@@ -202,7 +218,8 @@ __global__ void __launch_bounds__(kRtThreads, 1)
       const uint32_t a_s = s0 + s * stage_bytes, b_s = a_s + kRtABytes;
 #pragma unroll
       for (int kk = 0; kk < kRtBK / 16; ++kk) {
-        const uint64_t ad = tc::smem_desc_sw128(a_s + kk * 32, 16, 1024);
+        const uint64_t ad = DW ? tc::smem_desc_sw128(a_s + kk * 2048, 8192, 1024)
+                               : tc::smem_desc_sw128(a_s + kk * 32, 16, 1024);
 #pragma unroll
         for (int j = 0; j < 3; ++j) {
           const uint64_t bd = tc::smem_desc_sw128(b_s + j * b_bytes + kk * 32, 16, 1024);
@@ -217,7 +234,7 @@ __global__ void __launch_bounds__(kRtThreads, 1)
   }
   __syncwarp();
 
-  // ---- epilogue: TMEM lane quarter `warp` -> 32 tokens x NP partial logits ----
+  // ---- epilogue: TMEM lane quarter `warp` -> 32 output rows x NP partial sums ----
   int ok = 0;
   if (lane == 0) {
     ok = tc::mbar_wait(done_bar, 0, kRtWaitNs, abort_flag) ? 1 : 0;
@@ -230,12 +247,12 @@ __global__ void __launch_bounds__(kRtThreads, 1)
   if (ok) {
     tc::fence_after_sync();
     const int t = mt * kRtBM + warp * 32 + lane;
-    float *dst = p.partial + (size_t(split) * p.T + t) * p.NE;
+    float *dst = p.partial + (size_t(split) * p.M + t) * p.NE;
     for (int c0 = 0; c0 < p.NP; c0 += 32) {
       uint32_t r[32];
       tc::tmem_ld_32x32b_x32(tmem_base + (uint32_t(warp * 32) << 16) + uint32_t(c0), r);
       tc::tmem_ld_wait();
-      if (t < p.T) {
+      if (t < p.M) {
 #pragma unroll
         for (int q = 0; q < 8; ++q)
           stg_v4(dst + c0 + 4 * q, make_uint4(r[4 * q], r[4 * q + 1], r[4 * q + 2], r[4 * q + 3]));
@@ -353,99 +370,70 @@ __global__ void load_stats_kernel(const int32_t *__restrict__ topk_idx, int64_t 
 
 // ---- router backward -------------------------------------------------------
 
-// d_logits[t,j] = g_j (dg_j - sum_i g_i dg_i); also scattered to the grouped rows.
-__global__ void route_bwd_dz_kernel(const float *__restrict__ gate, const float *__restrict__ dgate,
-                                    const int32_t *__restrict__ row_of_assignment, int T, int k,
-                                    int64_t rows_cap, float *__restrict__ d_logits,
-                                    float *__restrict__ dz_perm) {
+// Softmax backward over the selected k, d_logits[t,j] = g_j (dg_j - sum_i g_i dg_i),
+// and dZ (the [T, E] logit gradient, zero off the selected experts) as three bf16
+// terms, K-major for the tensor cores: dz3[s][e][t] for e < NP, t < Tp (tokens padded
+// to 64; the padding is zero). One thread per token and 16 experts (blockIdx.y); the
+// y = 0 blocks also write d_logits.
+constexpr int kDzExperts = 16;
+__global__ void route_bwd_dz_kernel(const int32_t *__restrict__ topk_idx,
+                                    const float *__restrict__ gate, const float *__restrict__ dgate,
+                                    int T, int Tp, int k, int NP, float *__restrict__ d_logits,
+                                    uint16_t *__restrict__ dz3) {
   const int t = blockIdx.x * blockDim.x + threadIdx.x;
-  if (t >= T) return;
+  if (t >= Tp) return;
   float g[8], dg[8], s = 0.f;
+  int ei[8];
 #pragma unroll
   for (int j = 0; j < 8; ++j) {
-    if (j < k) {
+    g[j] = 0.f;
+    dg[j] = 0.f;
+    ei[j] = -1;
+    if (j < k && t < T) {
       g[j] = gate[size_t(t) * k + j];
       dg[j] = dgate[size_t(t) * k + j];
+      ei[j] = topk_idx[size_t(t) * k + j];
       s = fmaf(g[j], dg[j], s);
     }
   }
 #pragma unroll
   for (int j = 0; j < 8; ++j) {
-    if (j < k) {
-      const float dz = g[j] * (dg[j] - s);
-      d_logits[size_t(t) * k + j] = dz;
-      const int r = row_of_assignment[size_t(t) * k + j];
-      if (r >= 0 && r < rows_cap) dz_perm[r] = dz;
-    }
+    g[j] = g[j] * (dg[j] - s);
+    if (blockIdx.y == 0 && j < k && t < T) d_logits[size_t(t) * k + j] = g[j];
+  }
+  const size_t plane = size_t(NP) * Tp;
+  const int e0 = blockIdx.y * kDzExperts;
+  for (int e = e0; e < min(NP, e0 + kDzExperts); ++e) {
+    float v = 0.f;
+#pragma unroll
+    for (int j = 0; j < 8; ++j)
+      if (ei[j] == e) v = g[j];  // the k selected experts of a token are distinct
+    const __nv_bfloat16 hi = __float2bfloat16_rn(v);
+    const float r1 = v - __bfloat162float(hi);
+    const __nv_bfloat16 mid = __float2bfloat16_rn(r1);
+    const float r2 = r1 - __bfloat162float(mid);
+    const __nv_bfloat16 lo = __float2bfloat16_rn(r2);
+    const size_t at = size_t(e) * Tp + t;
+    dz3[at] = __bfloat16_as_ushort(hi);
+    dz3[plane + at] = __bfloat16_as_ushort(mid);
+    dz3[2 * plane + at] = __bfloat16_as_ushort(lo);
   }
 }
 
-// One CTA per 128-row tile of the grouped layout: partial[tile, :] =
-// sum over the tile's real rows of dz_perm[r] * X_perm[r, :], where X_perm row r is
-// x_src row r, or x_src row token_of_row[r] when token_of_row is given (x itself).
-__global__ void __launch_bounds__(256) route_bwd_partial_kernel(
-    const uint16_t *__restrict__ x_src, const int32_t *__restrict__ token_of_row,
-    const float *__restrict__ dz_perm, const int32_t *__restrict__ group_offsets,
-    const int32_t *__restrict__ group_counts, int E, int d, float *__restrict__ partial) {
-  const int tile = blockIdx.x;
-  const int row0 = tile * moe::kGroupPad;
-  if (row0 >= group_offsets[E]) return;
-  // group containing row0: last e with group_offsets[e] <= row0
-  int lo = 0, hi = E - 1;
-  while (lo < hi) {
-    const int mid = (lo + hi + 1) >> 1;
-    if (group_offsets[mid] <= row0) lo = mid; else hi = mid - 1;
-  }
-  const int e = lo;
-  const int row_end = min(row0 + moe::kGroupPad, group_offsets[e] + group_counts[e]);
-  for (int c8 = threadIdx.x; c8 < d / 8; c8 += blockDim.x) {
-    float acc[8];
-#pragma unroll
-    for (int q = 0; q < 8; ++q) acc[q] = 0.f;
-    int r = row0;
-    // eight rows per step: eight independent 16-byte loads in flight per thread
-    for (; r + 8 <= row_end; r += 8) {
-      uint4 v[8];
-      float w[8];
-#pragma unroll
-      for (int u = 0; u < 8; ++u) {
-        w[u] = dz_perm[r + u];
-        const size_t src = token_of_row != nullptr ? size_t(token_of_row[r + u]) : size_t(r + u);
-        v[u] = ldg_nc_v4(x_src + src * d + c8 * 8);
-      }
-#pragma unroll
-      for (int u = 0; u < 8; ++u) {
-        float f[8];
-        unpack8(v[u], f);
-#pragma unroll
-        for (int q = 0; q < 8; ++q) acc[q] = fmaf(w[u], f[q], acc[q]);
-      }
-    }
-    for (; r < row_end; ++r) {
-      const float w = dz_perm[r];
-      const size_t src = token_of_row != nullptr ? size_t(token_of_row[r]) : size_t(r);
-      float f[8];
-      unpack8(ldg_nc_v4(x_src + src * d + c8 * 8), f);
-#pragma unroll
-      for (int q = 0; q < 8; ++q) acc[q] = fmaf(w, f[q], acc[q]);
-    }
-    float4 *dst = reinterpret_cast<float4 *>(partial + size_t(tile) * d + c8 * 8);
-    dst[0] = make_float4(acc[0], acc[1], acc[2], acc[3]);
-    dst[1] = make_float4(acc[4], acc[5], acc[6], acc[7]);
+// dw_router[i, e] = sum over the splits, in order, of partial[split][i][e].
+__global__ void route_dw_reduce_kernel(const float *__restrict__ partial, int splits, int d,
+                                       int E, int NE, float *__restrict__ dw_router) {
+  const int n = d * E;
+  for (int idx = blockIdx.x * blockDim.x + threadIdx.x; idx < n; idx += gridDim.x * blockDim.x) {
+    const int i = idx / E, e = idx - i * E;
+    float acc = 0.f;
+    for (int y = 0; y < splits; ++y) acc += partial[(size_t(y) * d + i) * NE + e];
+    dw_router[idx] = acc;
   }
 }
 
-// dw_router[i, e] = sum over the tiles of group e of partial[tile, i]
-__global__ void route_bwd_reduce_kernel(const float *__restrict__ partial,
-                                        const int32_t *__restrict__ group_offsets, int E, int d,
-                                        float *__restrict__ dw_router) {
-  const int e = blockIdx.y;
-  const int i = blockIdx.x * blockDim.x + threadIdx.x;
-  if (i >= d) return;
-  const int tb = group_offsets[e] / moe::kGroupPad, te = group_offsets[e + 1] / moe::kGroupPad;
-  float s = 0.f;
-  for (int tile = tb; tile < te; ++tile) s += partial[size_t(tile) * d + i];
-  dw_router[size_t(i) * E + e] = s;
+__global__ void zero_f32_kernel(float *p, int n) {
+  for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < n; i += gridDim.x * blockDim.x) p[i] = 0.f;
 }
 
 // Tensor-core logits: splits W into its three bf16 terms (w3), then one CTA per
@@ -457,7 +445,7 @@ int launch_route_tc(const uint16_t *x, const float *w, int T, int d, int E, int 
   const size_t smem = route_tc_smem(NP, stages);
   static bool attr_set = false;
   if (!attr_set) {
-    cudaError_t e = cudaFuncSetAttribute(route_logits_tc_kernel,
+    cudaError_t e = cudaFuncSetAttribute(route_tc_kernel<false>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, kRtMaxSmem);
     if (e != cudaSuccess) return moe::cuda_status(e, "moe_route: set smem attribute");
     attr_set = true;
@@ -473,7 +461,7 @@ int launch_route_tc(const uint16_t *x, const float *w, int T, int d, int E, int 
   int splits = 1, per = 1;
   route_tc_split(T, d, &splits, &per);
   RouteTcParams p;
-  p.T = T;
+  p.M = T;
   p.kb_per_split = per;
   p.nkb = (d + kRtBK - 1) / kRtBK;
   p.NP = NP;
@@ -482,7 +470,7 @@ int launch_route_tc(const uint16_t *x, const float *w, int T, int d, int E, int 
   p.tmem_cols = route_tc_tmem_cols(NP);
   p.partial = partial;
   dim3 grid((T + kRtBM - 1) / kRtBM, splits);
-  MOE_LAUNCH("route_logits", s, route_logits_tc_kernel<<<grid, kRtThreads, smem, s>>>(mx, mw, p));
+  MOE_LAUNCH("route_logits", s, route_tc_kernel<false><<<grid, kRtThreads, smem, s>>>(mx, mw, p));
   *splits_out = splits;
   return moe::launch_status("moe_route: logits");
 }
@@ -512,6 +500,15 @@ size_t route_partial_bytes(int T, int d, int E) {
   return size_t(splits) * size_t(T) * size_t(padded_experts(E)) * 4;
 }
 size_t route_w3_bytes(int d, int E) { return size_t(3) * route_tc_np(E) * size_t(d) * 2; }
+size_t route_dz3_bytes(int T, int E) {
+  return size_t(3) * route_tc_np(E) * size_t(route_tokens_padded(T)) * 2;
+}
+size_t route_dw_partial_bytes(int T, int d, int E) {
+  if (T <= 0) return 0;
+  int splits = 1, per = 1;
+  route_tc_split(d, route_tokens_padded(T), &splits, &per);
+  return size_t(splits) * size_t(d) * size_t(route_dw_stride(E)) * 4;
+}
 }  // namespace moe
 
 extern "C" {
@@ -569,62 +566,75 @@ int moe_load_stats(const int32_t *topk_idx, int T, int k, int E, int32_t *counts
 }  // extern "C"
 
 namespace {
-int route_bwd_impl(const char *fn, const uint16_t *x_src, const int32_t *token_of_row,
-                   const float *topk_gate, const float *d_gate, const int32_t *row_of_assignment,
-                   const int32_t *group_offsets, const int32_t *group_counts, int T, int d, int E,
-                   int k, int64_t rows_cap, float *d_logits, float *dw_router, void *ws,
-                   size_t ws_bytes, cudaStream_t s) {
-  if (E < 1 || E > 256 || k < 1 || k > 8 || T < 0 || d <= 0 || d % 8)
-    return moe::set_error(MOE_ERR_ARG, "%s: sizes", fn);
-  if (!group_offsets || !group_counts || !dw_router || !ws ||
-      (T > 0 && (!x_src || !topk_gate || !d_gate || !row_of_assignment || !d_logits)))
-    return moe::set_error(MOE_ERR_ARG, "%s: null pointer", fn);
-  if (rows_cap < moe_perm_rows_max(T, k, E)) return moe::set_error(MOE_ERR_ARG, "%s: rows_cap too small", fn);
-  if ((x_src && !moe::aligned16(x_src)) || !moe::aligned16(ws))
-    return moe::set_error(MOE_ERR_ARG, "%s: alignment", fn);
-  const moe::WsLayout L = moe::ws_layout(T, d, E, k, 0);
-  if (ws_bytes < L.total) return moe::set_error(MOE_ERR_WORKSPACE, "%s: workspace", fn);
-  float *dz_perm = reinterpret_cast<float *>(static_cast<char *>(ws) + L.dz_perm);
-  float *partial = reinterpret_cast<float *>(static_cast<char *>(ws) + L.rb_partial);
-  if (T > 0) {
-    MOE_LAUNCH("route_bwd_dz", s, route_bwd_dz_kernel<<<(T + 255) / 256, 256, 0, s>>>(topk_gate, d_gate, row_of_assignment, T, k,
-                                                        rows_cap, d_logits, dz_perm));
-    if (int st = moe::launch_status("moe_route_bwd: dz")) return st;
-    const int tiles = int(rows_cap / moe::kGroupPad);
-    MOE_LAUNCH("route_bwd_partial", s, route_bwd_partial_kernel<<<tiles, 256, 0, s>>>(
-                                           x_src, token_of_row, dz_perm, group_offsets,
-                                           group_counts, E, d, partial));
-    if (int st = moe::launch_status("moe_route_bwd: partial")) return st;
+// Weight-gradient launch on the tensor cores: partial[split][i][e] over the split's tokens.
+int launch_route_dw(const uint16_t *x, const uint16_t *dz3, int T, int d, int E, float *partial,
+                    int *splits_out, cudaStream_t s) {
+  const int NP = route_tc_np(E), Tp = route_tokens_padded(T);
+  const int stages = route_tc_stages(NP);
+  const size_t smem = route_tc_smem(NP, stages);
+  static bool attr_set = false;
+  if (!attr_set) {
+    cudaError_t e = cudaFuncSetAttribute(route_tc_kernel<true>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, kRtMaxSmem);
+    if (e != cudaSuccess) return moe::cuda_status(e, "moe_route_bwd: set smem attribute");
+    attr_set = true;
   }
-  dim3 grid((d + 255) / 256, E);
-  MOE_LAUNCH("route_bwd_reduce", s, route_bwd_reduce_kernel<<<grid, 256, 0, s>>>(partial, group_offsets, E, d, dw_router));
-  return moe::launch_status("moe_route_bwd: reduce");
+  CUtensorMap mx, mz;
+  int st;
+  // x [T, d] read as 64 features x 64 tokens boxes (features contiguous: MN-major A)
+  if ((st = moe::make_map(&mx, x, uint64_t(T), uint64_t(d), 64, kRtBK, "router bwd x"))) return st;
+  if ((st = moe::make_map(&mz, dz3, uint64_t(3 * NP), uint64_t(Tp), kRtBK, uint32_t(NP), "router bwd dz")))
+    return st;
+  int splits = 1, per = 1;
+  route_tc_split(d, Tp, &splits, &per);
+  RouteTcParams p;
+  p.M = d;
+  p.kb_per_split = per;
+  p.nkb = Tp / kRtBK;
+  p.NP = NP;
+  p.NE = route_dw_stride(E);
+  p.stages = stages;
+  p.tmem_cols = route_tc_tmem_cols(NP);
+  p.partial = partial;
+  dim3 grid((d + kRtBM - 1) / kRtBM, splits);
+  MOE_LAUNCH("route_bwd_dw", s, route_tc_kernel<true><<<grid, kRtThreads, smem, s>>>(mx, mz, p));
+  *splits_out = splits;
+  return moe::launch_status("moe_route_bwd: weight gradient");
 }
 }  // namespace
 
 extern "C" {
 
-int moe_route_bwd(const uint16_t *x_perm, const int32_t *topk_idx, const float *topk_gate,
-                  const float *d_gate, const int32_t *row_of_assignment,
-                  const int32_t *group_offsets, const int32_t *group_counts, int T, int d, int E,
-                  int k, int64_t rows_cap, float *d_logits, float *dw_router, void *ws,
-                  size_t ws_bytes, moe_stream_t stream) {
-  (void)topk_idx;
-  if (!x_perm) return moe::set_error(MOE_ERR_ARG, "moe_route_bwd: null x_perm");
-  return route_bwd_impl("moe_route_bwd", x_perm, nullptr, topk_gate, d_gate, row_of_assignment,
-                        group_offsets, group_counts, T, d, E, k, rows_cap, d_logits, dw_router,
-                        ws, ws_bytes, reinterpret_cast<cudaStream_t>(stream));
-}
-
-int moe_route_bwd_gather(const uint16_t *x, const int32_t *token_of_row, const float *topk_gate,
-                         const float *d_gate, const int32_t *row_of_assignment,
-                         const int32_t *group_offsets, const int32_t *group_counts, int T, int d,
-                         int E, int k, int64_t rows_cap, float *d_logits, float *dw_router,
-                         void *ws, size_t ws_bytes, moe_stream_t stream) {
-  if (T > 0 && !token_of_row) return moe::set_error(MOE_ERR_ARG, "moe_route_bwd_gather: null token_of_row");
-  return route_bwd_impl("moe_route_bwd_gather", x, token_of_row, topk_gate, d_gate,
-                        row_of_assignment, group_offsets, group_counts, T, d, E, k, rows_cap,
-                        d_logits, dw_router, ws, ws_bytes, reinterpret_cast<cudaStream_t>(stream));
+int moe_route_bwd(const uint16_t *x, const int32_t *topk_idx, const float *topk_gate,
+                  const float *d_gate, int T, int d, int E, int k, float *d_logits,
+                  float *dw_router, void *ws, size_t ws_bytes, moe_stream_t stream) {
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if (E < 1 || E > 256 || k < 1 || k > 8 || k > E || T < 0 || d <= 0 || d % 8)
+    return moe::set_error(MOE_ERR_ARG, "moe_route_bwd: sizes");
+  if (!dw_router || (T > 0 && (!x || !topk_idx || !topk_gate || !d_gate || !d_logits || !ws)))
+    return moe::set_error(MOE_ERR_ARG, "moe_route_bwd: null pointer");
+  if ((x && !moe::aligned16(x)) || (ws && !moe::aligned16(ws)))
+    return moe::set_error(MOE_ERR_ARG, "moe_route_bwd: alignment");
+  if (T == 0) {
+    const int n = d * E;
+    MOE_LAUNCH("zero_dw_router", s, zero_f32_kernel<<<std::min((n + 255) / 256, 1024), 256, 0, s>>>(dw_router, n));
+    return moe::launch_status("moe_route_bwd: zero");
+  }
+  const moe::WsLayout L = moe::ws_layout(T, d, E, k, 0);
+  if (ws_bytes < L.total) return moe::set_error(MOE_ERR_WORKSPACE, "moe_route_bwd: workspace");
+  uint16_t *dz3 = reinterpret_cast<uint16_t *>(static_cast<char *>(ws) + L.route_dz3);
+  float *partial = reinterpret_cast<float *>(static_cast<char *>(ws) + L.route_dw_partial);
+  const int NP = route_tc_np(E), Tp = route_tokens_padded(T);
+  dim3 zgrid((Tp + 255) / 256, (NP + kDzExperts - 1) / kDzExperts);
+  MOE_LAUNCH("route_bwd_dz", s, route_bwd_dz_kernel<<<zgrid, 256, 0, s>>>(
+                                    topk_idx, topk_gate, d_gate, T, Tp, k, NP, d_logits, dz3));
+  if (int st = moe::launch_status("moe_route_bwd: dz")) return st;
+  int splits = 0;
+  if (int st = launch_route_dw(x, dz3, T, d, E, partial, &splits, s)) return st;
+  const int n = d * E;
+  MOE_LAUNCH("route_bwd_reduce", s, route_dw_reduce_kernel<<<std::min((n + 255) / 256, 4 * moe::num_sms()), 256, 0, s>>>(
+                                        partial, splits, d, E, route_dw_stride(E), dw_router));
+  return moe::launch_status("moe_route_bwd: reduce");
 }
 
 }  // extern "C"

@@ -41,7 +41,7 @@ class MoELayerBuffers:
         s = shape
         self.shape = s
         self.gather = gather
-        self.x = None  # the forward's input, kept for the backward in gather mode
+        self.x = None  # the forward's input, kept for the backward
         R = s.rows_cap
         dev = torch.device(device)
         bf16, f32, i32 = torch.bfloat16, torch.float32, torch.int32
@@ -93,8 +93,8 @@ def forward(b: MoELayerBuffers, x, w_router, bias, w_gate_up, w_down, active_mas
     s = b.shape
     R = s.rows_cap
     route(b, x, w_router, bias, active_mask, logits_in, keep_logits, stream)
+    b.x = x
     if b.gather:
-        b.x = x
         L.moe_permute_map(b.topk_idx, b.counts, s.T, s.E, s.k, R, b.group_offsets,
                           b.group_counts, b.row_of_assignment, b.token_of_row, b.ws, b.ws_bytes,
                           stream)
@@ -130,14 +130,8 @@ def backward(b: MoELayerBuffers, dy, w_router, w_gate_up, w_down, stream=None,
         ev = torch.cuda.Event()
         ev.record(main)
         side.wait_event(ev)
-    if b.gather:
-        L.moe_route_bwd_gather(b.x, b.token_of_row, b.topk_gate, b.d_gate, b.row_of_assignment,
-                               b.group_offsets, b.group_counts, s.T, s.d, s.E, s.k, R,
-                               b.d_logits, b.dw_router, b.ws, b.ws_bytes, side)
-    else:
-        L.moe_route_bwd(b.x_perm, b.topk_idx, b.topk_gate, b.d_gate, b.row_of_assignment,
-                        b.group_offsets, b.group_counts, s.T, s.d, s.E, s.k, R, b.d_logits,
-                        b.dw_router, b.ws, b.ws_bytes, side)
+    L.moe_route_bwd(b.x, b.topk_idx, b.topk_gate, b.d_gate, s.T, s.d, s.E, s.k, b.d_logits,
+                    b.dw_router, b.ws, b.ws_bytes, side)
     L.moe_grouped_ffn_bwd_dgrad(b.d_out_perm, b.ab, b.group_offsets, s.E, s.d, s.F, R,
                                 w_gate_up, w_down, b.d_ab, b.dx_perm, main)
     if overlap:

@@ -87,13 +87,12 @@ def main():
                                                  ws_bytes), a.iters, a.warmup)
             nbytes = 2 * T * k * d + 2 * T * d
         elif a.call == "route_bwd":
-            permute()
             dg = torch.randn(T, k, generator=gen, device=dev)
             dl = torch.empty(T, k, dtype=torch.float32, device=dev)
             dw = torch.empty(d, E, dtype=torch.float32, device=dev)
-            ms = _time(lambda: L.moe_route_bwd(xp, idx, gate, dg, row, goff, gcnt, T, d, E, k, R,
-                                               dl, dw, ws, ws_bytes), a.iters, a.warmup)
-            nbytes = 2 * T * k * d
+            ms = _time(lambda: L.moe_route_bwd(x, idx, gate, dg, T, d, E, k, dl, dw, ws,
+                                               ws_bytes), a.iters, a.warmup)
+            nbytes = 2 * T * d
         else:
             permute()
             y = torch.empty(T, d, dtype=torch.bfloat16, device=dev)

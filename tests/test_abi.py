@@ -37,8 +37,12 @@ def test_sizes(lib):
     assert L.moe_version() == 100
     assert L.moe_perm_rows_max(100, 8, 64) == 800 + 128 * 64
     ws = L.moe_workspace_size(16384, 4096, 64, 8, 2048)
-    R = 16384 * 8 + 128 * 64
-    assert ws >= R * 4 + (R // 128) * 4096 * 4 + 64 * 4096 * 4
+    # router backward: dZ as three bf16 terms [3, 64, T] and the split partial sums of
+    # dW_r [splits >= 1, d, 64]; transposed router [E, d]; partial logits [T, 64]; W_r
+    # as three bf16 terms [3, 64, d]
+    assert ws >= 3 * 64 * 16384 * 2 + 4096 * 64 * 4 + 64 * 4096 * 4 + 16384 * 64 * 4 \
+        + 3 * 64 * 4096 * 2
+    assert L.moe_workspace_size(0, 4096, 64, 8, 2048) >= 64 * 4096 * 4
 
 
 def test_laep_prune_mask_golden(lib):
@@ -155,10 +159,18 @@ def test_new_entry_points_validate_before_launch(lib):
         L.moe_grouped_ffn_bwd_wgrad_gather(16, 16, 20, 10, 16, 16, 16, 8, 128, 256, R, 16, 16,
                                            stream=0)
     assert e.value.status == -1
-    with pytest.raises(L.MoEError) as e:  # router backward through the map needs the map
-        L.moe_route_bwd_gather(16, None, 16, 16, 16, 16, 16, 10, 128, 8, 2, R, 16, 16, 16,
-                               1 << 20, stream=0)
+    with pytest.raises(L.MoEError) as e:  # router backward: x missing with tokens present
+        L.moe_route_bwd(None, 16, 16, 16, 10, 128, 8, 2, 16, 16, 16, 1 << 20, stream=0)
     assert e.value.status == -1
+    with pytest.raises(L.MoEError) as e:  # router backward: unaligned x
+        L.moe_route_bwd(24, 16, 16, 16, 10, 128, 8, 2, 16, 16, 16, 1 << 20, stream=0)
+    assert e.value.status == -1
+    with pytest.raises(L.MoEError) as e:  # router backward: k above E
+        L.moe_route_bwd(16, 16, 16, 16, 10, 128, 4, 5, 16, 16, 16, 1 << 20, stream=0)
+    assert e.value.status == -1
+    with pytest.raises(L.MoEError) as e:  # router backward: workspace too small
+        L.moe_route_bwd(16, 16, 16, 16, 10, 128, 8, 2, 16, 16, 16, 4, stream=0)
+    assert e.value.status == -6
     with pytest.raises(L.MoEError) as e:  # combine backward with neither output
         L.moe_unpermute_combine_bwd(16, 16, 16, 16, 16, 16, 10, 128, 8, 2, None, None, stream=0)
     assert e.value.status == -1

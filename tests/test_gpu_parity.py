@@ -90,6 +90,45 @@ def test_route_logits_fp32(T, d, E):
     assert (idx[clear] == oidx[clear]).all()
 
 
+@pytest.mark.parametrize("T,d,E,k", [(3000, 256, 64, 8), (777, 512, 171, 4), (129, 200, 256, 8),
+                                     # tokens not a multiple of the 64-token k-block, d not a
+                                     # multiple of the 128-feature tile, MMA N = 16, one token
+                                     (333, 136, 13, 2), (1, 72, 5, 1), (64, 8, 2, 2),
+                                     (4100, 1024, 16, 2)])
+def test_route_bwd_against_oracle(T, d, E, k):
+    """moe_route_bwd alone, from the same fp32 gates and d_gate as the oracle."""
+    dev = "cuda"
+    inp = case_inputs(T, d, E, k, 128, seed=11)
+    gen = torch.Generator().manual_seed(T + d)
+    z = torch.randn(T, E, generator=gen)
+    idx = torch.argsort(z, dim=1, descending=True)[:, :k].to(torch.int32).contiguous()
+    gate = torch.softmax(torch.gather(z, 1, idx.long()), dim=1).contiguous()
+    dg = torch.randn(T, k, generator=gen).contiguous()
+    x = inp["x"]
+    dz_ref, dw_ref = O.router_backward(x.double().numpy(), idx.numpy(), gate.double().numpy(),
+                                       dg.double().numpy(), E)
+    ws_bytes = L.moe_workspace_size(T, d, E, k, 128)
+    ws = torch.empty(ws_bytes, dtype=torch.uint8, device=dev)
+    dl = torch.empty(T, k, dtype=torch.float32, device=dev)
+    dw = torch.full((d, E), float("nan"), dtype=torch.float32, device=dev)
+    L.moe_route_bwd(x.to(dev), idx.to(dev), gate.to(dev), dg.to(dev), T, d, E, k, dl, dw, ws,
+                    ws_bytes)
+    torch.cuda.synchronize()
+    g64, dg64 = gate.double().numpy(), dg.double().numpy()
+    # fp32 arithmetic on both terms of the softmax backward
+    zscale = np.abs(g64) * (np.abs(dg64) + np.sum(np.abs(g64 * dg64), axis=1, keepdims=True))
+    assert (np.abs(dl.cpu().numpy() - dz_ref) <= 2e-6 * zscale + 1e-30).all()
+    # dZ carried exactly by three bf16 terms, products exact, fp32 accumulation over T
+    dzs = np.zeros((T, E))
+    np.put_along_axis(dzs, idx.numpy().astype(np.int64), zscale, axis=1)
+    scale = np.abs(x.double().numpy()).T @ dzs
+    got = dw.cpu().numpy().astype(np.float64)
+    assert np.isfinite(got).all()
+    assert (np.abs(got - dw_ref) <= 1e-5 * scale + 1e-30).all()
+    unused = np.setdiff1d(np.arange(E), idx.numpy())
+    assert (got[:, unused] == 0).all()
+
+
 def test_load_stats_bit_exact_and_accumulate():
     T, k, E = 5000, 8, 200
     rng = np.random.default_rng(1)

@@ -146,7 +146,7 @@ class Workload:
 
     def __init__(self, cfg_id: int, device: str, compact_override=None, tokens=None,
                  experts=None, no_prune=False, bias=None, gather=False, overlap=True,
-                 backward=None):
+                 backward=None, fused_combine=False):
         c = synth.CONFIGS[cfg_id]
         if tokens or experts or no_prune or bias:  # a variant of the workload (profiling)
             import dataclasses
@@ -190,7 +190,7 @@ class Workload:
         # the forward-only workloads time the forward pass (backward=True forces both)
         self.backward = c.backward if backward is None else bool(backward)
         self.bufs = layer.MoELayerBuffers(self.shape, device, backward=self.backward,
-                                          gather=gather)
+                                          gather=gather, fused_combine=fused_combine)
 
         self.graph = None
         self.overlap = overlap
@@ -413,7 +413,7 @@ def laep_comparison(args, world, local, pruned_tps, wl_pruned):
     wl_pruned.bufs = None
     torch.cuda.empty_cache()
     wl_u = Workload(args.config, "cuda", no_prune=True, gather=bool(args.gather),
-                    overlap=bool(args.overlap))
+                    overlap=bool(args.overlap), fused_combine=bool(args.fused_combine))
     for _ in range(args.warmup):
         wl_u.step()
     if args.graph:
@@ -443,7 +443,7 @@ def run_ours(args):
     peaks = measured_peaks()
     wl = Workload(args.config, "cuda", tokens=args.tokens, experts=args.experts,
                   no_prune=args.no_prune, bias=args.bias, gather=bool(args.gather),
-                  overlap=bool(args.overlap))
+                  overlap=bool(args.overlap), fused_combine=bool(args.fused_combine))
     s = wl.shape
     torch.cuda.synchronize()
     for _ in range(args.warmup):
@@ -604,7 +604,9 @@ def run_ours(args):
                           % (2 * s.T * s.d / 1e6, 6 * s.E * s.d * s.F / 1e9)),
                    "parallelism": "replicas" if world > 1 else "1 GPU",
                    "dispatch": ("TMA gathers from x (X_perm not materialized)" if args.gather
-                                else "materialized X_perm")},
+                                else "materialized X_perm"),
+                   "combine": ("in the down GEMM's epilogue (fp32 atomics)" if args.fused_combine
+                               else "separate kernel")},
         "grouped_gemm": {"tflops": round(all_gemm_tflops, 1),
                          "frac_of_peak": round(all_gemm_tflops / peak, 4),
                          "peak_tflops": peak, "peak": f"bf16 sustained, {peaks['source']}",
@@ -695,6 +697,9 @@ def main():
     ap.add_argument("--gather", type=int, default=0,
                     help="dispatch through a materialized X_perm (0), or by 4-row TMA gathers "
                          "from x with X_perm never written (1; same results, slower GEMMs)")
+    ap.add_argument("--fused-combine", type=int, default=0,
+                    help="combine in a separate kernel (0) or in the down GEMM's epilogue with "
+                         "fp32 atomics (1; y's last bits may vary from run to run)")
     ap.add_argument("--overlap", type=int, default=1,
                     help="router backward and unpermute-sum on a second stream beside the "
                          "GEMMs (1) or on the main stream after them (0)")

@@ -253,6 +253,28 @@ int moe_grouped_ffn_fwd(const uint16_t *x_perm, const int32_t *group_offsets, in
                         uint16_t *out_perm, void *ws, size_t ws_bytes, moe_stream_t stream);
 
 /*
+ * moe_grouped_ffn_fwd_combine - moe_grouped_ffn_fwd with the combine of
+ * moe_unpermute_combine done in the down GEMM's epilogue:
+ *   y[t,:] = bf16( sum_j topk_gate[t,j] * O[row_of_assignment[t,j], :] )
+ * The epilogue adds gate * O (its fp32 accumulator, before any bf16 rounding) into
+ * y_acc with fp32 atomics, so the order of the k terms of a token, and the last
+ * bits of y, can change from run to run (the unfused pair is bitwise
+ * reproducible). out_perm may be NULL: O is then not stored (enough for a forward
+ * without backward). y_acc [T,d] fp32 is caller-owned scratch (overwritten); y
+ * [T,d] bf16 (out). row_of_assignment, topk_gate [T,k] as moe_permute/moe_route
+ * wrote them; ws: moe_workspace_size(T, d, E, k, F) bytes (the token and gate of
+ * each grouped row live there). Other arguments, outputs and limits as in
+ * moe_grouped_ffn_fwd; 1 <= k <= min(8, E); rows_cap >= moe_perm_rows_max(T,k,E).
+ * A row index outside [0, moe_perm_rows_max) sets MOE_DEV_ROWS_OVERFLOW.
+ */
+int moe_grouped_ffn_fwd_combine(const uint16_t *x_perm, const int32_t *group_offsets, int E, int d,
+                                int F, int64_t rows_cap, const uint16_t *w_gate_up,
+                                const uint16_t *w_down, const int32_t *row_of_assignment,
+                                const float *topk_gate, int T, int k, uint16_t *ab_saved,
+                                uint16_t *h, uint16_t *out_perm, float *y_acc, uint16_t *y,
+                                void *ws, size_t ws_bytes, moe_stream_t stream);
+
+/*
  * Gathered form of the dispatch (no X_perm in memory). The grouped operand X_perm
  * of the forward GEMM and of the dW_gate_up GEMM is taken from x itself through a
  * row -> token map: grouped

@@ -60,6 +60,7 @@ _SIGS = {
     "moe_route_bwd": (I, [P, P, P, P, I, I, I, I, P, P, P, SZ, P]),
     "moe_permute_bwd": (I, [P, P, P, P, P, I, I, I, I, P, P, SZ, P]),
     "moe_permute_map": (I, [P, P, I, I, I, I64, P, P, P, P, P, SZ, P]),
+    "moe_grouped_ffn_fwd_combine": (I, [P, P, I, I, I, I64, P, P, P, P, I, I, P, P, P, P, P, P, SZ, P]),
     "moe_grouped_ffn_fwd_gather": (I, [P, P, I, P, I, I, I, I64, P, P, P, P, P, P, SZ, P]),
     "moe_grouped_ffn_bwd_wgrad_gather": (I, [P, P, P, I, P, P, P, I, I, I, I64, P, P, P]),
     "moe_selftest_wait_timeout": (I, [I64, P]),
@@ -276,6 +277,15 @@ def moe_permute_map(topk_idx, counts, T, E, k, rows_cap, group_offsets, group_co
     _check("moe_permute_map", load().moe_permute_map(
         _ptr(topk_idx), _ptr(counts), T, E, k, rows_cap, _ptr(group_offsets), _ptr(group_counts),
         _ptr(row_of_assignment), _ptr(token_of_row), _ptr(ws), ws_bytes, _stream(stream)))
+
+
+def moe_grouped_ffn_fwd_combine(x_perm, group_offsets, E, d, F, rows_cap, w_gate_up, w_down,
+                                row_of_assignment, topk_gate, T, k, ab_saved, h, out_perm, y_acc,
+                                y, ws, ws_bytes, stream=None):
+    _check("moe_grouped_ffn_fwd_combine", load().moe_grouped_ffn_fwd_combine(
+        _ptr(x_perm), _ptr(group_offsets), E, d, F, rows_cap, _ptr(w_gate_up), _ptr(w_down),
+        _ptr(row_of_assignment), _ptr(topk_gate), T, k, _ptr(ab_saved), _ptr(h), _ptr(out_perm),
+        _ptr(y_acc), _ptr(y), _ptr(ws), ws_bytes, _stream(stream)))
 
 
 def moe_grouped_ffn_fwd_gather(x, token_of_row, T, group_offsets, E, d, F, rows_cap, w_gate_up,

@@ -85,6 +85,12 @@ struct GemmParams {
   // Gathered operand (kGateUp: A, kWgradGateUp: B): grouped row r reads row
   // token_of_row[r] of x [T, d] instead of row r of X_perm (nullptr: X_perm).
   const int32_t *token_of_row;
+  // kDown with the combine in the epilogue (nullptr: no combine): for every real
+  // grouped row r, y_acc[row_token[r], cols] += row_gate[r] * O[r, cols] in fp32
+  // (row_token[r] < 0 on padding rows). out == nullptr then skips the O store.
+  float *y_acc;
+  const int32_t *row_token;
+  const float *row_gate;
 };
 
 struct Tile {
@@ -228,14 +234,30 @@ __device__ __forceinline__ void epilogue_tile(const GemmParams &p, const CUtenso
     } else {
       trow = int(row) - lane;
     }
+    // combine: this lane's row goes to token `tok` with weight `g` (tok < 0: padding)
+    int tok = -1;
+    float g = 0.f;
+    if (MODE == kDown && p.y_acc != nullptr) {
+      tok = p.row_token[row];
+      g = p.row_gate[row];
+    }
 #pragma unroll 1
     for (int c = half * (BN / 2); c < (half + 1) * (BN / 2); c += 32) {
       uint32_t r[32];
       tc::tmem_ld_32x32b_x32(tb + c, r);
       tc::tmem_ld_wait();
-      uint4 v[4];
-      pack32(r, v);
-      stage_and_store(tmO, stage, lane, v, nt * BN + c, trow);
+      if (MODE == kDown && tok >= 0) {
+        float4 *dst = reinterpret_cast<float4 *>(p.y_acc + size_t(tok) * p.d + nt * BN + c);
+#pragma unroll
+        for (int q = 0; q < 8; ++q)
+          atomicAdd(dst + q, make_float4(g * __uint_as_float(r[4 * q]), g * __uint_as_float(r[4 * q + 1]),
+                                         g * __uint_as_float(r[4 * q + 2]), g * __uint_as_float(r[4 * q + 3])));
+      }
+      if (MODE != kDown || p.out != nullptr) {
+        uint4 v[4];
+        pack32(r, v);
+        stage_and_store(tmO, stage, lane, v, nt * BN + c, trow);
+      }
     }
   }
 }
@@ -971,9 +993,24 @@ int launch_pair(const CUtensorMap &a, const CUtensorMap &b, const CUtensorMap &o
 // bf16; B likewise. N = output columns (for kGateUp: 2F, in tiles of 128 gate + 128 up).
 // The output p.out is [o_rows, o_cols] row-major bf16.
 template <int MODE>
+int run_gemm_out(int N, const void *a_base, uint64_t a_rows, uint64_t a_cols, const void *b_base,
+                 uint64_t b_rows, uint64_t b_cols, const void *o_base, uint64_t o_rows,
+                 uint64_t o_cols, GemmParams p, cudaStream_t s, const char *what);
+
+template <int MODE>
 int run_gemm(int N, const void *a_base, uint64_t a_rows, uint64_t a_cols, const void *b_base,
              uint64_t b_rows, uint64_t b_cols, uint64_t o_rows, uint64_t o_cols, GemmParams p,
              cudaStream_t s, const char *what) {
+  return run_gemm_out<MODE>(N, a_base, a_rows, a_cols, b_base, b_rows, b_cols, p.out, o_rows,
+                            o_cols, p, s, what);
+}
+
+// As run_gemm, with the output tensor map built over o_base (p.out may be nullptr when
+// the epilogue stores no output tile).
+template <int MODE>
+int run_gemm_out(int N, const void *a_base, uint64_t a_rows, uint64_t a_cols, const void *b_base,
+                 uint64_t b_rows, uint64_t b_cols, const void *o_base, uint64_t o_rows,
+                 uint64_t o_cols, GemmParams p, cudaStream_t s, const char *what) {
   using Tr = Traits<MODE>;
   const bool pair = use_pair<MODE>();
   const int BN = (MODE == kGateUp || N % 256 == 0) ? 256 : 128;
@@ -997,7 +1034,7 @@ int run_gemm(int N, const void *a_base, uint64_t a_rows, uint64_t a_cols, const 
                        : make_map(&mb, b_base, b_rows, b_cols, BK, b_box_rows, what)))
     return st;
   CUtensorMap mo;  // the epilogue's output, in 32 x 32 chunks
-  if ((st = make_map(&mo, p.out, o_rows, o_cols, 32, 32, what, CU_TENSOR_MAP_SWIZZLE_64B))) return st;
+  if ((st = make_map(&mo, o_base, o_rows, o_cols, 32, 32, what, CU_TENSOR_MAP_SWIZZLE_64B))) return st;
   if (pair) {
     if constexpr (MODE == kGateUp || MODE == kWgradGateUp) {
       if (gather)
@@ -1034,6 +1071,48 @@ __global__ void wait_timeout_selftest_kernel(uint64_t limit_ns) {
   tc::fence_mbar_init();
   abort_word = 0;
   if (!tc::mbar_wait(b, 0, limit_ns, &abort_word)) dev_flag(&g_dev_err, MOE_DEV_WAIT_TIMEOUT);
+}
+
+// ---- combine in the down GEMM's epilogue: helpers ----
+// row_token[r] = -1 for every grouped row (padding rows keep it).
+__global__ void combine_rows_fill_kernel(int32_t *__restrict__ row_token, int64_t R) {
+  for (int64_t r = blockIdx.x * int64_t(blockDim.x) + threadIdx.x; r < R;
+       r += int64_t(gridDim.x) * blockDim.x)
+    row_token[r] = -1;
+}
+// The row of assignment a = t*k + j gets token t and weight topk_gate[a].
+__global__ void combine_rows_scatter_kernel(const int32_t *__restrict__ row_of_assignment,
+                                            const float *__restrict__ topk_gate, int64_t A, int k,
+                                            int64_t R, int32_t *__restrict__ row_token,
+                                            float *__restrict__ row_gate) {
+  for (int64_t a = blockIdx.x * int64_t(blockDim.x) + threadIdx.x; a < A;
+       a += int64_t(gridDim.x) * blockDim.x) {
+    const int32_t r = row_of_assignment[a];
+    if (r >= 0 && r < R) {
+      row_token[r] = int32_t(a / k);
+      row_gate[r] = topk_gate[a];
+    } else {
+      dev_flag(&g_dev_err, MOE_DEV_ROWS_OVERFLOW);
+    }
+  }
+}
+__global__ void zero_f32x4_kernel(float4 *__restrict__ p, int64_t n4) {
+  for (int64_t i = blockIdx.x * int64_t(blockDim.x) + threadIdx.x; i < n4;
+       i += int64_t(gridDim.x) * blockDim.x)
+    p[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+}
+// y = bf16(y_acc), 8 elements per thread (n8 = T*d/8).
+__global__ void f32_to_bf16_kernel(const float4 *__restrict__ src, uint4 *__restrict__ dst,
+                                   int64_t n8) {
+  for (int64_t i = blockIdx.x * int64_t(blockDim.x) + threadIdx.x; i < n8;
+       i += int64_t(gridDim.x) * blockDim.x) {
+    const float4 a = src[2 * i], b = src[2 * i + 1];
+    dst[i] = make_uint4(pack_bf16x2(a.x, a.y), pack_bf16x2(a.z, a.w), pack_bf16x2(b.x, b.y),
+                        pack_bf16x2(b.z, b.w));
+  }
+}
+int grid_for(int64_t n) {
+  return int(std::max<int64_t>(1, std::min<int64_t>((n + 255) / 256, int64_t(moe::num_sms()) * 8)));
 }
 
 }  // namespace
@@ -1084,6 +1163,73 @@ int moe_grouped_ffn_fwd(const uint16_t *x_perm, const int32_t *group_offsets, in
   q.out = out_perm;
   return run_gemm<kDown>(d, h, R, F, w_down, uint64_t(E) * d, F, R, d, q, s,
                          "moe_grouped_ffn_fwd: down GEMM");
+}
+
+int moe_grouped_ffn_fwd_combine(const uint16_t *x_perm, const int32_t *group_offsets, int E, int d,
+                                int F, int64_t rows_cap, const uint16_t *w_gate_up,
+                                const uint16_t *w_down, const int32_t *row_of_assignment,
+                                const float *topk_gate, int T, int k, uint16_t *ab_saved,
+                                uint16_t *h, uint16_t *out_perm, float *y_acc, uint16_t *y,
+                                void *ws, size_t ws_bytes, moe_stream_t stream) {
+  const char *fn = "moe_grouped_ffn_fwd_combine";
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if (int st = check_common(E, d, F, rows_cap, fn)) return st;
+  if (T < 0 || k < 1 || k > 8 || k > E) return moe::set_error(MOE_ERR_ARG, "%s: T=%d k=%d", fn, T, k);
+  if (rows_cap < moe_perm_rows_max(T, k, E)) return moe::set_error(MOE_ERR_ARG, "%s: rows_cap too small", fn);
+  const void *ptrs[] = {x_perm, group_offsets, w_gate_up, w_down, ab_saved, h, ws};
+  for (const void *q : ptrs)
+    if (!q || !moe::aligned16(q)) return moe::set_error(MOE_ERR_ARG, "%s: null or unaligned pointer", fn);
+  if (out_perm && !moe::aligned16(out_perm)) return moe::set_error(MOE_ERR_ARG, "%s: unaligned out_perm", fn);
+  if (T > 0 && (!row_of_assignment || !topk_gate || !y_acc || !y || !moe::aligned16(y_acc) ||
+                !moe::aligned16(y)))
+    return moe::set_error(MOE_ERR_ARG, "%s: null or unaligned combine argument", fn);
+  const moe::WsLayout L = moe::ws_layout(T, d, E, k, F);
+  if (ws_bytes < L.total) return moe::set_error(MOE_ERR_WORKSPACE, "%s: workspace", fn);
+  const uint64_t R = uint64_t(rows_cap);
+  const int64_t Rr = moe_perm_rows_max(T, k, E);  // rows the layout can use
+  int32_t *row_token = reinterpret_cast<int32_t *>(static_cast<char *>(ws) + L.combine_rows);
+  float *row_gate = reinterpret_cast<float *>(row_token + Rr);
+  GemmParams p{};
+  p.group_offsets = group_offsets;
+  p.E = E; p.d = d; p.F = F;
+  p.nkb = d / BK;
+  p.out = h;
+  p.out2 = ab_saved;
+  if (int st = run_gemm<kGateUp>(2 * F, x_perm, R, d, w_gate_up, uint64_t(E) * 2 * F, d, R, F, p,
+                                 s, "moe_grouped_ffn_fwd_combine: gate/up GEMM"))
+    return st;
+  const int64_t A = int64_t(T) * k, n = int64_t(T) * d;
+  if (T > 0) {
+    MOE_LAUNCH("combine_rows_fill", s, combine_rows_fill_kernel<<<grid_for(Rr), 256, 0, s>>>(row_token, Rr));
+    if (int st = moe::launch_status("moe_grouped_ffn_fwd_combine: row fill")) return st;
+    MOE_LAUNCH("combine_rows_scatter", s, combine_rows_scatter_kernel<<<grid_for(A), 256, 0, s>>>(
+                                              row_of_assignment, topk_gate, A, k, Rr, row_token, row_gate));
+    if (int st = moe::launch_status("moe_grouped_ffn_fwd_combine: row scatter")) return st;
+    MOE_LAUNCH("zero_y_acc", s, zero_f32x4_kernel<<<grid_for(n / 4), 256, 0, s>>>(
+                                    reinterpret_cast<float4 *>(y_acc), n / 4));
+    if (int st = moe::launch_status("moe_grouped_ffn_fwd_combine: zero")) return st;
+  }
+  // O = H W_down^T, combined into y_acc by the epilogue (O itself stored only if asked)
+  GemmParams q{};
+  q.group_offsets = group_offsets;
+  q.E = E; q.d = d; q.F = F;
+  q.nkb = F / BK;
+  q.out = out_perm;
+  if (T > 0) {
+    q.y_acc = y_acc;
+    q.row_token = row_token;
+    q.row_gate = row_gate;
+  }
+  // without out_perm the output map is built over h (never stored to)
+  void *o_base = out_perm ? static_cast<void *>(out_perm) : static_cast<void *>(h);
+  const uint64_t o_cols = out_perm ? uint64_t(d) : uint64_t(F);
+  if (int st = run_gemm_out<kDown>(d, h, R, F, w_down, uint64_t(E) * d, F, o_base, R, o_cols, q, s,
+                                   "moe_grouped_ffn_fwd_combine: down GEMM"))
+    return st;
+  if (T == 0) return MOE_OK;
+  MOE_LAUNCH("combine_y_bf16", s, f32_to_bf16_kernel<<<grid_for(n / 8), 256, 0, s>>>(
+                                      reinterpret_cast<const float4 *>(y_acc), reinterpret_cast<uint4 *>(y), n / 8));
+  return moe::launch_status("moe_grouped_ffn_fwd_combine: bf16 output");
 }
 
 int moe_grouped_ffn_fwd_gather(const uint16_t *x, const int32_t *token_of_row, int T,

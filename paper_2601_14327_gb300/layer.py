@@ -34,13 +34,20 @@ class MoELayerBuffers:
     GEMMs' 4-row TMA gathers (moe_permute_map and the *_gather calls), so X_perm is not
     allocated; the results are identical, but on GB300 the gathers make the two GEMMs
     that read X_perm about 3.3x slower (32 gathers of 4 x 128 bytes per 128-row k-block
-    against one tile load), far more than the separate gather pass costs."""
+    against one tile load), far more than the separate gather pass costs.
+
+    fused_combine=True: the combine runs in the down GEMM's epilogue
+    (moe_grouped_ffn_fwd_combine, fp32 atomics into y_acc; the last bits of y can
+    change from run to run); O is then stored only when a backward follows."""
 
     def __init__(self, shape: LayerShape, device="cuda", backward: bool = True,
-                 gather: bool = False):
+                 gather: bool = False, fused_combine: bool = False):
         s = shape
         self.shape = s
         self.gather = gather
+        self.fused_combine = fused_combine
+        if fused_combine and gather:
+            raise ValueError("fused_combine reads X_perm: use it with gather=False")
         self.x = None  # the forward's input, kept for the backward
         R = s.rows_cap
         dev = torch.device(device)
@@ -62,7 +69,9 @@ class MoELayerBuffers:
             self.x_perm = torch.empty(R, s.d, dtype=bf16, device=dev)
         self.ab = torch.empty(R, 2 * s.F, dtype=bf16, device=dev)
         self.h = torch.empty(R, s.F, dtype=bf16, device=dev)
-        self.out_perm = torch.empty(R, s.d, dtype=bf16, device=dev)
+        self.out_perm = (torch.empty(R, s.d, dtype=bf16, device=dev)
+                         if backward or not fused_combine else None)
+        self.y_acc = torch.empty(s.T, s.d, dtype=f32, device=dev) if fused_combine else None
         self.y = torch.empty(s.T, s.d, dtype=bf16, device=dev)
         if backward:
             self.d_out_perm = torch.empty(R, s.d, dtype=bf16, device=dev)
@@ -89,7 +98,8 @@ def route(b: MoELayerBuffers, x, w_router, bias, active_mask=None, logits_in=Non
 
 def forward(b: MoELayerBuffers, x, w_router, bias, w_gate_up, w_down, active_mask=None,
             logits_in=None, keep_logits: bool = False, stream=None):
-    """route -> permute -> grouped SwiGLU FFN -> combine. Returns b.y."""
+    """route -> permute -> grouped SwiGLU FFN -> combine (in the down GEMM's epilogue
+    when b.fused_combine). Returns b.y."""
     s = b.shape
     R = s.rows_cap
     route(b, x, w_router, bias, active_mask, logits_in, keep_logits, stream)
@@ -104,6 +114,12 @@ def forward(b: MoELayerBuffers, x, w_router, bias, w_gate_up, w_down, active_mas
     else:
         L.moe_permute(x, b.topk_idx, b.counts, s.T, s.d, s.E, s.k, R, b.group_offsets,
                       b.group_counts, b.row_of_assignment, b.x_perm, b.ws, b.ws_bytes, stream)
+        if b.fused_combine:
+            L.moe_grouped_ffn_fwd_combine(b.x_perm, b.group_offsets, s.E, s.d, s.F, R, w_gate_up,
+                                          w_down, b.row_of_assignment, b.topk_gate, s.T, s.k,
+                                          b.ab, b.h, b.out_perm, b.y_acc, b.y, b.ws, b.ws_bytes,
+                                          stream)
+            return b.y
         L.moe_grouped_ffn_fwd(b.x_perm, b.group_offsets, s.E, s.d, s.F, R, w_gate_up, w_down,
                               b.ab, b.h, b.out_perm, b.ws, b.ws_bytes, stream)
     L.moe_unpermute_combine(b.out_perm, b.row_of_assignment, b.topk_gate, s.T, s.d, s.k, b.y,

@@ -42,13 +42,14 @@ def oracle_inputs(inp):
     return {n: (v.double().numpy() if v.is_floating_point() else v.numpy()) for n, v in inp.items()}
 
 
-def run_gpu_layer(inp, E, k, mask=None, logits_in=None, backward=True):
+def run_gpu_layer(inp, E, k, mask=None, logits_in=None, backward=True, fused_combine=False):
     """Full step through the C ABI; returns the buffers object."""
     T, d = inp["x"].shape
     F = inp["w_down"].shape[2]
     dev = "cuda"
     g = {n: v.to(dev) for n, v in inp.items()}
-    b = layer.MoELayerBuffers(layer.LayerShape(T, d, E, k, F), dev, backward=backward)
+    b = layer.MoELayerBuffers(layer.LayerShape(T, d, E, k, F), dev, backward=backward,
+                              fused_combine=fused_combine)
     m = None if mask is None else torch.as_tensor(mask, dtype=torch.uint8).to(dev)
     li = None if logits_in is None else torch.as_tensor(logits_in, dtype=torch.float32).to(dev)
     layer.forward(b, g["x"], g["w_router"], g["bias"], g["w_gate_up"], g["w_down"], m, li,

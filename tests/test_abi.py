@@ -171,6 +171,23 @@ def test_new_entry_points_validate_before_launch(lib):
     with pytest.raises(L.MoEError) as e:  # router backward: workspace too small
         L.moe_route_bwd(16, 16, 16, 16, 10, 128, 8, 2, 16, 16, 16, 4, stream=0)
     assert e.value.status == -6
+    Rf = L.moe_perm_rows_max(10, 2, 8)
+    with pytest.raises(L.MoEError) as e:  # fused combine: k above E
+        L.moe_grouped_ffn_fwd_combine(16, 16, 8, 128, 128, Rf, 16, 16, 16, 16, 10, 9, 16, 16,
+                                      16, 16, 16, 16, 1 << 20, stream=0)
+    assert e.value.status == -1
+    with pytest.raises(L.MoEError) as e:  # fused combine: no y_acc with tokens present
+        L.moe_grouped_ffn_fwd_combine(16, 16, 8, 128, 128, Rf, 16, 16, 16, 16, 10, 2, 16, 16,
+                                      None, None, 16, 16, 1 << 20, stream=0)
+    assert e.value.status == -1
+    with pytest.raises(L.MoEError) as e:  # fused combine: rows_cap below T*k + 128*E
+        L.moe_grouped_ffn_fwd_combine(16, 16, 8, 128, 128, 200, 16, 16, 16, 16, 10, 2, 16, 16,
+                                      16, 16, 16, 16, 1 << 20, stream=0)
+    assert e.value.status == -1
+    with pytest.raises(L.MoEError) as e:  # fused combine: workspace too small
+        L.moe_grouped_ffn_fwd_combine(16, 16, 8, 128, 128, Rf, 16, 16, 16, 16, 10, 2, 16, 16,
+                                      16, 16, 16, 16, 4, stream=0)
+    assert e.value.status == -6
     with pytest.raises(L.MoEError) as e:  # combine backward with neither output
         L.moe_unpermute_combine_bwd(16, 16, 16, 16, 16, 16, 10, 128, 8, 2, None, None, stream=0)
     assert e.value.status == -1

@@ -506,3 +506,69 @@ def test_layer_is_deterministic_and_stream_layout_independent():
     for other in outs[1:]:
         for n in names:
             assert torch.equal(getattr(outs[0], n), getattr(other, n)), n
+
+
+FUSED_COMBINE_CASES = [
+    # T, d, E, k, F, bias, n_masked
+    (512, 256, 16, 2, 512, "none", 0),
+    (1, 256, 4, 2, 256, "zipf", 0),
+    (1500, 384, 12, 4, 640, "zipf", 3),       # BN = 128 down GEMM, empty groups
+    (700, 512, 8, 8, 256, "zipf", 0),
+    (3000, 256, 256, 8, 256, "zipf", 40),
+]
+
+
+@pytest.mark.parametrize("T,d,E,k,F,bias,n_masked", FUSED_COMBINE_CASES)
+def test_fused_combine_against_oracle_and_unfused(T, d, E, k, F, bias, n_masked):
+    """Combine in the down GEMM's epilogue: y against the oracle, against the unfused
+    path within its rounding, O and every gradient bit for bit as unfused."""
+    inp = case_inputs(T, d, E, k, F, bias=bias, seed=T + 3)
+    o = oracle_inputs(inp)
+    mask = None
+    if n_masked:
+        mask = np.ones(E, np.uint8)
+        mask[np.random.default_rng(2).permutation(E)[:n_masked]] = 0
+    z = O.router_logits(o["x"], o["w_router"], o["bias"])
+    ref = O.moe_layer(o["x"], o["w_router"], o["bias"], mask, k, o["w_gate_up"], o["w_down"],
+                      logits32=z)
+    b0 = run_gpu_layer(inp, E, k, mask=mask, logits_in=z)
+    b1 = run_gpu_layer(inp, E, k, mask=mask, logits_in=z, fused_combine=True)
+    b2 = run_gpu_layer(inp, E, k, mask=mask, logits_in=z, backward=False, fused_combine=True)
+    assert b2.out_perm is None
+    assert_close("y", to_np(b1.y), ref["y"])
+    # the unfused combine sums gate * bf16(O) in fp32 and rounds once; the fused one sums
+    # gate * O before O's bf16 rounding: at most u = 2^-8 (bf16's unit roundoff, 8-bit
+    # significand) of sum |gate * O| apart, plus each side's final rounding (u of |y|) and
+    # the fp32 sums' own error
+    row = b0.row_of_assignment.cpu().numpy()
+    g = b0.topk_gate.cpu().numpy().astype(np.float64)
+    absgo = (np.abs(to_np(b0.out_perm).astype(np.float64))[row] * g[:, :, None]).sum(axis=1)
+    y0 = to_np(b0.y).astype(np.float64)
+    for b in (b1, b2):
+        y = to_np(b.y).astype(np.float64)
+        bound = 2.0 ** -8 * (absgo + np.abs(y0) + np.abs(y)) + 2.0 ** -20 * absgo + 1e-30
+        assert (np.abs(y - y0) <= bound).all(), float(np.max(np.abs(y - y0) / bound))
+    # same [A|B], H and O on every real row, same backward
+    flat = torch.from_numpy(row.reshape(-1).astype(np.int64)).cuda()
+    for name in ["h", "out_perm"]:
+        assert torch.equal(getattr(b0, name)[flat], getattr(b1, name)[flat]), name
+    assert torch.equal(b0.h[flat], b2.h[flat])
+    assert (unblock_ab(to_np(b0.ab), F)[row.reshape(-1)] ==
+            unblock_ab(to_np(b1.ab), F)[row.reshape(-1)]).all()
+    for name in ["dx", "dw_gate_up", "dw_down", "dw_router", "d_logits", "d_gate"]:
+        assert torch.equal(getattr(b0, name), getattr(b1, name)), name
+
+
+def test_fused_combine_without_tokens():
+    dev = "cuda"
+    s = layer.LayerShape(0, 256, 8, 2, 256)
+    b = layer.MoELayerBuffers(s, dev, backward=False, fused_combine=True)
+    gen = torch.Generator(device=dev).manual_seed(3)
+    wgu = (torch.randn(8, 512, 256, generator=gen, device=dev) * 0.02).to(torch.bfloat16)
+    wd = (torch.randn(8, 256, 256, generator=gen, device=dev) * 0.02).to(torch.bfloat16)
+    x = torch.empty(0, 256, dtype=torch.bfloat16, device=dev)
+    w = torch.randn(256, 8, generator=gen, device=dev)
+    layer.forward(b, x, w, None, wgu, wd)
+    torch.cuda.synchronize()
+    assert b.y.shape == (0, 256) and (b.counts == 0).all()
+

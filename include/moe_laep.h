@@ -10,8 +10,13 @@
  *   moe_permute            contiguous per-expert groups of token rows
  *   moe_grouped_ffn_fwd    grouped SwiGLU expert FFN (tcgen05 / TMEM / TMA)
  *   moe_unpermute_combine  gate-weighted combine back to token order
- * and the backward companions moe_unpermute_combine_bwd, moe_grouped_ffn_bwd,
- * moe_route_bwd, moe_permute_bwd.
+ * and the backward companions moe_unpermute_combine_bwd, moe_grouped_ffn_bwd
+ * (or its halves moe_grouped_ffn_bwd_dgrad / _wgrad), moe_route_bwd,
+ * moe_permute_bwd. Fused variants, same results, slower on GB300 and so not
+ * the default: moe_permute_map with the *_gather GEMM entry points (X_perm read
+ * from x by TMA gathers) and moe_grouped_ffn_fwd_combine (the combine in the
+ * down GEMM's epilogue). Host-side LAEP: laep_prune_mask, laep_prune_layers,
+ * laep_layer_alpha, laep_rearrange.
  *
  * Conventions (all entry points):
  *  - Pointers are DEVICE pointers owned by the caller unless marked "host".

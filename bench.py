@@ -484,21 +484,24 @@ def run_ours(args):
 
     # end to end through the public API: every step uploads its inputs from pinned host
     # memory and downloads its results (x, dy in; y, dx out; forward-only workloads: x in,
-    # y out). An upload stream, a download stream and two device slots pipeline the copies
-    # with the compute:
-    # step i+2's inputs and step i's results move while step i+1 computes; the first
-    # uploads and the last downloads are inside the timed region.
+    # y out). An upload stream, a download stream and NSLOT device slots pipeline the
+    # copies with the compute: step i+NSLOT's inputs and step i's results move while the
+    # steps in between compute, so a copy that stalls for a while (host-side stalls of
+    # ~20 ms were seen now and then on the Grace host) does not stop the compute stream;
+    # the first uploads and the last downloads are inside the timed region.
     e2e = None
     if not args.no_e2e:
+        NSLOT = 4
         in_names = ["x", "dy"] if wl.backward else ["x"]
         out_names = ["y", "dx"] if wl.backward else ["y"]
         host_in = {n: wl.inp[n].cpu().pin_memory() for n in in_names}
-        dev_in = [{n: torch.empty_like(wl.inp[n]) for n in in_names} for _ in range(2)]
-        dev_out = [{n: getattr(wl.bufs, n) for n in out_names},  # results alternate slots
-                   {n: torch.empty_like(getattr(wl.bufs, n)) for n in out_names}]
+        dev_in = [{n: torch.empty_like(wl.inp[n]) for n in in_names} for _ in range(NSLOT)]
+        dev_out = ([{n: getattr(wl.bufs, n) for n in out_names}] +  # results rotate slots
+                   [{n: torch.empty_like(getattr(wl.bufs, n)) for n in out_names}
+                    for _ in range(NSLOT - 1)])
         host_out = [{n: torch.empty_like(dev_out[0][n], device="cpu").pin_memory()
-                     for n in out_names} for _ in range(2)]
-        for j in range(2):
+                     for n in out_names} for _ in range(NSLOT)]
+        for j in range(NSLOT):
             for n in in_names:
                 dev_in[j][n].copy_(host_in[n])
 
@@ -510,15 +513,18 @@ def run_ours(args):
             return dev_in[j]["x"], dev_in[j].get("dy")
 
         graphs = []
-        for j in range(2):
+        for j in range(NSLOT):
             use_slot(j)
             wl.eager_step(*inputs(j))
             graphs.append(wl.make_graph(*inputs(j)) if args.graph else None)
         # uploads and downloads on separate streams: the two directions overlap
         up, down = torch.cuda.Stream(), torch.cuda.Stream()
-        in_ready = [torch.cuda.Event() for _ in range(2)]
-        step_done = [torch.cuda.Event() for _ in range(2)]
-        out_copied = [torch.cuda.Event() for _ in range(2)]
+        in_ready = [torch.cuda.Event() for _ in range(NSLOT)]
+        step_done = [torch.cuda.Event() for _ in range(NSLOT)]
+        out_copied = [torch.cuda.Event() for _ in range(NSLOT)]
+        for j in range(NSLOT):  # the copy path warmed up like the steps (untimed)
+            for n in out_names:
+                host_out[j][n].copy_(dev_out[j][n])
 
         def upload(j):
             with torch.cuda.stream(up):
@@ -526,11 +532,11 @@ def run_ours(args):
                     dev_in[j][n].copy_(host_in[n], non_blocking=True)
                 in_ready[j].record(up)
 
-        def run(i):
-            j = i % 2
+        def run(i, n):
+            j = i % NSLOT
             stream.wait_event(in_ready[j])
-            if i >= 2:
-                stream.wait_event(out_copied[j])  # results of step i-2 have left slot j
+            if i >= NSLOT:
+                stream.wait_event(out_copied[j])  # results of step i-NSLOT have left slot j
             if graphs[j] is not None:
                 graphs[j].replay()
             else:
@@ -539,26 +545,33 @@ def run_ours(args):
             step_done[j].record(stream)
             with torch.cuda.stream(down):
                 down.wait_event(step_done[j])
-                for n in out_names:
-                    host_out[j][n].copy_(dev_out[j][n], non_blocking=True)
+                for name in out_names:
+                    host_out[j][name].copy_(dev_out[j][name], non_blocking=True)
                 out_copied[j].record(down)
-            if i + 2 < args.steps:
+            if i + NSLOT < n:
                 up.wait_event(step_done[j])  # step i no longer reads slot j's inputs
                 upload(j)
 
+        def pipeline(n):
+            """n steps, each with its uploads and downloads; returns on the host at once."""
+            start = stream.record_event()
+            up.wait_event(start)
+            down.wait_event(start)
+            for j in range(min(NSLOT, n)):
+                upload(j)
+            for i in range(n):
+                run(i, n)
+            for j in range(min(NSLOT, n)):
+                stream.wait_event(out_copied[j])
+
+        # untimed warm-up of the whole pipeline, copies included: the host link's first
+        # copies after an idle spell were seen to take 15-25 ms instead of ~1.4 ms
+        pipeline(max(args.warmup, 1))
         ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         barrier(world)
         torch.cuda.synchronize()
         ev0.record(stream)
-        up.wait_event(ev0)
-        down.wait_event(ev0)
-        upload(0)
-        if args.steps > 1:
-            upload(1)
-        for i in range(args.steps):
-            run(i)
-        for j in range(min(2, args.steps)):
-            stream.wait_event(out_copied[j])
+        pipeline(args.steps)
         ev1.record(stream)
         torch.cuda.synchronize()
         barrier(world)
@@ -570,8 +583,8 @@ def run_ours(args):
                "h2d_bytes_per_step": nb(host_in.values()),
                "d2h_bytes_per_step": nb(host_out[0].values()),
                "note": f"{', '.join(in_names)} uploaded and {', '.join(out_names)} downloaded "
-                       "every step (an upload and a download stream), overlapped with the "
-                       "neighbouring steps' compute"}
+                       f"every step (an upload and a download stream, {NSLOT} device slots), "
+                       "overlapped with the neighbouring steps' compute"}
 
     # pruned vs unpruned, after the end-to-end run (it allocates a second workload)
     laep = None

@@ -12,7 +12,9 @@ same buffers and calls), on outputs the oracle can evaluate one by one:
   (heaviest, median, lightest non-empty) and exact zeros for empty experts;
 - the router gradient through a property that holds at any size: the softmax
   Jacobian makes every token's d_logits sum to zero, so the columns of
-  dw_router sum to zero as well.
+  dw_router sum to zero as well; and sampled feature rows of dw_router (plus
+  every d_logits entry) against the oracle's router backward evaluated on the
+  GPU's own routing, gates and d_gate.
 """
 import numpy as np
 import pytest
@@ -155,5 +157,16 @@ def test_full_size_sampled_parity(cfg_id):
     dwr = b.dw_router.cpu().numpy().astype(np.float64)
     col_scale = np.abs(x).T @ np.abs(dl).sum(1)  # bound on |sum_e dw_router[i, e]|
     assert (np.abs(dwr.sum(1)) <= 1e-4 * col_scale + 1e-6).all()
+    # sampled feature rows of dw_router against the oracle's router backward, from the
+    # GPU's own routing, gates and d_gate (so only the arithmetic is compared): fp32
+    # softmax backward and fp32 accumulation over T tokens
+    feats = np.unique(np.concatenate([[0, d - 1], rng.choice(d, size=14, replace=False)]))
+    dz_ref, dw_ref = O.router_backward(x[:, feats], gidx, g, dg, E)
+    zscale = np.abs(g) * (np.abs(dg) + np.abs(g * dg).sum(1, keepdims=True))
+    assert (np.abs(dl - dz_ref) <= 2e-6 * zscale + 1e-30).all()
+    dzs = np.zeros((T, E))
+    np.put_along_axis(dzs, gidx.astype(np.int64), zscale, axis=1)
+    scale = np.abs(x[:, feats]).T @ dzs
+    assert (np.abs(dwr[feats] - dw_ref) <= 1e-5 * scale + 1e-30).all()
     del wl
     torch.cuda.empty_cache()

@@ -572,3 +572,35 @@ def test_fused_combine_without_tokens():
     torch.cuda.synchronize()
     assert b.y.shape == (0, 256) and (b.counts == 0).all()
 
+
+
+def test_graph_replay_of_the_step_equals_eager():
+    """bench.py times replays of a CUDA graph of the whole step (both streams): the replay
+    on new inputs gives the same bits as an eager step on those inputs."""
+    T, d, E, k, F = 1500, 256, 16, 4, 256
+    dev = "cuda"
+    a = {n: v.to(dev) for n, v in case_inputs(T, d, E, k, F, seed=5).items()}
+    c = {n: v.to(dev) for n, v in case_inputs(T, d, E, k, F, seed=6).items()}
+    shape = layer.LayerShape(T, d, E, k, F)
+
+    def step(b, x, dy):
+        layer.forward(b, x, a["w_router"], a["bias"], a["w_gate_up"], a["w_down"])
+        layer.backward(b, dy, a["w_router"], a["w_gate_up"], a["w_down"])
+
+    bg = layer.MoELayerBuffers(shape, dev, backward=True)
+    x_in, dy_in = a["x"].clone(), a["dy"].clone()
+    step(bg, x_in, dy_in)  # eager warm-up (one-time setup outside the capture)
+    torch.cuda.synchronize()
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph):
+        step(bg, x_in, dy_in)
+    x_in.copy_(c["x"])
+    dy_in.copy_(c["dy"])
+    graph.replay()
+    torch.cuda.synchronize()
+    be = layer.MoELayerBuffers(shape, dev, backward=True)
+    step(be, c["x"], c["dy"])
+    torch.cuda.synchronize()
+    for n in ["topk_idx", "topk_gate", "counts", "row_of_assignment", "y", "dx", "dw_gate_up",
+              "dw_down", "dw_router", "d_logits"]:
+        assert torch.equal(getattr(bg, n), getattr(be, n)), n

@@ -42,7 +42,8 @@ __global__ void zero_i32_kernel(int32_t *p, int n) {
 constexpr int kRtBM = 128;       // tokens per tile (TMEM lanes)
 constexpr int kRtBK = 64;        // k-block: 64 bf16 = one 128-byte swizzle row
 constexpr int kRtThreads = 128;
-constexpr int kRtTargetCtas = 152;
+constexpr int kRtSms = 152;           // SMs of a GB300: the splits aim to fill them
+constexpr int kRtSmemPerSm = 233472;  // shared memory per SM (228 KB)
 constexpr int kRtMaxSplits = 8;
 constexpr uint32_t kRtABytes = kRtBM * kRtBK * 2;
 constexpr int kRtMaxSmem = 232448;  // opt-in dynamic shared memory per CTA
@@ -63,19 +64,32 @@ struct RouteTcParams {
 int route_tc_np(int E) { return (E + 15) / 16 * 16; }
 uint32_t route_tc_tmem_cols(int NP) { return NP <= 32 ? 32u : (NP <= 64 ? 64u : (NP <= 128 ? 128u : 256u)); }
 uint32_t route_tc_stage_bytes(int NP) { return kRtABytes + 3u * uint32_t(NP) * 128u; }
-int route_tc_stages(int NP) {
-  return std::min(8, int((kRtMaxSmem - 2048) / route_tc_stage_bytes(NP)));
-}
 size_t route_tc_smem(int NP, int stages) {
   return 1024 + size_t(stages) * route_tc_stage_bytes(NP) + size_t(2 * stages + 1) * 8 + 16;
 }
-// Splits of the reduction: enough CTAs to cover the SMs when the M rows (tokens for
-// the logits, d_model for the weight gradient) give few tiles. A function of
-// (M, K) alone, so the workspace size is too. K > 0.
-void route_tc_split(int M, int K, int *splits, int *kb_per_split) {
+// Two CTAs per SM with a ring of at least two stages each where that fits (more
+// independent x streams per SM: measured faster than one CTA with a deeper ring), else
+// one CTA per SM with the deepest ring that fits.
+bool route_tc_two_per_sm(int NP) {
+  return 2 * (route_tc_smem(NP, 2) + 1024) <= size_t(kRtSmemPerSm);
+}
+int route_tc_stages(int NP) {
+  int st = 2;
+  if (route_tc_two_per_sm(NP)) {
+    while (st < 8 && 2 * (route_tc_smem(NP, st + 1) + 1024) <= size_t(kRtSmemPerSm)) ++st;
+  } else {
+    st = int((kRtMaxSmem - 2048) / route_tc_stage_bytes(NP));
+  }
+  return std::min(8, st);
+}
+// Splits of the reduction: enough CTAs to fill the SMs' CTA slots when the M rows (tokens
+// for the logits, d_model for the weight gradient) give few tiles. A function of
+// (M, K, NP) alone, so the workspace size is too. K > 0.
+void route_tc_split(int M, int K, int NP, int *splits, int *kb_per_split) {
   const int tiles = std::max(1, (M + kRtBM - 1) / kRtBM);
   const int nkb = (K + kRtBK - 1) / kRtBK;
-  int s = std::max(1, std::min({kRtTargetCtas / tiles, kRtMaxSplits, nkb}));
+  const int target = kRtSms * (route_tc_two_per_sm(NP) ? 2 : 1);
+  int s = std::max(1, std::min({target / tiles, kRtMaxSplits, nkb}));
   const int per = (nkb + s - 1) / s;
   *kb_per_split = per;
   *splits = (nkb + per - 1) / per;  // every split gets at least one k-block
@@ -459,7 +473,7 @@ int launch_route_tc(const uint16_t *x, const float *w, int T, int d, int E, int 
   if ((st = moe::make_map(&mw, w3, uint64_t(3 * NP), uint64_t(d), kRtBK, uint32_t(NP), "router w")))
     return st;
   int splits = 1, per = 1;
-  route_tc_split(T, d, &splits, &per);
+  route_tc_split(T, d, route_tc_np(E), &splits, &per);
   RouteTcParams p;
   p.M = T;
   p.kb_per_split = per;
@@ -496,7 +510,7 @@ MOE_DEV_ERR_DEFINE_READER(route_dev_error)
 size_t route_partial_bytes(int T, int d, int E) {
   if (T <= 0) return 0;
   int splits = 1, per = 1;
-  route_tc_split(T, d, &splits, &per);
+  route_tc_split(T, d, route_tc_np(E), &splits, &per);
   return size_t(splits) * size_t(T) * size_t(padded_experts(E)) * 4;
 }
 size_t route_w3_bytes(int d, int E) { return size_t(3) * route_tc_np(E) * size_t(d) * 2; }
@@ -506,7 +520,7 @@ size_t route_dz3_bytes(int T, int E) {
 size_t route_dw_partial_bytes(int T, int d, int E) {
   if (T <= 0) return 0;
   int splits = 1, per = 1;
-  route_tc_split(d, route_tokens_padded(T), &splits, &per);
+  route_tc_split(d, route_tokens_padded(T), route_tc_np(E), &splits, &per);
   return size_t(splits) * size_t(d) * size_t(route_dw_stride(E)) * 4;
 }
 }  // namespace moe
@@ -586,7 +600,7 @@ int launch_route_dw(const uint16_t *x, const uint16_t *dz3, int T, int d, int E,
   if ((st = moe::make_map(&mz, dz3, uint64_t(3 * NP), uint64_t(Tp), kRtBK, uint32_t(NP), "router bwd dz")))
     return st;
   int splits = 1, per = 1;
-  route_tc_split(d, Tp, &splits, &per);
+  route_tc_split(d, Tp, NP, &splits, &per);
   RouteTcParams p;
   p.M = d;
   p.kb_per_split = per;

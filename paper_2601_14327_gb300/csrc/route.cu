@@ -17,10 +17,6 @@ namespace {
 constexpr int kRouteThreads = 256;
 int padded_experts(int E) { return E <= 64 ? 64 : (E <= 128 ? 128 : (E <= 192 ? 192 : 256)); }
 
-__device__ __forceinline__ bool better(float v, int e, float bv, int be) {
-  return v > bv || (v == bv && e < be);
-}
-
 __global__ void zero_i32_kernel(int32_t *p, int n) {
   for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < n; i += gridDim.x * blockDim.x) p[i] = 0;
 }
@@ -286,7 +282,7 @@ __global__ void __launch_bounds__(kRtThreads, 1)
 // (ties to the lower index), softmax over the selected logits, per-expert
 // histogram (shared per block, then one global add per expert and block).
 template <int NE>
-__global__ void __launch_bounds__(kRouteThreads) route_topk_kernel(
+__global__ void __launch_bounds__(kRouteThreads, 4) route_topk_kernel(
     const float *__restrict__ partial, int splits, const float *__restrict__ logits_in,
     const float *__restrict__ bias, const uint8_t *__restrict__ active_mask, int T, int E, int k,
     float *__restrict__ logits_out, int32_t *__restrict__ topk_idx, float *__restrict__ topk_gate,
@@ -313,27 +309,35 @@ __global__ void __launch_bounds__(kRouteThreads) route_topk_kernel(
       v[j] = z;
       if (logits_out != nullptr && e < E) logits_out[size_t(t) * E + e] = z;
     }
-    unsigned taken = 0;
+    // Order-preserving unsigned keys of the logits (a larger float gives a larger key,
+    // -0 is taken as +0 so that equal logits tie; 0 marks an expert that cannot be
+    // selected). Each round takes the warp maximum of the keys with one redux and the
+    // lowest expert holding it with one ballot per slot.
+    unsigned key[TK];
+#pragma unroll
+    for (int j = 0; j < TK; ++j) {
+      const unsigned u = __float_as_uint(v[j] == 0.f ? 0.f : v[j]);
+      key[j] = (lane + 32 * j < E) ? ((u & 0x80000000u) ? ~u : (u | 0x80000000u)) : 0u;
+    }
     float sel_v[8];
     int sel_e[8];
 #pragma unroll
     for (int s = 0; s < 8; ++s) {
       if (s >= k) break;
-      float bv = -INFINITY;
-      int be = 0x7fffffff;
+      unsigned best = 0;
 #pragma unroll
-      for (int j = 0; j < TK; ++j) {
-        const int e = lane + 32 * j;
-        if (e < E && !((taken >> j) & 1u) && better(v[j], e, bv, be)) { bv = v[j]; be = e; }
+      for (int j = 0; j < TK; ++j) best = max(best, key[j]);
+      const unsigned m = __reduce_max_sync(0xffffffffu, best);
+      int be = -1;
+#pragma unroll
+      for (int j = TK - 1; j >= 0; --j) {  // the lowest slot j wins, then the lowest lane
+        const unsigned bal = __ballot_sync(0xffffffffu, key[j] == m);
+        if (bal) be = 32 * j + __ffs(bal) - 1;
       }
 #pragma unroll
-      for (int off = 16; off > 0; off >>= 1) {
-        const float ov = __shfl_xor_sync(0xffffffffu, bv, off);
-        const int oe = __shfl_xor_sync(0xffffffffu, be, off);
-        if (better(ov, oe, bv, be)) { bv = ov; be = oe; }
-      }
-      if ((be & 31) == lane) taken |= 1u << (be >> 5);
-      sel_v[s] = bv;
+      for (int j = 0; j < TK; ++j)
+        if (32 * j + lane == be) key[j] = 0u;
+      sel_v[s] = __uint_as_float((m & 0x80000000u) ? (m & 0x7fffffffu) : ~m);
       sel_e[s] = be;
     }
     // softmax over the selected logits (renormalised top-k), fp32

@@ -547,8 +547,9 @@ __global__ void __launch_bounds__(kThreads, 1)
 // 256 x BN tile. Each CTA stages its own 128 rows of A and half of B (BN/2 rows)
 // per k-block; one thread of the even CTA issues M=256 MMAs that read both CTAs'
 // shared memory and write each CTA's 128 accumulator rows into its own TMEM.
-// Per SM this moves 32 KB per k-block instead of 48 KB through shared memory
-// and L2, and the ring gets 6 stages (BN 256) or 8 (BN 128).
+// Per SM this moves 32 KB per 64-deep k-block instead of 48 KB through shared
+// memory and L2; the ring holds 3 stages of 128-deep k-blocks (BN 256) or 4
+// (BN 128), and 6 or 8 64-deep stages in the gathered-operand variant.
 // Synchronization: both CTAs' loads complete on the even CTA's `full` barrier
 // (it expects both CTAs' bytes); the MMA commit arrives on the `empty` and
 // `tfull` barriers of both CTAs; both CTAs' epilogue warps arrive on the even

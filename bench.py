@@ -49,7 +49,6 @@ def committed_traffic(kernel):
     """DRAM bytes per launch of `kernel` from the committed ncu capture, or None when the
     sources that kernel is built from changed since the counters were taken (or no capture
     exists)."""
-    import hashlib
     path = os.path.join(ROOT, "profiles", "dram_traffic_laep_pruned_fwdbwd_T16384.json")
     if not os.path.exists(path):
         return None
@@ -57,11 +56,23 @@ def committed_traffic(kernel):
         rec = json.load(f).get("kernels", {}).get(kernel)
     if rec is None:
         return None
+    return rec["bytes_per_launch"] if sources_digest(rec["sources"]) == rec["sources_sha256"] else None
+
+
+def sources_digest(sources):
+    """SHA-256 over the code of the given source files with comments removed (string and
+    character literals kept), so that a comment edit does not invalidate a capture."""
+    import hashlib
+    import re
+    token = re.compile(r'//[^\n]*|/\*.*?\*/|"(?:\\.|[^"\\\n])*"|\'(?:\\.|[^\'\\\n])*\'',
+                       re.S)
     h = hashlib.sha256()
-    for src in rec["sources"]:
-        with open(os.path.join(ROOT, src), "rb") as f:
-            h.update(f.read())
-    return rec["bytes_per_launch"] if h.hexdigest() == rec["sources_sha256"] else None
+    for src in sources:
+        with open(os.path.join(ROOT, src), encoding="utf-8") as f:
+            text = f.read()
+        code = token.sub(lambda m: m.group(0) if m.group(0)[0] in "\"'" else " ", text)
+        h.update(re.sub(r"\s+", " ", code).encode())
+    return h.hexdigest()
 
 
 HBM_NOMINAL_GBS = 8000.0  # GB300 HBM3e, nominal (~8 TB/s); the measured copy peak is below it

@@ -31,10 +31,12 @@ __global__ void zero_i32_kernel(int32_t *p, int n) {
 // in tensor memory, so the logits carry fp32 accumulation error only.
 //
 // One CTA = one 128-token tile x one range of k-blocks (a split of the
-// reduction over d when there are fewer tiles than SMs). Warp 0 issues the TMA
-// loads (x tile + the three weight terms per k-block), warp 1 owns TMEM and
+// reduction over d when there are fewer tiles than CTA slots). Warp 0 issues the
+// TMA loads (x tile + the three weight terms per k-block), warp 1 owns TMEM and
 // issues the MMAs, then all four warps read the accumulator (one TMEM lane
-// quarter each) and write the partial logits partial[split][t][0..NP).
+// quarter each) and write the partial logits partial[split][t][0..NP). The same
+// kernel computes the router weight gradient with the roles changed (see
+// route_tc_kernel): 128-feature tiles of x^T, the reduction over tokens.
 constexpr int kRtBM = 128;       // tokens per tile (TMEM lanes)
 constexpr int kRtBK = 64;        // k-block: 64 bf16 = one 128-byte swizzle row
 constexpr int kRtThreads = 128;

@@ -93,7 +93,9 @@ def measured_peaks():
 # --------------------------------------------------------------------- clocks
 
 class ClockSampler:
-    """nvidia-smi samples during the timed region (median SM clock under load)."""
+    """nvidia-smi samples during the timed region (median SM clock under load). Samples
+    are kept with their arrival time; those between mark_start() and mark_end() (the
+    timed region) are the ones reported, when there are any."""
 
     Q = ("clocks.sm,clocks.max.sm,utilization.gpu,power.draw,clocks_event_reasons.hw_slowdown,"
          "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
@@ -103,6 +105,13 @@ class ClockSampler:
         self.index = index
         self.proc = None
         self.lines = []
+        self.t0 = self.t1 = None
+
+    def mark_start(self):
+        self.t0 = time.monotonic()
+
+    def mark_end(self):
+        self.t1 = time.monotonic()
 
     def start(self):
         try:
@@ -117,7 +126,7 @@ class ClockSampler:
 
     def _read(self):
         for line in self.proc.stdout:
-            self.lines.append(line.strip())
+            self.lines.append((time.monotonic(), line.strip()))
 
     def stop(self):
         if self.proc is None:
@@ -130,7 +139,11 @@ class ClockSampler:
         self.thread.join(timeout=2)
         names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
         sm, mx, reasons, loaded = [], None, set(), []
-        for ln in self.lines:
+        lines = self.lines
+        if self.t0 is not None and self.t1 is not None:
+            inside = [(t, ln) for t, ln in lines if self.t0 <= t <= self.t1]
+            lines = inside or lines
+        for _, ln in lines:
             f = [x.strip() for x in ln.split(",")]
             if len(f) < 8:
                 continue
@@ -321,10 +334,11 @@ def timed_steps(wl, steps, world, local, per_kernel_timing=True, flush=None):
     L.moe_timing_read(reset=True)
     ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
           for _ in range(steps if flush is not None else 1)]
-    barrier(world)
-    torch.cuda.synchronize()
     clocks.start()
     time.sleep(0.3)  # let the sampler start
+    barrier(world)
+    torch.cuda.synchronize()
+    clocks.mark_start()
     if flush is None:
         ev[0][0].record(stream)
         for _ in range(steps):
@@ -337,6 +351,7 @@ def timed_steps(wl, steps, world, local, per_kernel_timing=True, flush=None):
             wl.step()
             ev[i][1].record(stream)
     torch.cuda.synchronize()
+    clocks.mark_end()
     barrier(world)
     clk = clocks.stop()
     L.moe_timing_enable(False)
@@ -667,7 +682,10 @@ def run_reference(args):
     if rank != 0:
         return
     c = synth.CONFIGS[args.config]
-    n_tok = min(args.ref_tokens, c.T)
+    # tokens per step: 64 at 30 steps, fewer for more steps, so that the whole run keeps
+    # to a couple of minutes of host time
+    ref_tokens = args.ref_tokens or max(8, min(64, (64 * 30) // max(args.steps, 1)))
+    n_tok = min(ref_tokens, c.T)
     dev = "cuda" if torch.cuda.is_available() else "cpu"
     inp = synth.make_config_inputs(args.config, device=dev)
     mask_h = None
@@ -708,12 +726,13 @@ def run_reference(args):
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=30)
+    ap.add_argument("--steps", type=int, default=100)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--config", type=int, default=2, choices=sorted(synth.CONFIGS))
     ap.add_argument("--cpu-tokens", type=int, default=4096)
-    ap.add_argument("--ref-tokens", type=int, default=64)
+    ap.add_argument("--ref-tokens", type=int, default=None,
+                    help="tokens per reference-arm step (default: 64 x 30 / steps, 8 to 64)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-laep", action="store_true",

@@ -963,11 +963,20 @@ int launch_pair(const CUtensorMap &a, const CUtensorMap &b, const CUtensorMap &o
                 const GemmParams &p, cudaStream_t s, const char *what) {
   using Sh = PairShape<BN, GATHER ? 64 : 128>;
   auto kern = grouped_gemm_pair_kernel<MODE, BN, GATHER>;
-  cudaLaunchAttribute at[1];
+  cudaLaunchAttribute at[2];
   at[0].id = cudaLaunchAttributeClusterDimension;
   at[0].val.clusterDim.x = 2;
   at[0].val.clusterDim.y = 1;
   at[0].val.clusterDim.z = 1;
+  // the highest scheduling priority: a kernel launched beside it on another stream
+  // does not take the SMs its persistent CTA pairs are waiting for
+  static int prio = [] {
+    int least = 0, greatest = 0;
+    cudaDeviceGetStreamPriorityRange(&least, &greatest);
+    return greatest;
+  }();
+  at[1].id = cudaLaunchAttributePriority;
+  at[1].val.priority = prio;
   cudaLaunchConfig_t cfg = {};
   cfg.blockDim = dim3(kThreads);
   cfg.dynamicSmemBytes = Sh::SMEM;
@@ -986,6 +995,7 @@ int launch_pair(const CUtensorMap &a, const CUtensorMap &b, const CUtensorMap &o
     nclusters = n;
   }
   cfg.gridDim = dim3(2 * nclusters);
+  cfg.numAttrs = 2;
   MOE_LAUNCH(kGemmName[MODE], s, cudaLaunchKernelEx(&cfg, kern, a, b, o, p));
   return moe::launch_status(what);
 }

@@ -1,0 +1,51 @@
+"""Host-side logic of bench.py that needs no GPU: the key that ties a committed DRAM
+capture to the code it measured, and the clock sampler's restriction to the timed
+region."""
+import os
+
+import bench
+
+
+def test_traffic_key_ignores_comments_not_code(tmp_path, monkeypatch):
+    src = "paper_2601_14327_gb300/csrc/route.cu"
+    text = open(os.path.join(bench.ROOT, src), encoding="utf-8").read()
+    base = bench.sources_digest([src])
+    monkeypatch.setattr(bench, "ROOT", str(tmp_path))
+    os.makedirs(tmp_path / os.path.dirname(src))
+
+    def digest_of(t):
+        (tmp_path / src).write_text(t, encoding="utf-8")
+        return bench.sources_digest([src])
+
+    assert digest_of(text) == base
+    # comment edits and re-indentation keep the key
+    assert digest_of(text.replace("// ", "//  the ", 3)) == base
+    assert digest_of("/* a new block\n comment */\n" + text) == base
+    assert digest_of(text.replace("\n", "\n  ", 5)) == base
+    # a code edit, or an edit inside a string literal, changes it
+    assert digest_of(text.replace("kRtBM = 128", "kRtBM = 64", 1)) != base
+    assert digest_of(text.replace('"moe_route: logits"', '"moe_route: logit"', 1)) != base
+
+
+def test_clock_sampler_keeps_the_timed_region():
+    c = bench.ClockSampler(0)
+    row = "{sm},2070,{u},1000,Not Active,Not Active,Not Active,{cap}"
+    c.lines = [(0.0, row.format(sm=2070, u=0, cap="Not Active")),      # idle, before
+               (1.0, row.format(sm=1500, u=100, cap="Active")),        # timed region
+               (1.1, row.format(sm=1520, u=100, cap="Active")),
+               (1.2, row.format(sm=1480, u=30, cap="Active")),         # a lagging sample
+               (3.0, row.format(sm=2070, u=0, cap="Not Active"))]      # idle, after
+    c.t0, c.t1 = 0.5, 2.0
+
+    class _Done:
+        def terminate(self): pass
+        def wait(self, timeout=None): pass
+
+    class _Joined:
+        def join(self, timeout=None): pass
+
+    c.proc, c.thread = _Done(), _Joined()
+    out = c.stop()
+    assert out["samples"] == 3 and out["samples_under_load"] == 2
+    assert out["sm_mhz"] == 1510 and out["sm_max_mhz"] == 2070
+    assert out["reasons"] == ["sw_power_cap"]

@@ -8,9 +8,11 @@ SwiGLU FFN forward -> combine -> combine backward -> grouped FFN backward
 decision itself runs once before the timed steps, as in the paper (one prune
 once the loads are stable), on the histogram of a first routing pass.
 
-Default workload: T=16384 tokens, d_model=4096, 64 experts of which the 16
-least-loaded are pruned (48 live), top-8, d_ff=2048, Zipf(1.2) gate bias,
-bf16 data with an fp32 router, seeded synthetic inputs.
+Default workload: the largest one, T=65536 tokens, d_model=7168, 256 experts of
+which the 85 least-loaded are pruned and removed from the weights (171 kept),
+top-8, d_ff=2048, Zipf(1.0) gate bias, bf16 data with an fp32 router, seeded
+synthetic inputs; its line also times the unpruned layer (all 256 experts) for
+the pruned-vs-unpruned ratio. `--config N` selects another workload.
 
 Prints ONE JSON line (rank 0). `--impl reference` times the CPU oracle on a
 bounded token sample of the same workload instead.
@@ -45,11 +47,11 @@ GEMMS = ["gemm_gate_up", "gemm_down", "gemm_dgrad_down", "gemm_dgrad_gate_up",
          "gemm_wgrad_down", "gemm_wgrad_gate_up"]
 
 
-def committed_traffic(kernel):
-    """DRAM bytes per launch of `kernel` from the committed ncu capture, or None when the
-    sources that kernel is built from changed since the counters were taken (or no capture
-    exists)."""
-    path = os.path.join(ROOT, "profiles", "dram_traffic_laep_pruned_fwdbwd_T16384.json")
+def committed_traffic(workload, kernel):
+    """DRAM bytes per launch of `kernel` at `workload` from the committed ncu record
+    (profiles/dram_traffic_<workload>.json), or None when the sources that kernel is built
+    from changed since the counters were taken (or no record exists)."""
+    path = os.path.join(ROOT, "profiles", f"dram_traffic_{workload}.json")
     if not os.path.exists(path):
         return None
     with open(path) as f:
@@ -76,6 +78,8 @@ def sources_digest(sources):
 
 
 HBM_NOMINAL_GBS = 8000.0  # GB300 HBM3e, nominal (~8 TB/s); the measured copy peak is below it
+BF16_NOMINAL_TFLOPS = 2250.0  # GB300 dense bf16 tensor peak, nominal (no 2:4 sparsity)
+SUSTAINED_REGION_S = 1.0  # timed regions at least this long use the sustained bf16 peak
 
 
 def measured_peaks():
@@ -88,6 +92,20 @@ def measured_peaks():
                 "source": "measured"}
     return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0,
             "source": "fallback"}
+
+
+def tensor_peak(peaks, region_s):
+    """bf16 denominator for kernels timed inside a region of `region_s` seconds, and its
+    name. A region of a second or more runs at the clock the power cap settles at, so it is
+    compared with the sustained cuBLAS rate (a seconds-long loop under the cap); a shorter
+    region with the burst rate (cuBLAS timed alone)."""
+    if region_s >= SUSTAINED_REGION_S:
+        return (peaks["bf16_tflops_sustained"],
+                f"bf16_tflops_sustained of MEASURED_PEAKS.json ({peaks['source']}): timed region "
+                f"{region_s:.2f} s >= {SUSTAINED_REGION_S:g} s")
+    return (peaks["bf16_tflops"],
+            f"bf16_tflops (burst) of MEASURED_PEAKS.json ({peaks['source']}): timed region "
+            f"{region_s:.2f} s < {SUSTAINED_REGION_S:g} s")
 
 
 # --------------------------------------------------------------------- clocks
@@ -127,6 +145,12 @@ class ClockSampler:
     def _read(self):
         for line in self.proc.stdout:
             self.lines.append((time.monotonic(), line.strip()))
+
+    def wait_first(self, timeout=5.0):
+        """Blocks until the sampler has delivered a line (or `timeout` seconds)."""
+        t_end = time.monotonic() + timeout
+        while self.proc is not None and not self.lines and time.monotonic() < t_end:
+            time.sleep(0.02)
 
     def stop(self):
         if self.proc is None:
@@ -231,7 +255,7 @@ class Workload:
                       i["w_down"], self.mask)
         if self.backward:
             layer.backward(b, i["dy"] if dy is None else dy, i["w_router"], i["w_gate_up"],
-                           i["w_down"], overlap=self.overlap)
+                           i["w_down"], overlap=self.overlap, active_mask=self.mask)
 
     def make_graph(self, x=None, dy=None):
         """A CUDA graph of one whole step (both streams) on inputs x, dy. The library's calls
@@ -247,6 +271,15 @@ class Workload:
     def capture(self):
         """Later steps without explicit inputs replay a graph of the step."""
         self.graph = self.make_graph()
+
+    def live_counts(self):
+        """Rows per live expert (pruned experts of a mask excluded: they get no tile and
+        no weight-gradient write)."""
+        counts = self.bufs.counts.cpu().tolist()
+        if self.mask is None:
+            return counts
+        m = self.mask.cpu().tolist()
+        return [c for c, keep in zip(counts, m) if keep]
 
     def gemm_flops(self):
         """Algorithmic FLOPs per GEMM kernel launch (real assignments only)."""
@@ -301,27 +334,45 @@ def replica_throughput(world, tokens_per_rank, steps, ms_max):
     return world * tokens_per_rank * steps / (ms_max / 1e3)
 
 
-def oracle_sample(wl_inputs_host, mask_host, k, n_tok, backward=True):
-    """Runs the CPU oracle over the first n_tok tokens (forward, and backward unless the
-    workload is forward-only); returns the seconds it took."""
+def oracle_sample(h, k, backward=True):
+    """Runs the CPU oracle's whole layer on a sample prepared by sample_inputs (forward, and
+    backward unless the workload is forward-only); returns the seconds it took."""
     from oracle import moe_oracle as O
-    h = wl_inputs_host
     t0 = time.perf_counter()
-    O.moe_layer(h["x"][:n_tok], h["w_router"], h["bias"], mask_host, k, h["w_gate_up"],
-                h["w_down"], dy=h["dy"][:n_tok] if backward else None)
+    O.moe_layer(h["x"], h["w_router"], h["bias"], h["mask"], k, h["w_gate_up"], h["w_down"],
+                dy=h["dy"] if backward else None)
     return time.perf_counter() - t0
 
 
-def host_inputs(inp, n_tok):
-    """float32 host copies of the inputs the oracle reads (bf16 values are exact)."""
-    out = {}
-    for n in ("x", "dy"):
-        out[n] = inp[n][:n_tok].float().cpu().numpy()
-    for n in ("w_router", "bias"):
-        out[n] = inp[n].float().cpu().numpy()
-    for n in ("w_gate_up", "w_down"):
-        out[n] = inp[n].float().cpu().numpy()
-    return out
+def sample_inputs(inp, mask, k, n_tok):
+    """float32 host inputs of a bounded oracle sample: the first n_tok tokens, and of the
+    experts only those the sample's tokens are routed to (the router's columns, bias and
+    expert weights of that subset, in expert order). Every token's k selected experts are in
+    the subset and the order of expert ids is kept, so the top-k, the gates and every output
+    and gradient of these tokens are the full layer's; the weights of the experts no sampled
+    token reaches (up to 22.5 GB at T=65536, d=7168, 256 experts) stay on the device.
+    Returns (inputs, number of experts in the subset)."""
+    from oracle import moe_oracle as O
+    x = inp["x"][:n_tok].float().cpu().numpy()
+    wr = inp["w_router"].float().cpu().numpy()
+    b = inp["bias"].float().cpu().numpy()
+    m = None if mask is None else mask.cpu().numpy()
+    idx, _ = O.route_topk(O.router_logits(x, wr, b, m), k)
+    used = np.unique(idx)
+    sel = torch.as_tensor(used, dtype=torch.long, device=inp["w_gate_up"].device)
+    out = {"x": x, "w_router": np.ascontiguousarray(wr[:, used]), "bias": b[used],
+           "mask": None,  # the subset holds only experts tokens were routed to: all live
+           "w_gate_up": inp["w_gate_up"].index_select(0, sel).float().cpu().numpy(),
+           "w_down": inp["w_down"].index_select(0, sel).float().cpu().numpy()}
+    if "dy" in inp:
+        out["dy"] = inp["dy"][:n_tok].float().cpu().numpy()
+    return out, int(used.size)
+
+
+# tokens of the oracle sample per workload: the CPU baseline of the main arm (10-30 s of host
+# time on 16 cores), and one step of the reference arm at 30 steps (fewer at more steps)
+CPU_TOKENS = {0: 512, 1: 1024, 2: 4096, 3: 1024, 4: 16}
+REF_TOKENS_30 = {0: 512, 1: 256, 2: 64, 3: 32, 4: 3}
 
 
 def timed_steps(wl, steps, world, local, per_kernel_timing=True, flush=None):
@@ -335,7 +386,7 @@ def timed_steps(wl, steps, world, local, per_kernel_timing=True, flush=None):
     ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
           for _ in range(steps if flush is not None else 1)]
     clocks.start()
-    time.sleep(0.3)  # let the sampler start
+    clocks.wait_first()  # the sampler is running before the timed region opens
     barrier(world)
     torch.cuda.synchronize()
     clocks.mark_start()
@@ -361,17 +412,16 @@ def timed_steps(wl, steps, world, local, per_kernel_timing=True, flush=None):
     return max_over_ranks(ms, world), per_kernel, clk
 
 
-def group_bound_seconds(shape, counts, peaks):
+def group_bound_seconds(shape, counts, peaks, tflops_peak):
     """Per GEMM: the sum over experts of max(FLOPs_e / tensor peak, bytes_e / HBM peak),
     each expert's group taken alone at full machine speed. Under skewed loads a light
-    expert's GEMM is bound by its weight (or weight-gradient) bytes, not its FLOPs, and a
-    pruned expert's weight gradients are still written (zeros), so this, not the FLOP
-    roofline, is what a grouped GEMM can reach on these loads."""
+    expert's GEMM is bound by its weight (or weight-gradient) bytes, not its FLOPs, so
+    this, not the FLOP roofline, is what a grouped GEMM can reach on these loads. `counts`
+    holds the live experts' rows; pruned experts get no tile and no write."""
     d, F = shape.d, shape.F
-    P = peaks["bf16_tflops_sustained"] * 1e12
+    P = tflops_peak * 1e12
     BW = peaks["hbm_gbs"] * 1e9
-    out = dict.fromkeys(["gemm_gate_up", "gemm_down", "gemm_dgrad_down", "gemm_dgrad_gate_up",
-                         "gemm_wgrad_down", "gemm_wgrad_gate_up"], 0.0)
+    out = dict.fromkeys(GEMMS, 0.0)
     for m in counts:
         m = int(m)
         fl = {  # FLOPs, bytes (activations read/written, weights or weight gradients)
@@ -384,17 +434,33 @@ def group_bound_seconds(shape, counts, peaks):
         }
         for n, (f, b) in fl.items():
             if m == 0 and not n.startswith("gemm_wgrad"):
-                continue  # no rows: no tile (weight gradients are still written)
+                continue  # no rows: no tile (a live expert's zero weight gradient is written)
             out[n] += max(f / P, b / BW)
     return out
 
 
-def kernel_report(wl, per_kernel, steps, peaks):
-    """Per-kernel live CUDA-event times with achieved rates against the roofline."""
+# kernels of the second stream: timed in a pass of their own with the second stream off,
+# because beside the persistent GEMMs their CUDA events also count the time they queue
+SIDE_KERNELS = ("route_bwd_dz", "route_bwd_dw", "route_bwd_reduce", "transpose_router",
+                "permute_bwd")
+
+
+def route_tc_flops(s):
+    """Tensor-core FLOPs of the router's two contractions (logits x.W_r and dW_r = x^T.dZ):
+    the fp32 operand is carried as three bf16 terms, so 3 x 2 x T x d x NP, with NP the
+    experts rounded up to 16 (the MMA's N)."""
+    NP = (s.E + 15) // 16 * 16
+    return 3 * 2 * s.T * s.d * NP
+
+
+def kernel_report(wl, per_kernel, steps, peaks, tflops_peak, counts, sm_mhz=None,
+                  alone=None, alone_steps=1):
+    """Per-kernel live CUDA-event times with achieved rates against the roofline. Entries of
+    `alone` (a pass with the second stream off) replace the second-stream kernels'."""
     s = wl.shape
     A = s.T * s.k
     flops = wl.gemm_flops()
-    bound = group_bound_seconds(s, wl.bufs.counts.cpu().tolist(), peaks)
+    bound = group_bound_seconds(s, counts, peaks, tflops_peak)
     hbm = {  # algorithmic bytes per launch of the HBM-bound kernels
         "perm_gather": 2 * s.T * s.d + 2 * A * s.d,
         "combine": 2 * A * s.d + 2 * s.T * s.d,
@@ -405,19 +471,34 @@ def kernel_report(wl, per_kernel, steps, peaks):
         "route_bwd_dw": 2 * s.T * s.d + 4 * s.d * s.E,
         "route_logits": 2 * s.T * s.d + 4 * s.d * s.E + 4 * s.T * s.E,
     }
+    tc_route = {"route_logits": route_tc_flops(s), "route_bwd_dw": route_tc_flops(s)}
     tot = sum(v[1] for v in per_kernel.values())
     out = {}
     for n, (c, ms) in per_kernel.items():
         e = {"launches": c, "ms_per_step": round(ms / steps, 4), "share": round(ms / tot, 4)}
-        per_launch_s = ms / c / 1e3
+        if alone and n in SIDE_KERNELS and n in alone:
+            c, ms = alone[n]
+            e.update(ms_per_step_alone=round(ms / alone_steps, 4),
+                     timed="alone (second stream off); ms_per_step is the overlapped pass, "
+                           "queueing behind the GEMMs included")
+            ms_launch = ms / c
+        else:
+            ms_launch = ms / c
+        per_launch_s = ms_launch / 1e3
         if n in flops:
             tf = flops[n] / per_launch_s / 1e12
-            e.update(tflops=round(tf, 1), frac=round(tf / peaks["bf16_tflops_sustained"], 4),
+            e.update(tflops=round(tf, 1), frac=round(tf / tflops_peak, 4),
+                     frac_nominal=round(tf / BF16_NOMINAL_TFLOPS, 4),
                      group_bound_frac=round(bound[n] / per_launch_s, 4))
+            if sm_mhz:
+                e["gflops_per_mhz"] = round(tf * 1e3 / sm_mhz, 1)
         elif n in hbm:
             gbs = hbm[n] / per_launch_s / 1e9
             e.update(gbs=round(gbs, 1), frac=round(gbs / peaks["hbm_gbs"], 4),
                      frac_nominal=round(gbs / HBM_NOMINAL_GBS, 4))
+            if n in tc_route:
+                tf = tc_route[n] / per_launch_s / 1e12
+                e.update(tc_tflops=round(tf, 1), tc_frac=round(tf / tflops_peak, 4))
         out[n] = e
     return out
 
@@ -434,10 +515,6 @@ def laep_comparison(args, world, local, pruned_tps, wl_pruned):
     # live experts: the compacted count, or the unmasked ones when pruning is a mask
     pruned_params = 3 * wl_pruned.E_live * wl_pruned.shape.d * wl_pruned.shape.F
     c = wl_pruned.cfg
-    # free the pruned workload's activations while the unpruned one runs
-    saved = wl_pruned.bufs
-    wl_pruned.bufs = None
-    torch.cuda.empty_cache()
     wl_u = Workload(args.config, "cuda", no_prune=True, gather=bool(args.gather),
                     overlap=bool(args.overlap), fused_combine=bool(args.fused_combine))
     for _ in range(args.warmup):
@@ -451,16 +528,31 @@ def laep_comparison(args, world, local, pruned_tps, wl_pruned):
     unpruned_params = 3 * wl_u.shape.E * wl_u.shape.d * wl_u.shape.F
     del wl_u
     torch.cuda.empty_cache()
-    wl_pruned.bufs = saved
     return {"experts_unpruned": c.E, "experts_pruned": wl_pruned.E_live,
             "pruning": ("compacted (pruned experts' weights removed)" if wl_pruned.mask is None
-                        else "mask (pruned experts get no token; their weight gradients are "
-                             "still written, as zeros)"),
+                        else "mask (pruned experts get no token and no tile; their weight "
+                             "gradients are not written)"),
             "unpruned_tokens_per_s": round(tps_u, 1), "pruned_tokens_per_s": round(pruned_tps, 1),
             "speedup": round(pruned_tps / tps_u, 4),
             "expert_params_unpruned": unpruned_params, "expert_params_pruned": pruned_params,
             "expert_param_reduction": round(1 - pruned_params / unpruned_params, 4),
             "unpruned_steps": steps, "context": PARAMS_NOTE}
+
+
+def workload_config(args, c, T, E_held, E_live, n_pruned, backward, world):
+    """The `config` object of both arms' lines. E_held = experts whose weights the timed
+    layer holds (after compaction), E_live = experts tokens can be routed to."""
+    return {"workload": c.name, "T": T, "d_model": c.d, "experts": c.E, "experts_live": E_live,
+            "top_k": c.k, "d_ff": c.F, "gate_bias": c.bias, "pruned": n_pruned,
+            "pass": "forward+backward" if backward else "forward",
+            "l2": ("256 MB buffer rewritten before every timed step" if args.flush_l2
+                   else "no flush (inputs larger than L2: x %.0f MB, expert weights %.2f GB)"
+                   % (2 * T * c.d / 1e6, 6 * E_held * c.d * c.F / 1e9)),
+            "parallelism": "replicas" if world > 1 else "1 GPU",
+            "dispatch": ("TMA gathers from x (X_perm not materialized)" if args.gather
+                         else "materialized X_perm"),
+            "combine": ("in the down GEMM's epilogue (fp32 atomics)" if args.fused_combine
+                        else "separate kernel")}
 
 
 def run_ours(args):
@@ -483,8 +575,8 @@ def run_ours(args):
              else None)
     if args.graph:
         # per-kernel CUDA-event table from eager steps, the timed steps replay a graph
-        _, per_kernel, _ = timed_steps(wl, args.steps, world, local, per_kernel_timing=True,
-                                       flush=flush)
+        ms_eager, per_kernel, clk_eager = timed_steps(wl, args.steps, world, local,
+                                                      per_kernel_timing=True, flush=flush)
         wl.capture()
         for _ in range(args.warmup):
             wl.step()
@@ -492,20 +584,33 @@ def run_ours(args):
                                        flush=flush)
     else:
         ms_total, per_kernel, clk = timed_steps(wl, args.steps, world, local, flush=flush)
+        ms_eager, clk_eager = ms_total, clk
     ms_step = ms_total / args.steps
     tokens_per_s = replica_throughput(world, s.T, args.steps, ms_total)
     launches = sum(n for n, _ in per_kernel.values())
 
-    # dominant kernel and its roofline
+    # the second-stream kernels at their own rates: a few eager steps with that stream off
+    alone, alone_steps = None, 0
+    if wl.backward and wl.overlap:
+        alone_steps = min(args.steps, 5)
+        graph, wl.graph, wl.overlap = wl.graph, None, False
+        _, alone, _ = timed_steps(wl, alone_steps, world, local, per_kernel_timing=True)
+        wl.graph, wl.overlap = graph, True
+
+    # dominant kernel and its roofline; the peak follows the length of the region the
+    # kernels were timed in (the eager pass, as long as the timed one)
+    tflops_peak, peak_source = tensor_peak(peaks, ms_eager / 1e3)
     gemm_ms = {n: per_kernel[n][1] / per_kernel[n][0] for n in GEMMS if n in per_kernel}
     flops = wl.gemm_flops()
     dom = max(gemm_ms, key=lambda n: per_kernel[n][1])
     dom_tflops = flops[dom] / (gemm_ms[dom] / 1e3) / 1e12
     all_gemm_ms = sum(per_kernel[n][1] for n in gemm_ms) / args.steps
     all_gemm_tflops = sum(flops[n] for n in gemm_ms) / (all_gemm_ms / 1e3) / 1e12
-    peak = peaks["bf16_tflops_sustained"]
-    kernel_table = kernel_report(wl, per_kernel, args.steps, peaks)
-    gb = group_bound_seconds(wl.shape, wl.bufs.counts.cpu().tolist(), peaks)
+    live_counts = wl.live_counts()
+    kernel_table = kernel_report(wl, per_kernel, args.steps, peaks, tflops_peak, live_counts,
+                                 sm_mhz=clk_eager.get("sm_mhz"), alone=alone,
+                                 alone_steps=alone_steps)
+    gb = group_bound_seconds(wl.shape, live_counts, peaks, tflops_peak)
     gemm_bound_frac = sum(gb[n] for n in gemm_ms) / (all_gemm_ms / 1e3)
 
     # end to end through the public API: every step uploads its inputs from pinned host
@@ -620,46 +725,46 @@ def run_ours(args):
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        n_tok = min(args.cpu_tokens, s.T)
-        hin = host_inputs(wl.inp, n_tok)
-        mask_h = None if wl.mask is None else wl.mask.cpu().numpy()
-        secs = oracle_sample(hin, mask_h, s.k, n_tok, backward=wl.backward)
+        n_tok = min(args.cpu_tokens or CPU_TOKENS[args.config], s.T)
+        hin, n_exp = sample_inputs(wl.inp, wl.mask, s.k, n_tok)
+        secs = oracle_sample(hin, s.k, backward=wl.backward)
+        del hin
         cpu = {"value": round(n_tok / secs, 3), "unit": "tokens/s",
                "cores": int(os.environ.get("OPENBLAS_NUM_THREADS", NCPU)), "kind": "oracle",
-               "sample": f"first {n_tok} of {s.T} tokens of the same layer step (all {s.E} experts, "
-                         f"same mask and weights), fp64 numpy oracle, {secs:.1f} s wall"}
+               "sample": f"first {n_tok} of {s.T} tokens of the same layer step "
+                         f"({'fwd+bwd' if wl.backward else 'forward'}), with the {n_exp} of "
+                         f"{s.E} experts they are routed to (same routing, mask and weights), "
+                         f"fp64 numpy oracle, {secs:.1f} s wall"}
 
     c = wl.cfg
+    default_workload = (args.tokens is None and args.experts is None and not args.no_prune
+                        and args.bias is None)
     out = {
         "metric": METRIC, "value": round(tokens_per_s, 1), "unit": "tokens/s", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_step, 4),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
         "data": "synthetic (seeded; random-init expert weights)",
-        "config": {"workload": c.name, "T": s.T, "d_model": s.d, "experts": c.E,
-                   "experts_live": wl.E_live, "top_k": s.k, "d_ff": s.F, "gate_bias": c.bias,
-                   "pruned": wl.n_pruned, "pass": "forward+backward" if wl.backward else "forward",
-                   "l2": ("256 MB buffer rewritten before every timed step" if args.flush_l2
-                          else "no flush (working set: x %.0f MB, expert weights %.2f GB)"
-                          % (2 * s.T * s.d / 1e6, 6 * s.E * s.d * s.F / 1e9)),
-                   "parallelism": "replicas" if world > 1 else "1 GPU",
-                   "dispatch": ("TMA gathers from x (X_perm not materialized)" if args.gather
-                                else "materialized X_perm"),
-                   "combine": ("in the down GEMM's epilogue (fp32 atomics)" if args.fused_combine
-                               else "separate kernel")},
+        "config": workload_config(args, c, s.T, s.E, wl.E_live, wl.n_pruned, wl.backward,
+                                  world),
         "grouped_gemm": {"tflops": round(all_gemm_tflops, 1),
-                         "frac_of_peak": round(all_gemm_tflops / peak, 4),
-                         "peak_tflops": peak, "peak": f"bf16 sustained, {peaks['source']}",
+                         "frac_of_peak": round(all_gemm_tflops / tflops_peak, 4),
+                         "peak_tflops": tflops_peak, "peak_source": peak_source,
+                         "frac_nominal": round(all_gemm_tflops / BF16_NOMINAL_TFLOPS, 4),
+                         "nominal_tflops": BF16_NOMINAL_TFLOPS,
+                         "gflops_per_mhz": (round(all_gemm_tflops * 1e3 / clk_eager["sm_mhz"], 1)
+                                            if clk_eager.get("sm_mhz") else None),
+                         "sm_mhz": clk_eager.get("sm_mhz"),
                          "ms_per_step": round(all_gemm_ms, 4),
                          "group_bound_frac": round(gemm_bound_frac, 4),
-                         "group_bound": "sum over experts of max(FLOPs/tensor peak, bytes/HBM "
-                                        "peak) over the measured time (pruned experts' zero "
-                                        "weight gradients included)"},
+                         "group_bound": "sum over live experts of max(FLOPs/tensor peak, "
+                                        "bytes/HBM peak) over the measured time"},
         "roofline": {"kernel": dom, "bound": "tensor", "achieved": round(dom_tflops, 1),
-                     "peak": peak, "unit": "TFLOP/s", "frac": round(dom_tflops / peak, 4),
-                     "traffic": (committed_traffic(dom) if wl.cfg_id == 2 and args.tokens is None
-                                 and args.experts is None and not args.no_prune
-                                 and args.bias is None else None),
-                     "peak_source": f"bf16 sustained ({peaks['source']})"},
+                     "peak": tflops_peak, "unit": "TFLOP/s", "frac": round(dom_tflops / tflops_peak, 4),
+                     "frac_nominal": round(dom_tflops / BF16_NOMINAL_TFLOPS, 4),
+                     "traffic": committed_traffic(c.name, dom) if default_workload else None,
+                     "peak_source": peak_source,
+                     "achieved_from": f"algorithmic FLOPs of one launch / mean CUDA-event "
+                                      f"duration over {args.steps} eager steps"},
         "timed_as": "CUDA graph replay of the whole step" if args.graph else "eager launches",
         "kernels": kernel_table,
         "laep": laep,
@@ -675,48 +780,127 @@ def run_ours(args):
         dist.destroy_process_group()
 
 
+def layer_calls(wl):
+    """One entry point of the layer step each, on the workload's buffers (as a step makes
+    them): `--call NAME` times one of them alone."""
+    i, b, s = wl.inp, wl.bufs, wl.shape
+    R = s.rows_cap
+    return {
+        "route": lambda: layer.route(b, i["x"], i["w_router"], i["bias"], wl.mask),
+        "permute": lambda: L.moe_permute(i["x"], b.topk_idx, b.counts, s.T, s.d, s.E, s.k, R,
+                                         b.group_offsets, b.group_counts, b.row_of_assignment,
+                                         b.x_perm, b.ws, b.ws_bytes),
+        "ffn_fwd": lambda: L.moe_grouped_ffn_fwd(b.x_perm, b.group_offsets, s.E, s.d, s.F, R,
+                                                 i["w_gate_up"], i["w_down"], b.ab, b.h,
+                                                 b.out_perm, b.ws, b.ws_bytes),
+        "combine": lambda: L.moe_unpermute_combine(b.out_perm, b.row_of_assignment, b.topk_gate,
+                                                   s.T, s.d, s.k, b.y),
+        "combine_bwd": lambda: L.moe_unpermute_combine_bwd(
+            i["dy"], b.out_perm, b.row_of_assignment, b.topk_gate, b.group_offsets,
+            b.group_counts, s.T, s.d, s.E, s.k, b.d_out_perm, b.d_gate),
+        "ffn_bwd_dgrad": lambda: L.moe_grouped_ffn_bwd_dgrad(
+            b.d_out_perm, b.ab, b.group_offsets, s.E, s.d, s.F, R, i["w_gate_up"], i["w_down"],
+            b.d_ab, b.dx_perm, b.ws, b.ws_bytes),
+        "ffn_bwd_wgrad": lambda: L.moe_grouped_ffn_bwd_wgrad(
+            b.d_out_perm, b.x_perm, b.h, b.d_ab, b.group_offsets, wl.mask, s.E, s.d, s.F, R,
+            b.dw_gate_up, b.dw_down, b.ws, b.ws_bytes),
+        "route_bwd": lambda: L.moe_route_bwd(b.x, b.topk_idx, b.topk_gate, b.d_gate, s.T, s.d,
+                                             s.E, s.k, b.d_logits, b.dw_router, b.ws,
+                                             b.ws_bytes),
+        "permute_bwd": lambda: L.moe_permute_bwd(b.dx_perm, b.row_of_assignment, b.topk_idx,
+                                                 b.d_logits, i["w_router"], s.T, s.d, s.E, s.k,
+                                                 b.dx, b.ws, b.ws_bytes),
+    }
+
+
+CALL_NAMES = ["route", "permute", "ffn_fwd", "combine", "combine_bwd", "ffn_bwd_dgrad",
+              "ffn_bwd_wgrad", "route_bwd", "permute_bwd"]
+
+
+def run_call(args):
+    """Times one entry point alone (`--call NAME`) on the workload's inputs and buffers after
+    one eager step: K calls between synchronizes, CUDA events per kernel. For single-kernel
+    profiler captures (use --tokens/--experts for a small case). One JSON line."""
+    L.load()
+    torch.cuda.set_device(0)
+    peaks = measured_peaks()
+    wl = Workload(args.config, "cuda", tokens=args.tokens, experts=args.experts,
+                  no_prune=args.no_prune, bias=args.bias, backward=True)
+    wl.eager_step()
+    fn = layer_calls(wl)[args.call]
+    for _ in range(args.warmup):
+        fn()
+    torch.cuda.synchronize()
+    L.moe_timing_enable(True)
+    L.moe_timing_read(reset=True)
+    stream = torch.cuda.current_stream()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record(stream)
+    for _ in range(args.steps):
+        fn()
+    b.record(stream)
+    torch.cuda.synchronize()
+    L.moe_timing_enable(False)
+    per_kernel = L.moe_timing_read(reset=True)
+    assert L.moe_device_error(clear=True) == 0, "device error during the timed calls"
+    ms = a.elapsed_time(b)
+    tflops_peak, peak_source = tensor_peak(peaks, ms / 1e3)
+    table = kernel_report(wl, per_kernel, args.steps, peaks, tflops_peak, wl.live_counts())
+    print(json.dumps({"call": args.call, "workload": wl.cfg.name,
+                      "config": {"T": wl.shape.T, "d_model": wl.shape.d, "experts": wl.shape.E,
+                                 "top_k": wl.shape.k, "d_ff": wl.shape.F},
+                      "calls": args.steps, "ms_per_call": round(ms / args.steps, 4),
+                      "peak_source": peak_source, "kernels": table}), flush=True)
+
+
 def run_reference(args):
-    """The CPU oracle on the host cores: each step a bounded token sample."""
+    """The CPU oracle on the host cores: each step a bounded sample of the same workload (the
+    first tokens, with the experts they are routed to; see sample_inputs)."""
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
     if rank != 0:
         return
     c = synth.CONFIGS[args.config]
-    # tokens per step: 64 at 30 steps, fewer for more steps, so that the whole run keeps
-    # to a couple of minutes of host time
-    ref_tokens = args.ref_tokens or max(8, min(64, (64 * 30) // max(args.steps, 1)))
-    n_tok = min(ref_tokens, c.T)
+    # tokens per step: REF_TOKENS_30 at 30 steps, fewer at more steps, so that the whole run
+    # keeps to a few minutes of host time
+    base = REF_TOKENS_30[args.config]
+    n_tok = min(args.ref_tokens or max(1, min(base, (base * 30) // max(args.steps, 1))), c.T)
     dev = "cuda" if torch.cuda.is_available() else "cpu"
     inp = synth.make_config_inputs(args.config, device=dev)
-    mask_h = None
-    E = c.E
+    mask = None
     if c.prune_lowest:
+        # the one-time prune on the oracle's histogram of a first routing pass
         from oracle import moe_oracle as O
         xr = inp["x"].float().cpu().numpy()
         z = O.router_logits(xr, inp["w_router"].cpu().numpy(), inp["bias"].cpu().numpy())
         idx, _ = O.route_topk(z, c.k)
-        mask_h, _ = O.prune_mask_lowest(O.expert_counts(idx, E), c.prune_lowest, c.k)
-        del xr, z
-    hin = host_inputs(inp, n_tok)
+        mask_np, _ = O.prune_mask_lowest(O.expert_counts(idx, c.E), c.prune_lowest, c.k)
+        mask = torch.as_tensor(np.asarray(mask_np, np.uint8))
+        del xr, z, idx
+    hin, n_exp = sample_inputs(inp, mask, c.k, n_tok)
     del inp
+    if dev == "cuda":
+        torch.cuda.empty_cache()
     for _ in range(args.warmup):
-        oracle_sample(hin, mask_h, c.k, n_tok, backward=c.backward)
+        oracle_sample(hin, c.k, backward=c.backward)
     secs = 0.0
     for _ in range(args.steps):
-        secs += oracle_sample(hin, mask_h, c.k, n_tok, backward=c.backward)
+        secs += oracle_sample(hin, c.k, backward=c.backward)
     v = n_tok * args.steps / secs
     cores = int(os.environ.get("OPENBLAS_NUM_THREADS", NCPU))
+    E_live = c.E - c.prune_lowest
     sample = (f"first {n_tok} of {c.T} tokens per step, full layer "
-              f"{'fwd+bwd' if c.backward else 'forward'} over all {E} experts"
-              + (f" ({c.prune_lowest} least-loaded masked)" if c.prune_lowest else "")
+              f"{'fwd+bwd' if c.backward else 'forward'} with the {n_exp} of {E_live} live "
+              f"experts they are routed to"
+              + (f" ({c.prune_lowest} least-loaded pruned)" if c.prune_lowest else "")
               + ", fp64 numpy oracle")
+    E_held = E_live if c.compact else c.E
     print(json.dumps({
         "impl": "reference", "metric": METRIC, "value": round(v, 3), "unit": "tokens/s",
         "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": round(secs / args.steps * 1e3, 1), "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-        "config": {"workload": c.name, "T": c.T, "d_model": c.d, "experts": c.E, "top_k": c.k,
-                   "d_ff": c.F},
+        "config": workload_config(args, c, c.T, E_held, E_live, c.prune_lowest, c.backward, 1),
         "cpu_baseline": {"value": round(v, 3), "unit": "tokens/s", "cores": cores,
                          "kind": "oracle", "sample": sample},
         "e2e": {"value": round(v, 3), "unit": "tokens/s", "h2d_bytes_per_step": 0,
@@ -726,13 +910,17 @@ def run_reference(args):
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=100)
+    ap.add_argument("--steps", type=int, default=30)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    ap.add_argument("--config", type=int, default=2, choices=sorted(synth.CONFIGS))
-    ap.add_argument("--cpu-tokens", type=int, default=4096)
+    ap.add_argument("--config", type=int, default=4, choices=sorted(synth.CONFIGS),
+                    help="workload (default 4, the largest: T=65536, d_model=7168, 256 -> 171 "
+                         "experts, top-8, d_ff=2048)")
+    ap.add_argument("--cpu-tokens", type=int, default=None,
+                    help="tokens of the CPU-baseline oracle sample (default per workload)")
     ap.add_argument("--ref-tokens", type=int, default=None,
-                    help="tokens per reference-arm step (default: 64 x 30 / steps, 8 to 64)")
+                    help="tokens per reference-arm step (default per workload, fewer at more "
+                         "steps)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-laep", action="store_true",
@@ -755,11 +943,15 @@ def main():
     ap.add_argument("--experts", type=int, default=None)
     ap.add_argument("--no-prune", action="store_true")
     ap.add_argument("--bias", choices=["none", "zipf", "loguniform"], default=None)
+    ap.add_argument("--call", choices=CALL_NAMES, default=None,
+                    help="time this entry point alone (K calls) instead of whole steps")
     args = ap.parse_args()
     if args.warmup < 3 and args.impl == "ours":
         args.warmup = 3
     if args.impl == "reference":
         run_reference(args)
+    elif args.call:
+        run_call(args)
     else:
         run_ours(args)
 

@@ -97,7 +97,13 @@ int moe_timing_read(char *buf, size_t buf_len, int reset);
 int64_t moe_perm_rows_max(int T, int k, int E);
 
 /* Bytes of scratch `ws` every device entry point below may use for a layer of
- * this shape (one buffer serves all calls of a step issued on one stream). */
+ * this shape (one buffer serves all calls of a step issued on one stream).
+ * Its first 256 bytes hold the grouped GEMMs' tile counter: the moe_grouped_ffn_*
+ * entry points need a ws of at least 256 bytes (16-byte aligned) and only use
+ * those; two GEMM calls whose kernels may overlap on the GPU need separate
+ * workspaces. The other calls use disjoint regions after them, so the router
+ * backward and the unpermute-sum may share one workspace with GEMM calls running
+ * beside them on another stream. */
 size_t moe_workspace_size(int T, int d, int E, int k, int F);
 
 /*
@@ -223,9 +229,12 @@ int moe_permute(const uint16_t *x, const int32_t *topk_idx, const int32_t *count
  * Limit: E * ceil(T*k / 4096) <= 65536 (e.g. 256 experts with at most
  * 1,048,576 assignments); larger problems return MOE_ERR_UNSUPPORTED before
  * anything is launched.
- * The first call on a device looks up the array's device address (once per
- * device, with that device current); make that first call before any stream
- * capture. Every GPU that loads the library holds the array until the
+ * The array's device address belongs to the CUDA context that loaded the
+ * library: the first call in each context (the current one of the calling
+ * thread: a device's primary context, another context of the same device, or
+ * the new primary context after cudaDeviceReset) looks it up and caches it under
+ * the context's unique id; make that first call in a context before any stream
+ * capture on it. Every GPU that loads the library holds the array until the
  * process exits. All calls share the one array and it keeps the last call's
  * contents (nothing in it needs to start at zero): calls whose kernels may
  * overlap on the GPU (other streams, other host threads) race on it and must
@@ -249,7 +258,14 @@ int moe_permute_noalloc(const uint16_t *x, const int32_t *topk_idx, const int32_
  * 32-row blocks: element (r, c) at ((r/32)*(2F/8) + c/8)*256 + (r%32)*8 + c%8,
  * so that the 32 rows one warp handles are contiguous), h [rows_cap,F] bf16,
  * out_perm [rows_cap,d] bf16. Only rows below group_offsets[E] are written.
- * Groups of 0 rows cost nothing.
+ * Groups of 0 rows cost nothing. ws: at least 256 bytes, 16-byte aligned (the
+ * tile counter; see moe_workspace_size).
+ * Schedule (all moe_grouped_ffn_* GEMMs): the tiles are listed heaviest expert
+ * first, the longest-processing-time order of Algorithm 2's greedy; CTA pairs
+ * that run out of work take the next tile of the list from a shared counter, so
+ * the heaviest tile left always goes to the least-loaded pair (Algorithm 2 with
+ * the GPU's CTA pairs as its devices, applied online). A tile's arithmetic does
+ * not depend on which pair runs it: results are bitwise reproducible.
  * Limits: d % 128 == 0, F % 128 == 0, all pointers 16-byte aligned.
  */
 int moe_grouped_ffn_fwd(const uint16_t *x_perm, const int32_t *group_offsets, int E, int d,
@@ -324,7 +340,11 @@ int moe_grouped_ffn_fwd_gather(const uint16_t *x, const int32_t *token_of_row, i
                                moe_stream_t stream);
 
 /*
- * moe_unpermute_combine - gate-weighted combine back to token order:
+ * moe_unpermute_combine - gate-weighted combine back to token order: the
+ * layer's output sums, for every token, the outputs of the experts its routing
+ * indicator selects (E[i,j,l] = 1, Sec. 3.2), weighted by the gates; the dispatch
+ * of Sec. 3.3 in reverse (the paper names the MoE layer but prints no combine
+ * formula; the gates are the softmax over the selected experts of moe_route):
  *   y[t,:] = sum_j topk_gate[t,j] * out_perm[row_of_assignment[t,j], :]
  * summed in fp32, rounded once to bf16. out_perm [rows_cap,d] bf16;
  * row_of_assignment [T,k]; topk_gate [T,k] fp32; y [T,d] bf16. d % 8 == 0.
@@ -334,7 +354,8 @@ int moe_unpermute_combine(const uint16_t *out_perm, const int32_t *row_of_assign
                           moe_stream_t stream);
 
 /*
- * moe_unpermute_combine_bwd - backward of the combine:
+ * moe_unpermute_combine_bwd - backward of the combine (the paper gives no
+ * backward; this is the derivative of moe_unpermute_combine):
  *   d_out_perm[row(t,j), :] = topk_gate[t,j] * dy[t, :]   (bf16)
  *   d_gate[t,j] = <dy[t,:], out_perm[row(t,j),:]>         (fp32)
  * and zeroes the padding rows of d_out_perm (group_offsets/group_counts from
@@ -352,39 +373,50 @@ int moe_unpermute_combine_bwd(const uint16_t *dy, const uint16_t *out_perm,
                               float *d_gate, moe_stream_t stream);
 
 /*
- * moe_grouped_ffn_bwd - backward of moe_grouped_ffn_fwd (dgrad and wgrad):
+ * moe_grouped_ffn_bwd - backward of moe_grouped_ffn_fwd (dgrad and wgrad) for
+ * the three-matrix SwiGLU expert of Table A1 (the paper gives no backward; this
+ * is the derivative of moe_grouped_ffn_fwd):
  *   dH_e = dO_e * W_down[e];  dA_e = dH_e * B_e * silu'(A_e);
  *   dB_e = dH_e * silu(A_e);  dX_e = [dA_e | dB_e] * W_gate_up[e]
  *   dW_down[e] = dO_e^T * H_e;  dW_gate_up[e] = [dA_e | dB_e]^T * X_e
- * Experts whose group is empty get exactly zero weight gradients.
+ * active_mask [E] uint8 or NULL (all live): the LAEP mask the routing used. A
+ * pruned expert (active_mask[e] == 0) is removed from the model (Sec. 4,
+ * Table 5), so it has no weight gradient: its dw_gate_up[e] and dw_down[e] are
+ * not written and keep what the caller left there. A live expert whose group is
+ * empty gets exactly zero weight gradients.
  * d_out_perm [rows_cap,d] (padding rows zero); x_perm, ab_saved, h from the
  * forward; d_ab [rows_cap,2F] bf16 caller scratch (receives [dA|dB]);
  * outputs dx_perm [rows_cap,d] bf16, dw_gate_up [E,2F,d] bf16,
- * dw_down [E,d,F] bf16 (fp32 accumulation). Limits as in the forward.
+ * dw_down [E,d,F] bf16 (fp32 accumulation). ws as in moe_grouped_ffn_fwd.
+ * Limits as in the forward.
  */
 int moe_grouped_ffn_bwd(const uint16_t *d_out_perm, const uint16_t *x_perm,
                         const uint16_t *ab_saved, const uint16_t *h,
-                        const int32_t *group_offsets, int E, int d, int F, int64_t rows_cap,
-                        const uint16_t *w_gate_up, const uint16_t *w_down, uint16_t *d_ab,
-                        uint16_t *dx_perm, uint16_t *dw_gate_up, uint16_t *dw_down, void *ws,
-                        size_t ws_bytes, moe_stream_t stream);
+                        const int32_t *group_offsets, const uint8_t *active_mask, int E, int d,
+                        int F, int64_t rows_cap, const uint16_t *w_gate_up,
+                        const uint16_t *w_down, uint16_t *d_ab, uint16_t *dx_perm,
+                        uint16_t *dw_gate_up, uint16_t *dw_down, void *ws, size_t ws_bytes,
+                        moe_stream_t stream);
 
 /*
  * moe_grouped_ffn_bwd_dgrad / moe_grouped_ffn_bwd_wgrad - the two halves of
  * moe_grouped_ffn_bwd (which calls them in this order on one stream), for
- * callers that overlap other work with the weight gradients:
+ * callers that overlap other work with the weight gradients (the derivative of
+ * Table A1's three-matrix expert; the paper gives no backward):
  *   dgrad: dH = dO W_down, [dA|dB] (into d_ab), dX = [dA|dB] W_gate_up
- *   wgrad: dW_down = dO^T H, dW_gate_up = [dA|dB]^T X  (needs d_ab from dgrad)
+ *   wgrad: dW_down = dO^T H, dW_gate_up = [dA|dB]^T X  (needs d_ab from dgrad;
+ *          pruned experts of active_mask are not written)
  * Arguments as in moe_grouped_ffn_bwd.
  */
 int moe_grouped_ffn_bwd_dgrad(const uint16_t *d_out_perm, const uint16_t *ab_saved,
                               const int32_t *group_offsets, int E, int d, int F, int64_t rows_cap,
                               const uint16_t *w_gate_up, const uint16_t *w_down, uint16_t *d_ab,
-                              uint16_t *dx_perm, moe_stream_t stream);
+                              uint16_t *dx_perm, void *ws, size_t ws_bytes, moe_stream_t stream);
 int moe_grouped_ffn_bwd_wgrad(const uint16_t *d_out_perm, const uint16_t *x_perm,
                               const uint16_t *h, const uint16_t *d_ab,
-                              const int32_t *group_offsets, int E, int d, int F, int64_t rows_cap,
-                              uint16_t *dw_gate_up, uint16_t *dw_down, moe_stream_t stream);
+                              const int32_t *group_offsets, const uint8_t *active_mask, int E,
+                              int d, int F, int64_t rows_cap, uint16_t *dw_gate_up,
+                              uint16_t *dw_down, void *ws, size_t ws_bytes, moe_stream_t stream);
 
 /*
  * moe_grouped_ffn_bwd_wgrad_gather - moe_grouped_ffn_bwd_wgrad with X_e read
@@ -393,9 +425,10 @@ int moe_grouped_ffn_bwd_wgrad(const uint16_t *d_out_perm, const uint16_t *x_perm
  */
 int moe_grouped_ffn_bwd_wgrad_gather(const uint16_t *d_out_perm, const uint16_t *x,
                                      const int32_t *token_of_row, int T, const uint16_t *h,
-                                     const uint16_t *d_ab, const int32_t *group_offsets, int E,
-                                     int d, int F, int64_t rows_cap, uint16_t *dw_gate_up,
-                                     uint16_t *dw_down, moe_stream_t stream);
+                                     const uint16_t *d_ab, const int32_t *group_offsets,
+                                     const uint8_t *active_mask, int E, int d, int F,
+                                     int64_t rows_cap, uint16_t *dw_gate_up, uint16_t *dw_down,
+                                     void *ws, size_t ws_bytes, moe_stream_t stream);
 
 /*
  * moe_route_bwd - backward of the router's softmax over the selected experts
@@ -416,7 +449,11 @@ int moe_route_bwd(const uint16_t *x, const int32_t *topk_idx, const float *topk_
                   float *dw_router, void *ws, size_t ws_bytes, moe_stream_t stream);
 
 /*
- * moe_permute_bwd - gradient of the layer input:
+ * moe_permute_bwd - gradient of the layer input (the paper gives no backward;
+ * this is the derivative of moe_permute's gather x_perm[row(t,j)] = x[t], the
+ * dispatch of Sec. 3.3 that sends each token to the experts its routing
+ * indicator E[i,j,l] selects (Sec. 3.2), plus the router's term from
+ * moe_route_bwd's d_logits):
  *   dx[t,:] = sum_j dx_perm[row(t,j), :] + sum_j d_logits[t,j] * w_router[:, e_j]
  * summed in fp32, one bf16 rounding. d_logits and w_router may both be NULL
  * (no router term). dx [T,d] bf16 (out).

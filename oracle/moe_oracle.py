@@ -373,31 +373,65 @@ def token_backward(dy_t, x_t, experts, gates_t, w_router, w_gate_up, w_down):
     return dx, dgate, dz
 
 
+def tokens_forward_backward(x_rows, experts, gates, dy_rows, w_router, w_gate_up, w_down):
+    """y, dx, d_gate and d_logits of a set of tokens from their selected experts and gates
+    (fp64): the definitions of token_forward / token_backward (and of moe_forward /
+    moe_backward restricted to these tokens), evaluated expert by expert so that each
+    expert's weights are read once for all the tokens routed to it.
+
+    x_rows, dy_rows [n, d]; experts [n, k] (distinct per token); gates [n, k].
+    Returns (y [n, d], dx [n, d], d_gate [n, k], d_logits [n, k]).
+    """
+    x = np.asarray(x_rows, np.float64)
+    dy = np.asarray(dy_rows, np.float64)
+    g = np.asarray(gates, np.float64)
+    experts = np.asarray(experts)
+    n, d = x.shape
+    k = experts.shape[1]
+    F = w_gate_up.shape[1] // 2
+    o = np.zeros((n, k, d))
+    dx = np.zeros((n, d))
+    for e in np.unique(experts):
+        t, j = np.nonzero(experts == e)  # each token at most once per expert
+        wg = np.asarray(w_gate_up[e, :F], np.float64)
+        wu = np.asarray(w_gate_up[e, F:], np.float64)
+        wd = np.asarray(w_down[e], np.float64)
+        xe = x[t]
+        ae = xe @ wg.T
+        be = xe @ wu.T
+        o[t, j] = (silu(ae) * be) @ wd.T
+        dh = (g[t, j][:, None] * dy[t]) @ wd
+        dx[t] += (dh * be * silu_grad(ae)) @ wg + (dh * silu(ae)) @ wu
+    y = np.einsum("tj,tjd->td", g, o)
+    d_gate = np.einsum("td,tjd->tj", dy, o)
+    dz = g * (d_gate - np.sum(g * d_gate, axis=1, keepdims=True))
+    dx += np.einsum("tj,dtj->td", dz, np.asarray(w_router, np.float64)[:, experts])
+    return y, dx, d_gate, dz
+
+
 def expert_weight_grad_columns(e, feats, x_rows, dy_rows, gates_rows, w_gate_up, w_down):
     """Selected feature slices of expert e's weight gradients (fp64).
 
     x_rows, dy_rows, gates_rows: the token inputs, upstream gradients and gates
     of every assignment routed to e. For each feature f in `feats` returns
     dWd[:, f] (length d), dWg[f, :] and dWu[f, :] (length d) as arrays
-    [len(feats), d].
+    [len(feats), d]. The features are evaluated together: a, b, h and dH are
+    [rows, len(feats)] matrices.
     """
     X = np.asarray(x_rows, np.float64)
     dY = np.asarray(dy_rows, np.float64)
     g = np.asarray(gates_rows, np.float64)
     F = w_gate_up.shape[1] // 2
+    feats = np.asarray(feats)
     wd = np.asarray(w_down[e], np.float64)
     d_o = g[:, None] * dY
-    dwd = np.zeros((len(feats), X.shape[1]))
-    dwg = np.zeros_like(dwd)
-    dwu = np.zeros_like(dwd)
-    for i, f in enumerate(feats):
-        a = X @ np.asarray(w_gate_up[e, f], np.float64)
-        b = X @ np.asarray(w_gate_up[e, F + f], np.float64)
-        h = silu(a) * b
-        dh = d_o @ wd[:, f]
-        dwd[i] = d_o.T @ h
-        dwg[i] = (dh * b * silu_grad(a)) @ X
-        dwu[i] = (dh * silu(a)) @ X
+    a = X @ np.asarray(w_gate_up[e, feats], np.float64).T
+    b = X @ np.asarray(w_gate_up[e, F + feats], np.float64).T
+    h = silu(a) * b
+    dh = d_o @ wd[:, feats]
+    dwd = h.T @ d_o
+    dwg = (dh * b * silu_grad(a)).T @ X
+    dwu = (dh * silu(a)).T @ X
     return dwd, dwg, dwu
 
 

@@ -54,15 +54,16 @@ _SIGS = {
     "moe_grouped_ffn_fwd": (I, [P, P, I, I, I, I64, P, P, P, P, P, P, SZ, P]),
     "moe_unpermute_combine": (I, [P, P, P, I, I, I, P, P]),
     "moe_unpermute_combine_bwd": (I, [P, P, P, P, P, P, I, I, I, I, P, P, P]),
-    "moe_grouped_ffn_bwd": (I, [P, P, P, P, P, I, I, I, I64, P, P, P, P, P, P, P, SZ, P]),
-    "moe_grouped_ffn_bwd_dgrad": (I, [P, P, P, I, I, I, I64, P, P, P, P, P]),
-    "moe_grouped_ffn_bwd_wgrad": (I, [P, P, P, P, P, I, I, I, I64, P, P, P]),
+    "moe_grouped_ffn_bwd": (I, [P, P, P, P, P, P, I, I, I, I64, P, P, P, P, P, P, P, SZ, P]),
+    "moe_grouped_ffn_bwd_dgrad": (I, [P, P, P, I, I, I, I64, P, P, P, P, P, SZ, P]),
+    "moe_grouped_ffn_bwd_wgrad": (I, [P, P, P, P, P, P, I, I, I, I64, P, P, P, SZ, P]),
     "moe_route_bwd": (I, [P, P, P, P, I, I, I, I, P, P, P, SZ, P]),
     "moe_permute_bwd": (I, [P, P, P, P, P, I, I, I, I, P, P, SZ, P]),
     "moe_permute_map": (I, [P, P, I, I, I, I64, P, P, P, P, P, SZ, P]),
     "moe_grouped_ffn_fwd_combine": (I, [P, P, I, I, I, I64, P, P, P, P, I, I, P, P, P, P, P, P, SZ, P]),
     "moe_grouped_ffn_fwd_gather": (I, [P, P, I, P, I, I, I, I64, P, P, P, P, P, P, SZ, P]),
-    "moe_grouped_ffn_bwd_wgrad_gather": (I, [P, P, P, I, P, P, P, I, I, I, I64, P, P, P]),
+    "moe_grouped_ffn_bwd_wgrad_gather": (I, [P, P, P, I, P, P, P, P, I, I, I, I64, P, P, P, SZ,
+                                             P]),
     "moe_selftest_wait_timeout": (I, [I64, P]),
 }
 
@@ -242,27 +243,29 @@ def moe_unpermute_combine_bwd(dy, out_perm, row_of_assignment, topk_gate, group_
         _ptr(group_counts), T, d, E, k, _ptr(d_out_perm), _ptr(d_gate), _stream(stream)))
 
 
-def moe_grouped_ffn_bwd(d_out_perm, x_perm, ab_saved, h, group_offsets, E, d, F, rows_cap,
-                        w_gate_up, w_down, d_ab, dx_perm, dw_gate_up, dw_down, ws, ws_bytes,
-                        stream=None):
+def moe_grouped_ffn_bwd(d_out_perm, x_perm, ab_saved, h, group_offsets, active_mask, E, d, F,
+                        rows_cap, w_gate_up, w_down, d_ab, dx_perm, dw_gate_up, dw_down, ws,
+                        ws_bytes, stream=None):
     _check("moe_grouped_ffn_bwd", load().moe_grouped_ffn_bwd(
-        _ptr(d_out_perm), _ptr(x_perm), _ptr(ab_saved), _ptr(h), _ptr(group_offsets), E, d, F,
-        rows_cap, _ptr(w_gate_up), _ptr(w_down), _ptr(d_ab), _ptr(dx_perm), _ptr(dw_gate_up),
-        _ptr(dw_down), _ptr(ws), ws_bytes, _stream(stream)))
+        _ptr(d_out_perm), _ptr(x_perm), _ptr(ab_saved), _ptr(h), _ptr(group_offsets),
+        _ptr(active_mask), E, d, F, rows_cap, _ptr(w_gate_up), _ptr(w_down), _ptr(d_ab),
+        _ptr(dx_perm), _ptr(dw_gate_up), _ptr(dw_down), _ptr(ws), ws_bytes, _stream(stream)))
 
 
 def moe_grouped_ffn_bwd_dgrad(d_out_perm, ab_saved, group_offsets, E, d, F, rows_cap, w_gate_up,
-                              w_down, d_ab, dx_perm, stream=None):
+                              w_down, d_ab, dx_perm, ws, ws_bytes, stream=None):
     _check("moe_grouped_ffn_bwd_dgrad", load().moe_grouped_ffn_bwd_dgrad(
         _ptr(d_out_perm), _ptr(ab_saved), _ptr(group_offsets), E, d, F, rows_cap,
-        _ptr(w_gate_up), _ptr(w_down), _ptr(d_ab), _ptr(dx_perm), _stream(stream)))
+        _ptr(w_gate_up), _ptr(w_down), _ptr(d_ab), _ptr(dx_perm), _ptr(ws), ws_bytes,
+        _stream(stream)))
 
 
-def moe_grouped_ffn_bwd_wgrad(d_out_perm, x_perm, h, d_ab, group_offsets, E, d, F, rows_cap,
-                              dw_gate_up, dw_down, stream=None):
+def moe_grouped_ffn_bwd_wgrad(d_out_perm, x_perm, h, d_ab, group_offsets, active_mask, E, d, F,
+                              rows_cap, dw_gate_up, dw_down, ws, ws_bytes, stream=None):
     _check("moe_grouped_ffn_bwd_wgrad", load().moe_grouped_ffn_bwd_wgrad(
-        _ptr(d_out_perm), _ptr(x_perm), _ptr(h), _ptr(d_ab), _ptr(group_offsets), E, d, F,
-        rows_cap, _ptr(dw_gate_up), _ptr(dw_down), _stream(stream)))
+        _ptr(d_out_perm), _ptr(x_perm), _ptr(h), _ptr(d_ab), _ptr(group_offsets),
+        _ptr(active_mask), E, d, F, rows_cap, _ptr(dw_gate_up), _ptr(dw_down), _ptr(ws),
+        ws_bytes, _stream(stream)))
 
 
 def moe_route_bwd(x, topk_idx, topk_gate, d_gate, T, d, E, k, d_logits, dw_router, ws, ws_bytes,
@@ -296,11 +299,13 @@ def moe_grouped_ffn_fwd_gather(x, token_of_row, T, group_offsets, E, d, F, rows_
         _stream(stream)))
 
 
-def moe_grouped_ffn_bwd_wgrad_gather(d_out_perm, x, token_of_row, T, h, d_ab, group_offsets, E,
-                                     d, F, rows_cap, dw_gate_up, dw_down, stream=None):
+def moe_grouped_ffn_bwd_wgrad_gather(d_out_perm, x, token_of_row, T, h, d_ab, group_offsets,
+                                     active_mask, E, d, F, rows_cap, dw_gate_up, dw_down, ws,
+                                     ws_bytes, stream=None):
     _check("moe_grouped_ffn_bwd_wgrad_gather", load().moe_grouped_ffn_bwd_wgrad_gather(
         _ptr(d_out_perm), _ptr(x), _ptr(token_of_row), T, _ptr(h), _ptr(d_ab),
-        _ptr(group_offsets), E, d, F, rows_cap, _ptr(dw_gate_up), _ptr(dw_down), _stream(stream)))
+        _ptr(group_offsets), _ptr(active_mask), E, d, F, rows_cap, _ptr(dw_gate_up),
+        _ptr(dw_down), _ptr(ws), ws_bytes, _stream(stream)))
 
 
 def moe_permute_bwd(dx_perm, row_of_assignment, topk_idx, d_logits, w_router, T, d, E, k, dx,

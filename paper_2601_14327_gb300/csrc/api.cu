@@ -104,6 +104,8 @@ WsLayout ws_layout(int T, int d, int E, int k, int F) {
   const int64_t A = int64_t(T) * k;
   const int64_t nblk = std::max<int64_t>(1, (A + kPermChunk - 1) / kPermChunk);
   size_t off = 0;
+  w.gemm_sched = off;
+  off += kGemmSchedBytes;
   w.perm_hist = off;
   off += align256(size_t(E) * nblk * 4);
   w.route_dz3 = off;

@@ -26,8 +26,13 @@ inline bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 
 
 int num_sms();
 
+// The first bytes of every workspace belong to the grouped GEMMs' tile scheduler
+// (their entry points know neither T nor k, so the region has a fixed offset and size).
+constexpr size_t kGemmSchedBytes = 256;
+
 // Workspace layout shared by the entry points (disjoint regions, 256-byte aligned).
 struct WsLayout {
+  size_t gemm_sched;    // int32 [1]               grouped GEMM tile counter (offset 0)
   size_t perm_hist;     // int32 [E * nblk]        moe_permute block histograms
   size_t route_dz3;     // bf16  [3, NP, Tp]       moe_route_bwd logit gradient as three bf16 terms
   size_t route_dw_partial; // fp32 [splits, d, NE] moe_route_bwd split-reduction partial sums

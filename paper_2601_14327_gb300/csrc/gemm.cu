@@ -91,6 +91,13 @@ struct GemmParams {
   float *y_acc;
   const int32_t *row_token;
   const float *row_gate;
+  // Weight-gradient modes: experts with active_mask[e] == 0 (pruned by LAEP) get no tile
+  // and no store; their gradient buffers are left as they are (nullptr: all experts live).
+  const uint8_t *active_mask;
+  // CTA-pair kernel: tile counter of the dynamic schedule (zero at launch, 4 bytes of the
+  // caller's workspace); dynamic = 0 walks the list with a fixed stride instead.
+  int *sched_ctr;
+  int dynamic;
 };
 
 struct Tile {
@@ -359,29 +366,32 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc::tmem_relinquish();
   }
   // ---- tile schedule, built from the device-resident group offsets ----
+  // Experts heaviest first (ties to the lower id); in the weight-gradient modes pruned
+  // experts (active_mask 0) come last with no tile, live experts without rows get tiles
+  // of zero k-blocks (their zero gradient).
   for (int e = threadIdx.x; e <= E; e += kThreads) s_goff[e] = p.group_offsets[e];
   __syncthreads();
-  if (Tr::WGRAD) {
-    for (int e = threadIdx.x; e < E; e += kThreads) {
-      const int ce = s_goff[e + 1] - s_goff[e];
-      int r = 0;
-      for (int q = 0; q < E; ++q) {
-        const int cq = s_goff[q + 1] - s_goff[q];
-        r += (cq > ce) || (cq == ce && q < e);
-      }
-      s_order[r] = e;
+  auto sort_key = [&](int e) {
+    const int rows = s_goff[e + 1] - s_goff[e];
+    return (Tr::WGRAD && p.active_mask != nullptr && p.active_mask[e] == 0) ? -1 : rows;
+  };
+  for (int e = threadIdx.x; e < E; e += kThreads) {
+    const int ce = sort_key(e);
+    int r = 0;
+    for (int q = 0; q < E; ++q) {
+      const int cq = sort_key(q);
+      r += (cq > ce) || (cq == ce && q < e);
     }
-  } else {
-    for (int e = threadIdx.x; e < E; e += kThreads) s_order[e] = e;
+    s_order[r] = e;
   }
   __syncthreads();
   if (threadIdx.x == 0) {
     int acc = 0;
     for (int i = 0; i < E; ++i) {
       s_prefix[i] = acc;
-      const int e = s_order[i];
-      const int rows = s_goff[e + 1] - s_goff[e];
-      acc += Tr::WGRAD ? p.m_tiles_w * p.n_tiles : (rows / BM) * p.n_tiles;
+      const int key = sort_key(s_order[i]);
+      if (key < 0) continue;  // pruned
+      acc += Tr::WGRAD ? p.m_tiles_w * p.n_tiles : (key / BM) * p.n_tiles;
     }
     s_prefix[E] = acc;
   }
@@ -560,15 +570,24 @@ __global__ void __launch_bounds__(kThreads, 1)
 // operand, K-half h at h * 16 KB of A and h * BNH * 128 bytes of B), or 64 for the
 // gathered-operand variant. Deeper stages halve the barrier waits, descriptor setup and
 // commits per FLOP (measured -2.5% to -4.4% cycles per k-block) at the same bytes in flight.
+// Tile hand-off ring of the CTA-pair kernel: the even CTA's producer claims tiles and
+// publishes each one in a slot of both CTAs' rings; the odd CTA's producer and the MMA
+// issuer read it there. A slot is rewritten kRing tiles later, which the load ring's
+// STAGES (< kRing) bound: a producer can run at most STAGES k-blocks, hence STAGES tiles,
+// ahead of the MMAs that need the other readers' progress.
+constexpr int kRing = 16;
+
 template <int BN, int KB> struct PairShape {
   static constexpr int BNH = BN / 2;  // B rows staged by each CTA
   static constexpr int STAGES = KB == 128 ? (BN == 256 ? 3 : 4) : (BN == 256 ? 6 : 8);
+  static_assert(STAGES + 1 < kRing, "the tile ring must outlast the load ring");
   static constexpr uint32_t A_BYTES = BM * KB * 2;
   static constexpr uint32_t B_BYTES = BNH * KB * 2;
   static constexpr uint32_t STAGE_BYTES = A_BYTES + B_BYTES;
-  static constexpr int NBARS = 2 * STAGES + 5;
+  // full/empty per stage, tfull/tempty per accumulator, drain, tile ring, epilogue tile
+  static constexpr int NBARS = 2 * STAGES + 5 + kRing + 2;
   static constexpr size_t SMEM = 1024 + size_t(STAGES) * STAGE_BYTES + NBARS * 8 +
-                                 (4 + 257 + 256 + 257) * 4 + 1024 + kEpiWarps * 2048;
+                                 (4 + 257 + 256 + 257 + kRing + 2) * 4 + 1024 + kEpiWarps * 2048;
   static constexpr uint32_t TMEM_COLS = 2 * BN;
 };
 
@@ -611,8 +630,10 @@ __global__ void __launch_bounds__(kThreads, 1)
   int *s_goff = misc + 4;
   int *s_order = s_goff + 257;
   int *s_prefix = s_order + 256;
+  volatile int *s_ring = s_prefix + 257;  // [kRing] tile hand-off (see kRing)
+  volatile int *s_epi = s_ring + kRing;   // [2] tile of each accumulator buffer, for the epilogue
   const uint32_t stage_base =
-      (tc::smem_u32(s_prefix + 257) + 1023u) & ~1023u;  // epilogue staging, 2 KB per warp
+      (tc::smem_u32(const_cast<int *>(s_epi + 2)) + 1023u) & ~1023u;  // epilogue staging, 2 KB per warp
   volatile int *abort_flag = misc + 1;
   volatile int no_abort = 0;
 
@@ -622,6 +643,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   auto tfull_bar = [&](int a) { return bar0 + 8u * (2 * STAGES + a); };
   auto tempty_bar = [&](int a) { return bar0 + 8u * (2 * STAGES + 2 + a); };
   const uint32_t drain_bar = bar0 + 8u * (2 * STAGES + 4);
+  auto ring_bar = [&](int r) { return bar0 + 8u * (2 * STAGES + 5 + r); };
+  auto epi_bar = [&](int a) { return bar0 + 8u * (2 * STAGES + 5 + kRing + a); };
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int E = p.E;
@@ -638,7 +661,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int a = 0; a < 2; ++a) {
       tc::mbar_init(tfull_bar(a), 1);
       tc::mbar_init(tempty_bar(a), 2 * kEpiWarps);  // the epilogue warps of both CTAs
+      tc::mbar_init(epi_bar(a), 1);                 // the even CTA's MMA issuer
     }
+    for (int r = 0; r < kRing; ++r) tc::mbar_init(ring_bar(r), 1);  // the even CTA's producer
     tc::mbar_init(drain_bar, 1);
     tc::fence_mbar_init();
     misc[1] = 0;
@@ -652,41 +677,45 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc::tmem_alloc_pair(tc::smem_u32(misc), Sh::TMEM_COLS);
     tc::tmem_relinquish_pair();
   }
-  // ---- tile schedule: identical in both CTAs of every pair ----
+  // ---- tile list: identical in both CTAs of every pair ----
+  // Experts in descending order of rows (ties to the lower id): the longest-processing-
+  // time order of Algorithm 2's greedy balancing. A pair that runs out of work claims the
+  // next tile of this list, i.e. the heaviest tile left goes to the least-loaded pair.
+  // Weight gradients: pruned experts (active_mask 0) come last and get nothing; live
+  // experts without rows come before them and get no tile either (their zero gradients
+  // are stored by the epilogue warps up front, while the first tiles' MMAs run).
   for (int e = threadIdx.x; e <= E; e += kThreads) s_goff[e] = p.group_offsets[e];
   __syncthreads();
-  if (Tr::WGRAD) {
-    for (int e = threadIdx.x; e < E; e += kThreads) {
-      const int ce = s_goff[e + 1] - s_goff[e];
-      int r = 0;
-      for (int q = 0; q < E; ++q) {
-        const int cq = s_goff[q + 1] - s_goff[q];
-        r += (cq > ce) || (cq == ce && q < e);
-      }
-      s_order[r] = e;
+  auto sort_key = [&](int e) {
+    const int rows = s_goff[e + 1] - s_goff[e];
+    return (Tr::WGRAD && p.active_mask != nullptr && p.active_mask[e] == 0) ? -1 : rows;
+  };
+  for (int e = threadIdx.x; e < E; e += kThreads) {
+    const int ce = sort_key(e);
+    int r = 0;
+    for (int q = 0; q < E; ++q) {
+      const int cq = sort_key(q);
+      r += (cq > ce) || (cq == ce && q < e);
     }
-  } else {
-    for (int e = threadIdx.x; e < E; e += kThreads) s_order[e] = e;
+    s_order[r] = e;
   }
   __syncthreads();
   if (threadIdx.x == 0) {
-    // Weight gradients: experts without rows get no tile in the list (they come last
-    // in the heaviest-first order); their zero gradients are stored by the epilogue
-    // warps up front instead, while the first tiles' MMAs run (misc[2] = their count).
-    int acc = 0, n_empty = 0;
+    int acc = 0, n_empty = 0, n_pruned = 0;
     for (int i = 0; i < E; ++i) {
       s_prefix[i] = acc;
       const int e = s_order[i];
-      const int rows = s_goff[e + 1] - s_goff[e];
-      if (Tr::WGRAD && rows == 0) {
-        ++n_empty;
+      const int key = sort_key(e);
+      if (Tr::WGRAD && key <= 0) {
+        if (key < 0) ++n_pruned; else ++n_empty;
         continue;
       }
-      const int mt = Tr::WGRAD ? p.m_tiles_w : rows / BM;
+      const int mt = Tr::WGRAD ? p.m_tiles_w : key / BM;
       acc += ((mt + 1) / 2) * p.n_tiles;
     }
     s_prefix[E] = acc;
     misc[2] = n_empty;
+    misc[3] = n_pruned;
   }
   tc::fence_before_sync();
   __syncthreads();
@@ -713,13 +742,46 @@ __global__ void __launch_bounds__(kThreads, 1)
     return t;
   };
 
+  // ---- tile hand-off. The even CTA's producer takes tile number n of this pair: the
+  // pair's index for n = 0, then the next unclaimed tile of the list (an atomic counter
+  // shared by all pairs; p.dynamic == 0: every nclusters-th tile), -1 once the list is
+  // exhausted. It writes the tile into slot n % kRing of both CTAs' rings and arrives on
+  // the slots' barriers before it issues the tile's loads; the odd CTA's producer and
+  // the MMA issuer wait there. The MMA issuer passes each tile on to both CTAs' epilogue
+  // warps through s_epi[buffer] and epi_bar[buffer] once that accumulator buffer is free.
+  const uint32_t ring_peer = tc::mapa(tc::smem_u32(const_cast<int *>(s_ring)), 1);
+  const uint32_t ring_bar_peer = tc::mapa(ring_bar(0), 1);
+  int claimed = cluster;  // even CTA's producer: the tile it publishes next
+  // Returns this pair's tile number n (-1: no more), or -2 after a failed wait.
+  auto next_tile = [&](uint32_t n) -> int {
+    const int slot = int(n % kRing);
+    if (leader) {
+      const int v = claimed < total ? claimed : -1;
+      s_ring[slot] = v;
+      tc::st_cluster_u32(ring_peer + 4u * slot, v);
+      tc::mbar_arrive(ring_bar(slot));
+      tc::mbar_arrive_cluster(ring_bar_peer + 8u * slot);
+      if (v >= 0) claimed = p.dynamic ? nclusters + atomicAdd(p.sched_ctr, 1) : claimed + nclusters;
+      return v;
+    }
+    if (!tc::mbar_wait_cluster(ring_bar(slot), (n / kRing) & 1u, kWaitLimitNs, abort_flag)) {
+      fail(abort_flag);
+      return -2;
+    }
+    return s_ring[slot];
+  };
+
   if (warp == 0 && GATHER) {
     // ============ TMA producer, gathered operand (the whole warp in each CTA) ============
     const uint32_t full_leader = tc::mapa(full_bar(0), 0);
     const int box = lane >> 4, grp = lane & 15;  // kWgradGateUp: B box and 4-row group
     uint32_t it = 0;
     bool ok = true;
-    for (int tile = cluster; tile < total && ok; tile += nclusters) {
+    for (uint32_t n = 0; ok; ++n) {
+      int tile = 0;
+      if (lane == 0) tile = next_tile(n);
+      tile = __shfl_sync(0xffffffffu, tile, 0);
+      if (tile < 0) break;
       const PairTile t = decode(tile);
       const int mt = 2 * t.mp + int(rank);
       int4 rows4 = make_int4(0, 0, 0, 0), nxt = make_int4(0, 0, 0, 0);
@@ -781,7 +843,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       const uint32_t full_leader = tc::mapa(full_bar(0), 0);
       uint32_t it = 0;
       bool ok = true;
-      for (int tile = cluster; tile < total && ok; tile += nclusters) {
+      for (uint32_t n = 0; ok; ++n) {
+        const int tile = next_tile(n);
+        if (tile < 0) break;
         const PairTile t = decode(tile);
         const int mt = 2 * t.mp + int(rank);  // this CTA's 128-row block
         for (int kb = 0; kb < t.nkb; ++kb, ++it) {
@@ -832,14 +896,24 @@ __global__ void __launch_bounds__(kThreads, 1)
   } else if (warp == 1) {
     // ============ MMA issuer (one thread of the even CTA) ============
     if (leader && lane == 0) {
-      uint32_t it = 0, tcount = 0;
+      const uint32_t epi_peer = tc::mapa(tc::smem_u32(const_cast<int *>(s_epi)), 1);
+      const uint32_t epi_bar_peer = tc::mapa(epi_bar(0), 1);
+      uint32_t it = 0;
       bool ok = true, issued = false;
-      for (int tile = cluster; tile < total && ok; tile += nclusters) {
-        const PairTile t = decode(tile);
-        if (t.nkb == 0) continue;
-        const uint32_t a = tcount & 1u, aph = (tcount >> 1) & 1u;
+      for (uint32_t n = 0; ok; ++n) {
+        const int slot = int(n % kRing);
+        if (!tc::mbar_wait(ring_bar(slot), (n / kRing) & 1u, kWaitLimitNs, abort_flag)) { fail(abort_flag); break; }
+        const int tile = s_ring[slot];
+        const uint32_t a = n & 1u, aph = (n >> 1) & 1u;
         if (!tc::mbar_wait(tempty_bar(a), aph ^ 1u, kWaitLimitNs, abort_flag)) { fail(abort_flag); break; }
+        // the epilogue warps of both CTAs learn the tile of buffer a (-1: no more tiles)
+        s_epi[a] = tile;
+        tc::st_cluster_u32(epi_peer + 4u * a, tile);
+        tc::mbar_arrive(epi_bar(a));
+        tc::mbar_arrive_cluster(epi_bar_peer + 8u * a);
+        if (tile < 0) break;
         tc::fence_after_sync();
+        const PairTile t = decode(tile);
         const uint32_t d_tmem = tmem_base + a * BN;
         for (int kb = 0; kb < t.nkb; ++kb, ++it) {
           const int s = it % STAGES;
@@ -863,7 +937,6 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         if (!ok) break;
         tc::mma_commit_pair_mc(tfull_bar(a), 0x3);  // both halves of the accumulator ready
-        ++tcount;
       }
       if (issued) {
         tc::mma_commit_pair(drain_bar);
@@ -878,29 +951,33 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int r_in_tile = q * 32 + lane;
     const uint32_t tempty_leader = tc::mapa(tempty_bar(0), 0);
     if (Tr::WGRAD) {
-      // Experts without rows: their weight gradient is exactly zero. Units of 128 rows
-      // x BN columns, spread over all CTAs; every store reads the same zeroed chunk.
-      const int n_empty = misc[2];
+      // Live experts without rows: their weight gradient is exactly zero. Units of 128
+      // rows x BN columns, spread over all CTAs; every store reads the same zeroed chunk.
+      const int n_empty = misc[2], n_pruned = misc[3];
       const int per_e = p.m_tiles_w * p.n_tiles;
       const int units = n_empty * per_e;
       if (int(blockIdx.x) < units) {
         const int M_out = p.m_tiles_w * BM;
         zero_fill_stage(stage, lane);
         for (int u = int(blockIdx.x); u < units; u += int(gridDim.x)) {
-          const int e = s_order[E - n_empty + u / per_e];
+          const int e = s_order[E - n_pruned - n_empty + u / per_e];
           const int rem = u % per_e;
           const int mb = rem / p.n_tiles, nt = rem - mb * p.n_tiles;
           if (lane == 0) store_chunks_from<BN>(&tmO, stage, e * M_out + mb * BM + q * 32, nt, half);
         }
       }
     }
-    uint32_t tcount = 0;
-    for (int tile = cluster; tile < total; tile += nclusters) {
+    for (uint32_t n = 0;; ++n) {
+      const uint32_t a = n & 1u, aph = (n >> 1) & 1u;
+      bool ok = tc::mbar_wait_cluster(epi_bar(a), aph, kWaitLimitNs, abort_flag);
+      __syncwarp();
+      if (!ok) { fail(abort_flag); break; }
+      const int tile = s_epi[a];
+      if (tile < 0) break;
       const PairTile t = decode(tile);
       const int mt = 2 * t.mp + int(rank);
       const bool mine = mt < t.mtiles;  // this CTA's row block exists
-      const uint32_t a = tcount & 1u, aph = (tcount >> 1) & 1u;
-      const bool ok = tc::mbar_wait(tfull_bar(a), aph, kWaitLimitNs, abort_flag);
+      ok = tc::mbar_wait(tfull_bar(a), aph, kWaitLimitNs, abort_flag);
       __syncwarp();
       if (!ok) { fail(abort_flag); break; }
       tc::fence_after_sync();
@@ -913,7 +990,6 @@ __global__ void __launch_bounds__(kThreads, 1)
       tc::fence_before_sync();
       __syncwarp();
       if (lane == 0) tc::mbar_arrive_cluster(tempty_leader + 8u * a);
-      ++tcount;
     }
     if (lane == 0) tc::bulk_wait0();  // this warp's output stores are complete
     __syncwarp();
@@ -941,6 +1017,28 @@ template <int MODE> bool use_pair() {
     v = (e && e[0] == '1') ? 0 : 1;
   }
   return v == 1;
+}
+
+// The CTA pairs claim tiles from a shared counter (Algorithm 2's greedy, online);
+// MOE_GEMM_STATIC=1 gives every pair a fixed stride of the list instead (for A/B runs).
+bool sched_dynamic() {
+  static int v = -1;
+  if (v < 0) {
+    const char *e = getenv("MOE_GEMM_STATIC");
+    v = (e && e[0] == '1') ? 0 : 1;
+  }
+  return v == 1;
+}
+
+// Points p at the tile counter in the first bytes of the caller's workspace.
+int use_sched_ws(GemmParams &p, void *ws, size_t ws_bytes, const char *fn) {
+  if (!ws || !moe::aligned16(ws) || ws_bytes < moe::kGemmSchedBytes)
+    return moe::set_error(MOE_ERR_WORKSPACE,
+                          "%s: workspace of at least %zu bytes, 16-byte aligned, needed", fn,
+                          moe::kGemmSchedBytes);
+  p.sched_ctr = static_cast<int *>(ws);
+  p.dynamic = sched_dynamic() ? 1 : 0;
+  return MOE_OK;
 }
 
 template <int MODE, int BN>
@@ -996,6 +1094,10 @@ int launch_pair(const CUtensorMap &a, const CUtensorMap &b, const CUtensorMap &o
   }
   cfg.gridDim = dim3(2 * nclusters);
   cfg.numAttrs = 2;
+  if (p.dynamic) {  // the tile counter starts at zero for every launch
+    cudaError_t e = cudaMemsetAsync(p.sched_ctr, 0, sizeof(int), s);
+    if (e != cudaSuccess) return moe::cuda_status(e, what);
+  }
   MOE_LAUNCH(kGemmName[MODE], s, cudaLaunchKernelEx(&cfg, kern, a, b, o, p));
   return moe::launch_status(what);
 }
@@ -1148,8 +1250,6 @@ int moe_grouped_ffn_fwd(const uint16_t *x_perm, const int32_t *group_offsets, in
                         int64_t rows_cap, const uint16_t *w_gate_up, const uint16_t *w_down,
                         uint16_t *ab_saved, uint16_t *h, uint16_t *out_perm, void *ws,
                         size_t ws_bytes, moe_stream_t stream) {
-  (void)ws;
-  (void)ws_bytes;
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   if (int st = check_common(E, d, F, rows_cap, "moe_grouped_ffn_fwd")) return st;
   const void *ptrs[] = {x_perm, group_offsets, w_gate_up, w_down, ab_saved, h, out_perm};
@@ -1157,6 +1257,7 @@ int moe_grouped_ffn_fwd(const uint16_t *x_perm, const int32_t *group_offsets, in
     if (!q || !moe::aligned16(q)) return moe::set_error(MOE_ERR_ARG, "moe_grouped_ffn_fwd: null or unaligned pointer");
   const uint64_t R = uint64_t(rows_cap);
   GemmParams p{};
+  if (int st = use_sched_ws(p, ws, ws_bytes, "moe_grouped_ffn_fwd")) return st;
   p.group_offsets = group_offsets;
   p.E = E; p.d = d; p.F = F;
   // [A | B] = X W_gate_up^T, H = silu(A) * B
@@ -1168,6 +1269,7 @@ int moe_grouped_ffn_fwd(const uint16_t *x_perm, const int32_t *group_offsets, in
     return st;
   // O = H W_down^T
   GemmParams q{};
+  use_sched_ws(q, ws, ws_bytes, "moe_grouped_ffn_fwd");
   q.group_offsets = group_offsets;
   q.E = E; q.d = d; q.F = F;
   q.nkb = F / BK;
@@ -1201,6 +1303,7 @@ int moe_grouped_ffn_fwd_combine(const uint16_t *x_perm, const int32_t *group_off
   int32_t *row_token = reinterpret_cast<int32_t *>(static_cast<char *>(ws) + L.combine_rows);
   float *row_gate = reinterpret_cast<float *>(row_token + Rr);
   GemmParams p{};
+  if (int st = use_sched_ws(p, ws, ws_bytes, fn)) return st;
   p.group_offsets = group_offsets;
   p.E = E; p.d = d; p.F = F;
   p.nkb = d / BK;
@@ -1222,6 +1325,7 @@ int moe_grouped_ffn_fwd_combine(const uint16_t *x_perm, const int32_t *group_off
   }
   // O = H W_down^T, combined into y_acc by the epilogue (O itself stored only if asked)
   GemmParams q{};
+  use_sched_ws(q, ws, ws_bytes, fn);
   q.group_offsets = group_offsets;
   q.E = E; q.d = d; q.F = F;
   q.nkb = F / BK;
@@ -1248,8 +1352,6 @@ int moe_grouped_ffn_fwd_gather(const uint16_t *x, const int32_t *token_of_row, i
                                int64_t rows_cap, const uint16_t *w_gate_up,
                                const uint16_t *w_down, uint16_t *ab_saved, uint16_t *h,
                                uint16_t *out_perm, void *ws, size_t ws_bytes, moe_stream_t stream) {
-  (void)ws;
-  (void)ws_bytes;
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   if (int st = check_common(E, d, F, rows_cap, "moe_grouped_ffn_fwd_gather")) return st;
   if (T < 0) return moe::set_error(MOE_ERR_ARG, "moe_grouped_ffn_fwd_gather: T=%d", T);
@@ -1261,6 +1363,7 @@ int moe_grouped_ffn_fwd_gather(const uint16_t *x, const int32_t *token_of_row, i
     return moe::set_error(MOE_ERR_ARG, "moe_grouped_ffn_fwd_gather: null or unaligned x");
   const uint64_t R = uint64_t(rows_cap);
   GemmParams p{};
+  if (int st = use_sched_ws(p, ws, ws_bytes, "moe_grouped_ffn_fwd_gather")) return st;
   p.group_offsets = group_offsets;
   p.E = E; p.d = d; p.F = F;
   p.nkb = d / BK;
@@ -1274,6 +1377,7 @@ int moe_grouped_ffn_fwd_gather(const uint16_t *x, const int32_t *token_of_row, i
                                  "moe_grouped_ffn_fwd_gather: gate/up GEMM"))
     return st;
   GemmParams q{};
+  use_sched_ws(q, ws, ws_bytes, "moe_grouped_ffn_fwd_gather");
   q.group_offsets = group_offsets;
   q.E = E; q.d = d; q.F = F;
   q.nkb = F / BK;
@@ -1285,7 +1389,7 @@ int moe_grouped_ffn_fwd_gather(const uint16_t *x, const int32_t *token_of_row, i
 int moe_grouped_ffn_bwd_dgrad(const uint16_t *d_out_perm, const uint16_t *ab_saved,
                               const int32_t *group_offsets, int E, int d, int F, int64_t rows_cap,
                               const uint16_t *w_gate_up, const uint16_t *w_down, uint16_t *d_ab,
-                              uint16_t *dx_perm, moe_stream_t stream) {
+                              uint16_t *dx_perm, void *ws, size_t ws_bytes, moe_stream_t stream) {
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   if (int st = check_common(E, d, F, rows_cap, "moe_grouped_ffn_bwd_dgrad")) return st;
   const void *ptrs[] = {d_out_perm, ab_saved, group_offsets, w_gate_up, w_down, d_ab, dx_perm};
@@ -1294,6 +1398,7 @@ int moe_grouped_ffn_bwd_dgrad(const uint16_t *d_out_perm, const uint16_t *ab_sav
   const uint64_t R = uint64_t(rows_cap);
   int st;
   GemmParams p{};
+  if ((st = use_sched_ws(p, ws, ws_bytes, "moe_grouped_ffn_bwd_dgrad"))) return st;
   p.group_offsets = group_offsets;
   p.E = E; p.d = d; p.F = F;
   // dH = dO W_down, fused SwiGLU backward -> [dA | dB]
@@ -1313,8 +1418,9 @@ int moe_grouped_ffn_bwd_dgrad(const uint16_t *d_out_perm, const uint16_t *ab_sav
 
 int moe_grouped_ffn_bwd_wgrad(const uint16_t *d_out_perm, const uint16_t *x_perm,
                               const uint16_t *h, const uint16_t *d_ab,
-                              const int32_t *group_offsets, int E, int d, int F, int64_t rows_cap,
-                              uint16_t *dw_gate_up, uint16_t *dw_down, moe_stream_t stream) {
+                              const int32_t *group_offsets, const uint8_t *active_mask, int E,
+                              int d, int F, int64_t rows_cap, uint16_t *dw_gate_up,
+                              uint16_t *dw_down, void *ws, size_t ws_bytes, moe_stream_t stream) {
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   if (int st = check_common(E, d, F, rows_cap, "moe_grouped_ffn_bwd_wgrad")) return st;
   const void *ptrs[] = {d_out_perm, x_perm, h, d_ab, group_offsets, dw_gate_up, dw_down};
@@ -1323,7 +1429,9 @@ int moe_grouped_ffn_bwd_wgrad(const uint16_t *d_out_perm, const uint16_t *x_perm
   const uint64_t R = uint64_t(rows_cap);
   int st;
   GemmParams p{};
+  if ((st = use_sched_ws(p, ws, ws_bytes, "moe_grouped_ffn_bwd_wgrad"))) return st;
   p.group_offsets = group_offsets;
+  p.active_mask = active_mask;
   p.E = E; p.d = d; p.F = F;
   // dW_down[e] = dO_e^T H_e   ([d, F])
   p.nkb = 0;
@@ -1341,9 +1449,10 @@ int moe_grouped_ffn_bwd_wgrad(const uint16_t *d_out_perm, const uint16_t *x_perm
 
 int moe_grouped_ffn_bwd_wgrad_gather(const uint16_t *d_out_perm, const uint16_t *x,
                                      const int32_t *token_of_row, int T, const uint16_t *h,
-                                     const uint16_t *d_ab, const int32_t *group_offsets, int E,
-                                     int d, int F, int64_t rows_cap, uint16_t *dw_gate_up,
-                                     uint16_t *dw_down, moe_stream_t stream) {
+                                     const uint16_t *d_ab, const int32_t *group_offsets,
+                                     const uint8_t *active_mask, int E, int d, int F,
+                                     int64_t rows_cap, uint16_t *dw_gate_up, uint16_t *dw_down,
+                                     void *ws, size_t ws_bytes, moe_stream_t stream) {
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   if (int st = check_common(E, d, F, rows_cap, "moe_grouped_ffn_bwd_wgrad_gather")) return st;
   if (T < 0) return moe::set_error(MOE_ERR_ARG, "moe_grouped_ffn_bwd_wgrad_gather: T=%d", T);
@@ -1356,7 +1465,9 @@ int moe_grouped_ffn_bwd_wgrad_gather(const uint16_t *d_out_perm, const uint16_t 
   const uint64_t R = uint64_t(rows_cap);
   int st;
   GemmParams p{};
+  if ((st = use_sched_ws(p, ws, ws_bytes, "moe_grouped_ffn_bwd_wgrad_gather"))) return st;
   p.group_offsets = group_offsets;
+  p.active_mask = active_mask;
   p.E = E; p.d = d; p.F = F;
   p.nkb = 0;
   p.m_tiles_w = d / BM;
@@ -1375,17 +1486,15 @@ int moe_grouped_ffn_bwd_wgrad_gather(const uint16_t *d_out_perm, const uint16_t 
 
 int moe_grouped_ffn_bwd(const uint16_t *d_out_perm, const uint16_t *x_perm,
                         const uint16_t *ab_saved, const uint16_t *h, const int32_t *group_offsets,
-                        int E, int d, int F, int64_t rows_cap, const uint16_t *w_gate_up,
-                        const uint16_t *w_down, uint16_t *d_ab, uint16_t *dx_perm,
-                        uint16_t *dw_gate_up, uint16_t *dw_down, void *ws, size_t ws_bytes,
-                        moe_stream_t stream) {
-  (void)ws;
-  (void)ws_bytes;
+                        const uint8_t *active_mask, int E, int d, int F, int64_t rows_cap,
+                        const uint16_t *w_gate_up, const uint16_t *w_down, uint16_t *d_ab,
+                        uint16_t *dx_perm, uint16_t *dw_gate_up, uint16_t *dw_down, void *ws,
+                        size_t ws_bytes, moe_stream_t stream) {
   if (int st = moe_grouped_ffn_bwd_dgrad(d_out_perm, ab_saved, group_offsets, E, d, F, rows_cap,
-                                         w_gate_up, w_down, d_ab, dx_perm, stream))
+                                         w_gate_up, w_down, d_ab, dx_perm, ws, ws_bytes, stream))
     return st;
-  return moe_grouped_ffn_bwd_wgrad(d_out_perm, x_perm, h, d_ab, group_offsets, E, d, F, rows_cap,
-                                   dw_gate_up, dw_down, stream);
+  return moe_grouped_ffn_bwd_wgrad(d_out_perm, x_perm, h, d_ab, group_offsets, active_mask, E, d,
+                                   F, rows_cap, dw_gate_up, dw_down, ws, ws_bytes, stream);
 }
 
 }  // extern "C"

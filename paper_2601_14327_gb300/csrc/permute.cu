@@ -4,6 +4,8 @@
 // (order inside a group: token, then slot), so the grouped layout is
 // deterministic and bit-exact. Groups start at multiples of 128 rows so that
 // every 128-row GEMM tile belongs to one expert; padding rows are zero.
+#include <cuda.h>
+
 #include <mutex>
 
 #include "common.cuh"
@@ -548,23 +550,67 @@ constexpr int kNoAllocScratchInts = 65536;
 static __device__ __align__(256) int32_t g_perm_noalloc_scratch[kNoAllocScratchInts];
 
 namespace {
-// Device address of the array on the current device, looked up once per
-// device (host code cannot use the array's name as a device pointer).
-int noalloc_scratch(int32_t **out) {
-  static std::mutex mu;
-  static int32_t *addr[128] = {nullptr};
-  int dev = 0;
-  cudaError_t e = cudaGetDevice(&dev);
-  if (e != cudaSuccess) return moe::cuda_status(e, "moe_permute_noalloc: cudaGetDevice");
-  if (dev < 0 || dev >= 128) return moe::set_error(MOE_ERR_UNSUPPORTED, "moe_permute_noalloc: device %d", dev);
-  std::lock_guard<std::mutex> g(mu);
-  if (addr[dev] == nullptr) {
+typedef CUresult (*CtxGetCurrentFn)(CUcontext *);
+typedef CUresult (*CtxGetIdFn)(CUcontext, unsigned long long *);
+
+// Unique id of the calling thread's current CUDA context (0: none is current yet).
+// Ids are never reused, so a context created after cudaDeviceReset, or another
+// context of the same device, has an id of its own.
+int current_context_id(unsigned long long *id) {
+  static CtxGetCurrentFn get_current = nullptr;
+  static CtxGetIdFn get_id = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
     void *p = nullptr;
-    e = cudaGetSymbolAddress(&p, g_perm_noalloc_scratch);
-    if (e != cudaSuccess) return moe::cuda_status(e, "moe_permute_noalloc: cudaGetSymbolAddress");
-    addr[dev] = static_cast<int32_t *>(p);
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess && q == cudaDriverEntryPointSuccess)
+      get_current = reinterpret_cast<CtxGetCurrentFn>(p);
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetId", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess && q == cudaDriverEntryPointSuccess)
+      get_id = reinterpret_cast<CtxGetIdFn>(p);
+  });
+  if (!get_current || !get_id)
+    return moe::set_error(MOE_ERR_CUDA, "moe_permute_noalloc: cuCtxGetCurrent/cuCtxGetId unavailable");
+  CUcontext ctx = nullptr;
+  if (get_current(&ctx) != CUDA_SUCCESS)
+    return moe::set_error(MOE_ERR_CUDA, "moe_permute_noalloc: cuCtxGetCurrent failed");
+  *id = 0;
+  if (ctx && get_id(ctx, id) != CUDA_SUCCESS)
+    return moe::set_error(MOE_ERR_CUDA, "moe_permute_noalloc: cuCtxGetId failed");
+  return MOE_OK;
+}
+
+// Device address of the array in the current context. Host code cannot use the
+// array's name as a device pointer, and the address belongs to the context that
+// loaded the library's module: it is looked up once per context (keyed by the
+// context's unique id) and cached; another context of the same device, or the new
+// primary context after cudaDeviceReset, gets a lookup of its own.
+int noalloc_scratch(int32_t **out) {
+  constexpr int kSlots = 64;
+  static std::mutex mu;
+  static unsigned long long ids[kSlots] = {0};
+  static int32_t *addr[kSlots] = {nullptr};
+  static int next = 0;
+  unsigned long long id = 0;
+  if (int st = current_context_id(&id)) return st;
+  std::lock_guard<std::mutex> g(mu);
+  if (id != 0) {
+    for (int i = 0; i < kSlots; ++i)
+      if (ids[i] == id) {
+        *out = addr[i];
+        return MOE_OK;
+      }
   }
-  *out = addr[dev];
+  void *p = nullptr;  // the runtime makes the primary context current if none is
+  cudaError_t e = cudaGetSymbolAddress(&p, g_perm_noalloc_scratch);
+  if (e != cudaSuccess) return moe::cuda_status(e, "moe_permute_noalloc: cudaGetSymbolAddress");
+  if (id == 0 && (current_context_id(&id) != MOE_OK || id == 0))
+    return moe::set_error(MOE_ERR_CUDA, "moe_permute_noalloc: no current context");
+  ids[next] = id;  // oldest entry replaced when all slots are taken
+  addr[next] = static_cast<int32_t *>(p);
+  next = (next + 1) % kSlots;
+  *out = static_cast<int32_t *>(p);
   return MOE_OK;
 }
 }  // namespace

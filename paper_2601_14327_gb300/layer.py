@@ -128,8 +128,12 @@ def forward(b: MoELayerBuffers, x, w_router, bias, w_gate_up, w_down, active_mas
 
 
 def backward(b: MoELayerBuffers, dy, w_router, w_gate_up, w_down, stream=None,
-             overlap: bool = True):
+             overlap: bool = True, active_mask=None):
     """combine bwd -> grouped FFN bwd (dgrad, then wgrad) -> router bwd -> permute bwd.
+
+    active_mask: the LAEP mask the forward routed with (None: all experts live). Pruned
+    experts' weight gradients are not written (their buffers keep what they held); live
+    experts without tokens get exact zeros.
 
     With overlap, the router backward (after the combine backward) and the
     unpermute-sum (after the dX GEMM) run on a second stream while the main stream
@@ -149,7 +153,7 @@ def backward(b: MoELayerBuffers, dy, w_router, w_gate_up, w_down, stream=None,
     L.moe_route_bwd(b.x, b.topk_idx, b.topk_gate, b.d_gate, s.T, s.d, s.E, s.k, b.d_logits,
                     b.dw_router, b.ws, b.ws_bytes, side)
     L.moe_grouped_ffn_bwd_dgrad(b.d_out_perm, b.ab, b.group_offsets, s.E, s.d, s.F, R,
-                                w_gate_up, w_down, b.d_ab, b.dx_perm, main)
+                                w_gate_up, w_down, b.d_ab, b.dx_perm, b.ws, b.ws_bytes, main)
     if overlap:
         ev = torch.cuda.Event()
         ev.record(main)
@@ -158,11 +162,12 @@ def backward(b: MoELayerBuffers, dy, w_router, w_gate_up, w_down, stream=None,
                       s.d, s.E, s.k, b.dx, b.ws, b.ws_bytes, side)
     if b.gather:
         L.moe_grouped_ffn_bwd_wgrad_gather(b.d_out_perm, b.x, b.token_of_row, s.T, b.h, b.d_ab,
-                                           b.group_offsets, s.E, s.d, s.F, R, b.dw_gate_up,
-                                           b.dw_down, main)
+                                           b.group_offsets, active_mask, s.E, s.d, s.F, R,
+                                           b.dw_gate_up, b.dw_down, b.ws, b.ws_bytes, main)
     else:
-        L.moe_grouped_ffn_bwd_wgrad(b.d_out_perm, b.x_perm, b.h, b.d_ab, b.group_offsets, s.E,
-                                    s.d, s.F, R, b.dw_gate_up, b.dw_down, main)
+        L.moe_grouped_ffn_bwd_wgrad(b.d_out_perm, b.x_perm, b.h, b.d_ab, b.group_offsets,
+                                    active_mask, s.E, s.d, s.F, R, b.dw_gate_up, b.dw_down, b.ws,
+                                    b.ws_bytes, main)
     if overlap:
         ev = torch.cuda.Event()
         ev.record(side)

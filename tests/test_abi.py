@@ -86,6 +86,20 @@ def test_argument_validation_without_launch(lib):
     with pytest.raises(L.MoEError) as e:
         L.moe_grouped_ffn_fwd(None, 16, 8, 256, 256, 4096, 16, 16, 16, 16, 16, 16, 0, stream=0)
     assert e.value.status == -1
+    # the grouped GEMMs need a workspace for their tile counter (16-byte aligned, 256 bytes)
+    for ws, ws_bytes in ((None, 0), (16, 128), (24, 1 << 20)):
+        with pytest.raises(L.MoEError) as e:
+            L.moe_grouped_ffn_fwd(16, 16, 8, 256, 256, 4096, 16, 16, 16, 16, 16, ws, ws_bytes,
+                                  stream=0)
+        assert e.value.status == -6
+        with pytest.raises(L.MoEError) as e:
+            L.moe_grouped_ffn_bwd_dgrad(16, 16, 16, 8, 256, 256, 4096, 16, 16, 16, 16, ws,
+                                        ws_bytes, stream=0)
+        assert e.value.status == -6
+        with pytest.raises(L.MoEError) as e:
+            L.moe_grouped_ffn_bwd_wgrad(16, 16, 16, 16, 16, None, 8, 256, 256, 4096, 16, 16, ws,
+                                        ws_bytes, stream=0)
+        assert e.value.status == -6
     with pytest.raises(L.MoEError) as e:  # rows_cap below T*k + 128*E
         L.moe_permute(16, 16, None, 100, 64, 8, 2, 100, 16, 16, 16, 16, 16, 1 << 20, stream=0)
     assert e.value.status == -1
@@ -156,8 +170,8 @@ def test_new_entry_points_validate_before_launch(lib):
                                      stream=0)
     assert e.value.status == -1
     with pytest.raises(L.MoEError) as e:  # unaligned token_of_row
-        L.moe_grouped_ffn_bwd_wgrad_gather(16, 16, 20, 10, 16, 16, 16, 8, 128, 256, R, 16, 16,
-                                           stream=0)
+        L.moe_grouped_ffn_bwd_wgrad_gather(16, 16, 20, 10, 16, 16, 16, None, 8, 128, 256, R, 16,
+                                           16, 16, 1 << 20, stream=0)
     assert e.value.status == -1
     with pytest.raises(L.MoEError) as e:  # router backward: x missing with tokens present
         L.moe_route_bwd(None, 16, 16, 16, 10, 128, 8, 2, 16, 16, 16, 1 << 20, stream=0)

@@ -49,3 +49,44 @@ def test_clock_sampler_keeps_the_timed_region():
     assert out["samples"] == 3 and out["samples_under_load"] == 2
     assert out["sm_mhz"] == 1510 and out["sm_max_mhz"] == 2070
     assert out["reasons"] == ["sw_power_cap"]
+
+
+def test_tensor_peak_follows_the_timed_region():
+    peaks = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0,
+             "source": "measured"}
+    p, name = bench.tensor_peak(peaks, 0.26)
+    assert p == 1900.0 and "burst" in name
+    p, name = bench.tensor_peak(peaks, 2.1)
+    assert p == 1700.0 and "sustained" in name
+
+
+def test_oracle_sample_on_routed_experts_equals_the_full_layer():
+    """The bounded CPU-baseline sample keeps only the experts its tokens are routed to; the
+    oracle on that subset must give these tokens the full layer's routing, outputs and
+    gradients (the subset's weight gradients are the full layer's rows of those experts)."""
+    import numpy as np
+    import torch
+
+    from oracle import moe_oracle as O
+    from paper_2601_14327_gb300 import synth
+
+    T, d, E, k, F = 48, 32, 12, 3, 16
+    inp = synth.make_layer_inputs(T, d, E, k, F, bias="zipf", zipf_s=1.2, seed=7)
+    mask = torch.ones(E, dtype=torch.uint8)
+    mask[[1, 5]] = 0
+    n = 5
+    h, n_exp = bench.sample_inputs(inp, mask, k, n)
+    full = O.moe_layer(inp["x"][:n].float().numpy(), inp["w_router"].numpy(),
+                       inp["bias"].numpy(), mask.numpy(), k, inp["w_gate_up"].float().numpy(),
+                       inp["w_down"].float().numpy(), dy=inp["dy"][:n].float().numpy())
+    sub = O.moe_layer(h["x"], h["w_router"], h["bias"], h["mask"], k, h["w_gate_up"],
+                      h["w_down"], dy=h["dy"])
+    used = np.unique(full["topk_idx"])
+    assert n_exp == used.size < E
+    np.testing.assert_array_equal(used[sub["topk_idx"]], full["topk_idx"])
+    for name in ("gates", "y", "dx", "d_gate", "d_logits"):
+        np.testing.assert_array_equal(sub[name], full[name])
+    np.testing.assert_array_equal(sub["dw_gate_up"], full["dw_gate_up"][used])
+    np.testing.assert_array_equal(sub["dw_down"], full["dw_down"][used])
+    np.testing.assert_array_equal(sub["dw_router"], full["dw_router"][:, used])
+    assert not full["dw_gate_up"][np.setdiff1d(np.arange(E), used)].any()

@@ -443,6 +443,61 @@ def test_one_sm_gemm_kernel_against_oracle():
     assert r.returncode == 0, r.stdout[-2000:] + r.stderr[-4000:]
 
 
+def test_dynamic_schedule_equals_fixed_stride(tmp_path):
+    """The CTA pairs claim tiles from a shared counter, so which pair computes a tile
+    changes from run to run, but not the tile's arithmetic: every output and gradient
+    equals, bit for bit, the fixed-stride schedule (MOE_GEMM_STATIC=1, read once per
+    process, so that half runs in a child process)."""
+    import gpu_schedule_check as G
+    path = str(tmp_path / "static.pt")
+    env = dict(os.environ, MOE_GEMM_STATIC="1")
+    script = os.path.join(os.path.dirname(os.path.abspath(__file__)), "gpu_schedule_check.py")
+    r = subprocess.run([sys.executable, script, path], env=env, capture_output=True, text=True,
+                       timeout=900)
+    assert r.returncode == 0, r.stdout[-2000:] + r.stderr[-4000:]
+    static = torch.load(path)
+    for i, dyn in enumerate(G.run_cases()):
+        for n in G.NAMES:
+            assert torch.equal(dyn[n], static[i][n]), (G.SCHEDULE_CASES[i], n)
+
+
+def test_pruned_experts_weight_gradients_untouched():
+    """Pruned experts (LAEP mask 0) get no tile and no store in the weight-gradient GEMMs:
+    their gradient buffers keep what the caller left there. A live expert that received no
+    token still gets exact zeros, and the live experts match the oracle."""
+    T, d, E, k, F = 1200, 256, 10, 2, 384
+    inp = case_inputs(T, d, E, k, F, seed=5)
+    o = oracle_inputs(inp)
+    mask = np.ones(E, np.uint8)
+    mask[[1, 6]] = 0
+    z = O.router_logits(o["x"], o["w_router"], o["bias"])
+    z[:, 3] = -1e30  # live, never selected
+    ref = O.moe_layer(o["x"], o["w_router"], o["bias"], mask, k, o["w_gate_up"], o["w_down"],
+                      dy=o["dy"], logits32=z)
+    assert ref["counts"][3] == 0 and (ref["counts"][[1, 6]] == 0).all()
+    dev = "cuda"
+    g = {n: v.to(dev) for n, v in inp.items()}
+    m = torch.as_tensor(mask).to(dev)
+    sentinel = 1.5
+    for one_stream in (False, True):
+        b = layer.MoELayerBuffers(layer.LayerShape(T, d, E, k, F), dev, backward=True)
+        b.dw_gate_up.fill_(sentinel)
+        b.dw_down.fill_(sentinel)
+        layer.forward(b, g["x"], g["w_router"], g["bias"], g["w_gate_up"], g["w_down"], m,
+                      torch.from_numpy(z).to(dev))
+        layer.backward(b, g["dy"], g["w_router"], g["w_gate_up"], g["w_down"],
+                       overlap=not one_stream, active_mask=m)
+        torch.cuda.synchronize()
+        assert L.moe_device_error(clear=True) == 0
+        for e in (1, 6):
+            assert (b.dw_gate_up[e] == sentinel).all() and (b.dw_down[e] == sentinel).all()
+        assert not b.dw_gate_up[3].any() and not b.dw_down[3].any()
+        live = np.nonzero(mask)[0]
+        assert_close("dw_gate_up", to_np(b.dw_gate_up)[live], ref["dw_gate_up"][live])
+        assert_close("dw_down", to_np(b.dw_down)[live], ref["dw_down"][live])
+        assert_close("dx", to_np(b.dx), ref["dx"])
+
+
 def test_bounded_wait_expires_and_reports():
     """A pipeline wait that nothing satisfies (an mbarrier no one arrives on) gives up
     after its limit: the kernel returns, the device error word reads

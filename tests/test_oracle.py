@@ -225,6 +225,15 @@ def test_per_element_evaluators_match_grouped_oracle():
     np.testing.assert_allclose(dwd, out["dw_down"][e][:, [0, 3, 9]].T, rtol=1e-11, atol=1e-12)
     np.testing.assert_allclose(dwg, out["dw_gate_up"][e][[0, 3, 9]], rtol=1e-11, atol=1e-12)
     np.testing.assert_allclose(dwu, out["dw_gate_up"][e][[10, 13, 19]], rtol=1e-11, atol=1e-12)
+    # a set of tokens, expert by expert, equals the grouped oracle on those tokens
+    toks = np.array([0, 3, 7, 8, 24])
+    y, dx, dg, dz = O.tokens_forward_backward(c["x"][toks], out["topk_idx"][toks],
+                                              out["gates"][toks], c["dy"][toks], c["w_router"],
+                                              c["w_gate_up"], c["w_down"])
+    np.testing.assert_allclose(y, out["y"][toks], rtol=1e-12, atol=1e-13)
+    np.testing.assert_allclose(dx, out["dx"][toks], rtol=1e-11, atol=1e-12)
+    np.testing.assert_allclose(dg, out["d_gate"][toks], rtol=1e-11, atol=1e-13)
+    np.testing.assert_allclose(dz, out["d_logits"][toks], rtol=1e-11, atol=1e-13)
 
 
 def test_three_matrix_expert_matches_table_a1_parameter_counts():

@@ -6,8 +6,14 @@ them the library offers one entry point that keeps its scratch in a fixed
 array compiled into the library. This test checks, through the C ABI, that
 it returns exactly what the workspace-based moe_permute returns, on two
 calls in a row (the second call reuses the array the first one left behind),
-and that a problem larger than the array is refused before any launch.
+also after the process's CUDA context was replaced (the array's address belongs
+to a context), and that a problem larger than the array is refused before any
+launch.
 """
+import os
+import subprocess
+import sys
+
 import numpy as np
 import pytest
 import torch
@@ -58,3 +64,12 @@ def test_permute_noalloc_refuses_problems_beyond_its_array():
                               16, 16, 16, 16)
     assert e.value.status == -2
     assert "scratch" in str(e.value)
+
+
+def test_permute_noalloc_after_device_reset():
+    """The array's device address is looked up per CUDA context: after cudaDeviceReset
+    the new context gets its own lookup, and the results still equal moe_permute's. The
+    reset would end this process's torch context, so it runs in a child process."""
+    script = os.path.join(os.path.dirname(os.path.abspath(__file__)), "gpu_noalloc_reset_check.py")
+    r = subprocess.run([sys.executable, script], capture_output=True, text=True, timeout=600)
+    assert r.returncode == 0, r.stdout[-2000:] + r.stderr[-4000:]

@@ -785,6 +785,13 @@ def layer_calls(wl):
     them): `--call NAME` times one of them alone."""
     i, b, s = wl.inp, wl.bufs, wl.shape
     R = s.rows_cap
+    if isinstance(wl, RouterWorkload):
+        return {
+            "route": lambda: layer.route(b, i["x"], i["w_router"], i["bias"]),
+            "route_bwd": lambda: L.moe_route_bwd(b.x, b.topk_idx, b.topk_gate, b.d_gate, s.T,
+                                                 s.d, s.E, s.k, b.d_logits, b.dw_router, b.ws,
+                                                 b.ws_bytes),
+        }
     return {
         "route": lambda: layer.route(b, i["x"], i["w_router"], i["bias"], wl.mask),
         "permute": lambda: L.moe_permute(i["x"], b.topk_idx, b.counts, s.T, s.d, s.E, s.k, R,
@@ -800,7 +807,8 @@ def layer_calls(wl):
             b.group_counts, s.T, s.d, s.E, s.k, b.d_out_perm, b.d_gate),
         "ffn_bwd_dgrad": lambda: L.moe_grouped_ffn_bwd_dgrad(
             b.d_out_perm, b.ab, b.group_offsets, s.E, s.d, s.F, R, i["w_gate_up"], i["w_down"],
-            b.d_ab, b.dx_perm, b.ws, b.ws_bytes),
+            b.topk_gate, b.d_gate, b.row_of_assignment, i["w_router"], s.T, s.k, b.d_ab,
+            b.dx_perm, b.ws, b.ws_bytes),
         "ffn_bwd_wgrad": lambda: L.moe_grouped_ffn_bwd_wgrad(
             b.d_out_perm, b.x_perm, b.h, b.d_ab, b.group_offsets, wl.mask, s.E, s.d, s.F, R,
             b.dw_gate_up, b.dw_down, b.ws, b.ws_bytes),
@@ -808,13 +816,59 @@ def layer_calls(wl):
                                              s.E, s.k, b.d_logits, b.dw_router, b.ws,
                                              b.ws_bytes),
         "permute_bwd": lambda: L.moe_permute_bwd(b.dx_perm, b.row_of_assignment, b.topk_idx,
-                                                 b.d_logits, i["w_router"], s.T, s.d, s.E, s.k,
-                                                 b.dx, b.ws, b.ws_bytes),
+                                                 None, None, s.T, s.d, s.E, s.k, b.dx, b.ws,
+                                                 b.ws_bytes),
     }
 
 
 CALL_NAMES = ["route", "permute", "ffn_fwd", "combine", "combine_bwd", "ffn_bwd_dgrad",
               "ffn_bwd_wgrad", "route_bwd", "permute_bwd"]
+ROUTER_CALLS = ("route", "route_bwd")
+
+
+class RouterWorkload:
+    """What the router's two calls read and write, and nothing else (no expert weights,
+    no grouped buffers), at the workload's T, d_model, live experts (the compacted count
+    where the workload compacts), top-k and gate bias; seeded like the workload. The
+    routing is made once; route_bwd reads it with a seeded d_gate."""
+
+    def __init__(self, cfg_id, device, tokens=None, experts=None, bias=None):
+        c = synth.CONFIGS[cfg_id]
+        E = experts or (c.E - c.prune_lowest if c.compact else c.E)
+        T = tokens or c.T
+        self.cfg = c
+        self.mask = None
+        inp = synth.make_layer_inputs(T, c.d, E, c.k, 128, bias=bias or c.bias, zipf_s=c.zipf_s,
+                                      seed=synth.seed_for(cfg_id), device=device,
+                                      with_weights=False, backward=False)
+        self.inp = inp
+        self.shape = layer.LayerShape(T, c.d, E, c.k, 128)
+        s = self.shape
+        ws_bytes = max(L.moe_workspace_size(T, c.d, E, c.k, 128), 256)
+
+        class _B:  # the buffers the two calls use, named as in MoELayerBuffers
+            pass
+        b = _B()
+        b.shape = self.shape
+        b.ws_bytes, b.ws = ws_bytes, torch.empty(ws_bytes, dtype=torch.uint8, device=device)
+        b.logits = None
+        b.topk_idx = torch.empty(T, c.k, dtype=torch.int32, device=device)
+        b.topk_gate = torch.empty(T, c.k, dtype=torch.float32, device=device)
+        b.counts = torch.empty(E, dtype=torch.int32, device=device)
+        b.x = inp["x"]
+        gen = torch.Generator(device=device)
+        gen.manual_seed(synth.seed_for(cfg_id) + 1)
+        b.d_gate = torch.randn(T, c.k, generator=gen, device=device)
+        b.d_logits = torch.empty(T, c.k, dtype=torch.float32, device=device)
+        b.dw_router = torch.empty(c.d, E, dtype=torch.float32, device=device)
+        self.bufs = b
+        layer.route(b, inp["x"], inp["w_router"], inp["bias"])
+
+    def live_counts(self):
+        return self.bufs.counts.cpu().tolist()
+
+    def gemm_flops(self):
+        return {}
 
 
 def run_call(args):
@@ -824,9 +878,13 @@ def run_call(args):
     L.load()
     torch.cuda.set_device(0)
     peaks = measured_peaks()
-    wl = Workload(args.config, "cuda", tokens=args.tokens, experts=args.experts,
-                  no_prune=args.no_prune, bias=args.bias, backward=True)
-    wl.eager_step()
+    if args.call in ROUTER_CALLS:
+        wl = RouterWorkload(args.config, "cuda", tokens=args.tokens, experts=args.experts,
+                            bias=args.bias)
+    else:
+        wl = Workload(args.config, "cuda", tokens=args.tokens, experts=args.experts,
+                      no_prune=args.no_prune, bias=args.bias, backward=True)
+        wl.eager_step()
     fn = layer_calls(wl)[args.call]
     for _ in range(args.warmup):
         fn()

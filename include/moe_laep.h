@@ -388,15 +388,28 @@ int moe_unpermute_combine_bwd(const uint16_t *dy, const uint16_t *out_perm,
  * forward; d_ab [rows_cap,2F] bf16 caller scratch (receives [dA|dB]);
  * outputs dx_perm [rows_cap,d] bf16, dw_gate_up [E,2F,d] bf16,
  * dw_down [E,d,F] bf16 (fp32 accumulation). ws as in moe_grouped_ffn_fwd.
+ * Router term (optional, on when w_router is not NULL; topk_gate, d_gate and
+ * row_of_assignment are then needed unless T == 0, and must be NULL otherwise): with
+ * topk_gate [T,k] and row_of_assignment [T,k] (moe_route, moe_permute), d_gate [T,k]
+ * (moe_unpermute_combine_bwd) and w_router [d,E] fp32, the dX GEMM's epilogue adds
+ * the router's share of the input gradient to every grouped row before rounding:
+ *   dx_perm[row(t,j), :] = dX(t,j) + dz[t,j] * w_router[:, e_j],
+ *   dz[t,j] = g[t,j] * (d_gate[t,j] - sum_i g[t,i] * d_gate[t,i])
+ * (the d_logits of moe_route_bwd, same arithmetic), so that moe_permute_bwd, called
+ * without its router term, sums the rows into the full dx. The epilogue reads one
+ * 256-wide slice of a w_router column per tile instead of k columns per token.
+ * ws then needs moe_workspace_size(T, d, E, k, F) bytes (dz per grouped row);
+ * 1 <= k <= min(8, E), rows_cap >= moe_perm_rows_max(T, k, E).
  * Limits as in the forward.
  */
 int moe_grouped_ffn_bwd(const uint16_t *d_out_perm, const uint16_t *x_perm,
                         const uint16_t *ab_saved, const uint16_t *h,
                         const int32_t *group_offsets, const uint8_t *active_mask, int E, int d,
                         int F, int64_t rows_cap, const uint16_t *w_gate_up,
-                        const uint16_t *w_down, uint16_t *d_ab, uint16_t *dx_perm,
-                        uint16_t *dw_gate_up, uint16_t *dw_down, void *ws, size_t ws_bytes,
-                        moe_stream_t stream);
+                        const uint16_t *w_down, const float *topk_gate, const float *d_gate,
+                        const int32_t *row_of_assignment, const float *w_router, int T, int k,
+                        uint16_t *d_ab, uint16_t *dx_perm, uint16_t *dw_gate_up,
+                        uint16_t *dw_down, void *ws, size_t ws_bytes, moe_stream_t stream);
 
 /*
  * moe_grouped_ffn_bwd_dgrad / moe_grouped_ffn_bwd_wgrad - the two halves of
@@ -404,14 +417,18 @@ int moe_grouped_ffn_bwd(const uint16_t *d_out_perm, const uint16_t *x_perm,
  * callers that overlap other work with the weight gradients (the derivative of
  * Table A1's three-matrix expert; the paper gives no backward):
  *   dgrad: dH = dO W_down, [dA|dB] (into d_ab), dX = [dA|dB] W_gate_up
+ *          (+ the router term when its arguments are given)
  *   wgrad: dW_down = dO^T H, dW_gate_up = [dA|dB]^T X  (needs d_ab from dgrad;
  *          pruned experts of active_mask are not written)
  * Arguments as in moe_grouped_ffn_bwd.
  */
 int moe_grouped_ffn_bwd_dgrad(const uint16_t *d_out_perm, const uint16_t *ab_saved,
                               const int32_t *group_offsets, int E, int d, int F, int64_t rows_cap,
-                              const uint16_t *w_gate_up, const uint16_t *w_down, uint16_t *d_ab,
-                              uint16_t *dx_perm, void *ws, size_t ws_bytes, moe_stream_t stream);
+                              const uint16_t *w_gate_up, const uint16_t *w_down,
+                              const float *topk_gate, const float *d_gate,
+                              const int32_t *row_of_assignment, const float *w_router, int T,
+                              int k, uint16_t *d_ab, uint16_t *dx_perm, void *ws, size_t ws_bytes,
+                              moe_stream_t stream);
 int moe_grouped_ffn_bwd_wgrad(const uint16_t *d_out_perm, const uint16_t *x_perm,
                               const uint16_t *h, const uint16_t *d_ab,
                               const int32_t *group_offsets, const uint8_t *active_mask, int E,
@@ -456,7 +473,9 @@ int moe_route_bwd(const uint16_t *x, const int32_t *topk_idx, const float *topk_
  * moe_route_bwd's d_logits):
  *   dx[t,:] = sum_j dx_perm[row(t,j), :] + sum_j d_logits[t,j] * w_router[:, e_j]
  * summed in fp32, one bf16 rounding. d_logits and w_router may both be NULL
- * (no router term). dx [T,d] bf16 (out).
+ * (no router term): the form to use after moe_grouped_ffn_bwd_dgrad added the router
+ * term to dx_perm (the layer's default; a pure gather-sum at the HBM rate), while
+ * with them each token reads k fp32 rows of w_router. dx [T,d] bf16 (out).
  */
 int moe_permute_bwd(const uint16_t *dx_perm, const int32_t *row_of_assignment,
                     const int32_t *topk_idx, const float *d_logits, const float *w_router,

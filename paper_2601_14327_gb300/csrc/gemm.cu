@@ -91,6 +91,12 @@ struct GemmParams {
   float *y_acc;
   const int32_t *row_token;
   const float *row_gate;
+  // kDgradGateUp with the router's term of the input gradient (nullptr: without):
+  // dX[r, :] += row_dz[r] * W_r[:, e] for every grouped row r of expert e, with
+  // row_dz [rows] the router logit gradient of the row's assignment (0 on padding rows)
+  // and w_router [d, E] fp32.
+  const float *row_dz;
+  const float *w_router;
   // Weight-gradient modes: experts with active_mask[e] == 0 (pruned by LAEP) get no tile
   // and no store; their gradient buffers are left as they are (nullptr: all experts live).
   const uint8_t *active_mask;
@@ -248,11 +254,23 @@ __device__ __forceinline__ void epilogue_tile(const GemmParams &p, const CUtenso
       tok = p.row_token[row];
       g = p.row_gate[row];
     }
+    // dX with the router's term: this lane's row gets dz * W_r[col, e] added (dz = 0 on
+    // padding rows); the W_r values of a 32-column chunk are loaded one per lane.
+    float dz = 0.f;
+    const bool router = MODE == kDgradGateUp && p.row_dz != nullptr;
+    if (router) dz = p.row_dz[row];
 #pragma unroll 1
     for (int c = half * (BN / 2); c < (half + 1) * (BN / 2); c += 32) {
       uint32_t r[32];
+      float w = 0.f;
+      if (router) w = __ldg(p.w_router + size_t(nt * BN + c + lane) * p.E + e);
       tc::tmem_ld_32x32b_x32(tb + c, r);
       tc::tmem_ld_wait();
+      if (router) {
+#pragma unroll
+        for (int v = 0; v < 32; ++v)
+          r[v] = __float_as_uint(fmaf(dz, __shfl_sync(0xffffffffu, w, v), __uint_as_float(r[v])));
+      }
       if (MODE == kDown && tok >= 0) {
         float4 *dst = reinterpret_cast<float4 *>(p.y_acc + size_t(tok) * p.d + nt * BN + c);
 #pragma unroll
@@ -576,6 +594,8 @@ __global__ void __launch_bounds__(kThreads, 1)
 // STAGES (< kRing) bound: a producer can run at most STAGES k-blocks, hence STAGES tiles,
 // ahead of the MMAs that need the other readers' progress.
 constexpr int kRing = 16;
+// Row pairs per block of the weight-gradient tile order (see decode).
+constexpr int kWgradBlock = 8;
 
 template <int BN, int KB> struct PairShape {
   static constexpr int BNH = BN / 2;  // B rows staged by each CTA
@@ -734,8 +754,27 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int local = tile - s_prefix[lo];
     t.e = s_order[lo];
     t.goff = s_goff[t.e];
-    t.mp = local / p.n_tiles;
-    t.nt = local - t.mp * p.n_tiles;
+    if (Tr::WGRAD && p.n_tiles > kWgradBlock) {
+      // Weight gradients with many column tiles: an expert's (row pair, column) tiles in
+      // blocks of kWgradBlock row pairs, column by column inside a block, so that the
+      // tiles the pairs run at the same time (consecutive in the list) share few operand
+      // panels: about kWgradBlock row panels and 76 / kWgradBlock column panels per wave
+      // instead of 3 row and 28 column panels (dW_gate_up at d_model = 7168). The pairs
+      // of a wave move through the reduction (the expert's rows) together, and each
+      // panel slice they share is read from DRAM once: measured at d_model = 7168,
+      // 65,536 rows over 8 experts, dW_gate_up read 3.8 GB instead of 6.9 GB and ran
+      // 8% faster. With few column tiles (dW_down: 8) the rows-first order already
+      // shares as few panels and stays.
+      const int MP = (p.m_tiles_w + 1) / 2;
+      const int blk = local / (kWgradBlock * p.n_tiles);
+      const int rem = local - blk * kWgradBlock * p.n_tiles;
+      const int bh = min(kWgradBlock, MP - blk * kWgradBlock);
+      t.nt = rem / bh;
+      t.mp = blk * kWgradBlock + (rem - t.nt * bh);
+    } else {
+      t.mp = local / p.n_tiles;
+      t.nt = local - t.mp * p.n_tiles;
+    }
     const int rows = s_goff[t.e + 1] - t.goff;
     t.nkb = Tr::WGRAD ? rows / KB : p.nkb / (KB / BK);
     t.mtiles = Tr::WGRAD ? p.m_tiles_w : rows / BM;
@@ -1209,6 +1248,36 @@ __global__ void combine_rows_scatter_kernel(const int32_t *__restrict__ row_of_a
     }
   }
 }
+// The router's logit gradient of every assignment (softmax over the k selected experts:
+// dz_j = g_j (dg_j - sum_i g_i dg_i), summed in slot order with fused multiply-adds, as
+// moe_route_bwd computes it) written to the assignment's grouped row. Padding rows keep
+// the zeros the caller wrote first.
+__global__ void router_row_dz_kernel(const float *__restrict__ topk_gate,
+                                     const float *__restrict__ d_gate,
+                                     const int32_t *__restrict__ row_of_assignment, int T, int k,
+                                     int64_t R, float *__restrict__ row_dz) {
+  for (int t = blockIdx.x * blockDim.x + threadIdx.x; t < T; t += gridDim.x * blockDim.x) {
+    float g[8], dg[8], s = 0.f;
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      g[j] = 0.f;
+      dg[j] = 0.f;
+      if (j < k) {
+        g[j] = topk_gate[size_t(t) * k + j];
+        dg[j] = d_gate[size_t(t) * k + j];
+        s = fmaf(g[j], dg[j], s);
+      }
+    }
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      if (j < k) {
+        const int32_t r = row_of_assignment[size_t(t) * k + j];
+        if (r >= 0 && r < R) row_dz[r] = g[j] * (dg[j] - s);
+        else dev_flag(&g_dev_err, MOE_DEV_ROWS_OVERFLOW);
+      }
+    }
+  }
+}
 __global__ void zero_f32x4_kernel(float4 *__restrict__ p, int64_t n4) {
   for (int64_t i = blockIdx.x * int64_t(blockDim.x) + threadIdx.x; i < n4;
        i += int64_t(gridDim.x) * blockDim.x)
@@ -1388,17 +1457,45 @@ int moe_grouped_ffn_fwd_gather(const uint16_t *x, const int32_t *token_of_row, i
 
 int moe_grouped_ffn_bwd_dgrad(const uint16_t *d_out_perm, const uint16_t *ab_saved,
                               const int32_t *group_offsets, int E, int d, int F, int64_t rows_cap,
-                              const uint16_t *w_gate_up, const uint16_t *w_down, uint16_t *d_ab,
-                              uint16_t *dx_perm, void *ws, size_t ws_bytes, moe_stream_t stream) {
+                              const uint16_t *w_gate_up, const uint16_t *w_down,
+                              const float *topk_gate, const float *d_gate,
+                              const int32_t *row_of_assignment, const float *w_router, int T,
+                              int k, uint16_t *d_ab, uint16_t *dx_perm, void *ws, size_t ws_bytes,
+                              moe_stream_t stream) {
+  const char *fn = "moe_grouped_ffn_bwd_dgrad";
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-  if (int st = check_common(E, d, F, rows_cap, "moe_grouped_ffn_bwd_dgrad")) return st;
+  if (int st = check_common(E, d, F, rows_cap, fn)) return st;
   const void *ptrs[] = {d_out_perm, ab_saved, group_offsets, w_gate_up, w_down, d_ab, dx_perm};
   for (const void *q : ptrs)
-    if (!q || !moe::aligned16(q)) return moe::set_error(MOE_ERR_ARG, "moe_grouped_ffn_bwd_dgrad: null or unaligned pointer");
+    if (!q || !moe::aligned16(q)) return moe::set_error(MOE_ERR_ARG, "%s: null or unaligned pointer", fn);
   const uint64_t R = uint64_t(rows_cap);
   int st;
   GemmParams p{};
-  if ((st = use_sched_ws(p, ws, ws_bytes, "moe_grouped_ffn_bwd_dgrad"))) return st;
+  if ((st = use_sched_ws(p, ws, ws_bytes, fn))) return st;
+  // the router's term of the input gradient, added in the dX GEMM's epilogue
+  const bool router = w_router != nullptr;
+  if (!router && (topk_gate || d_gate || row_of_assignment))
+    return moe::set_error(MOE_ERR_ARG, "%s: router term arguments without w_router", fn);
+  if (router) {
+    if (T < 0 || k < 1 || k > 8 || k > E) return moe::set_error(MOE_ERR_ARG, "%s: T=%d k=%d", fn, T, k);
+    if (T > 0 && (!topk_gate || !d_gate || !row_of_assignment))
+      return moe::set_error(MOE_ERR_ARG, "%s: the router term needs topk_gate, d_gate and "
+                            "row_of_assignment", fn);
+    const int64_t Rr = moe_perm_rows_max(T, k, E);
+    if (rows_cap < Rr) return moe::set_error(MOE_ERR_ARG, "%s: rows_cap too small", fn);
+    const moe::WsLayout L = moe::ws_layout(T, d, E, k, F);
+    if (ws_bytes < L.total) return moe::set_error(MOE_ERR_WORKSPACE, "%s: workspace", fn);
+    float *row_dz = reinterpret_cast<float *>(static_cast<char *>(ws) + L.row_dz);
+    cudaError_t e = cudaMemsetAsync(row_dz, 0, size_t(Rr) * 4, s);
+    if (e != cudaSuccess) return moe::cuda_status(e, "moe_grouped_ffn_bwd_dgrad: zero row_dz");
+    if (T > 0) {
+      MOE_LAUNCH("router_row_dz", s, router_row_dz_kernel<<<grid_for(T), 256, 0, s>>>(
+                                         topk_gate, d_gate, row_of_assignment, T, k, Rr, row_dz));
+      if ((st = moe::launch_status("moe_grouped_ffn_bwd_dgrad: router rows"))) return st;
+    }
+    p.row_dz = row_dz;
+    p.w_router = w_router;
+  }
   p.group_offsets = group_offsets;
   p.E = E; p.d = d; p.F = F;
   // dH = dO W_down, fused SwiGLU backward -> [dA | dB]
@@ -1487,11 +1584,14 @@ int moe_grouped_ffn_bwd_wgrad_gather(const uint16_t *d_out_perm, const uint16_t 
 int moe_grouped_ffn_bwd(const uint16_t *d_out_perm, const uint16_t *x_perm,
                         const uint16_t *ab_saved, const uint16_t *h, const int32_t *group_offsets,
                         const uint8_t *active_mask, int E, int d, int F, int64_t rows_cap,
-                        const uint16_t *w_gate_up, const uint16_t *w_down, uint16_t *d_ab,
-                        uint16_t *dx_perm, uint16_t *dw_gate_up, uint16_t *dw_down, void *ws,
-                        size_t ws_bytes, moe_stream_t stream) {
+                        const uint16_t *w_gate_up, const uint16_t *w_down,
+                        const float *topk_gate, const float *d_gate,
+                        const int32_t *row_of_assignment, const float *w_router, int T, int k,
+                        uint16_t *d_ab, uint16_t *dx_perm, uint16_t *dw_gate_up,
+                        uint16_t *dw_down, void *ws, size_t ws_bytes, moe_stream_t stream) {
   if (int st = moe_grouped_ffn_bwd_dgrad(d_out_perm, ab_saved, group_offsets, E, d, F, rows_cap,
-                                         w_gate_up, w_down, d_ab, dx_perm, ws, ws_bytes, stream))
+                                         w_gate_up, w_down, topk_gate, d_gate, row_of_assignment,
+                                         w_router, T, k, d_ab, dx_perm, ws, ws_bytes, stream))
     return st;
   return moe_grouped_ffn_bwd_wgrad(d_out_perm, x_perm, h, d_ab, group_offsets, active_mask, E, d,
                                    F, rows_cap, dw_gate_up, dw_down, ws, ws_bytes, stream);

@@ -152,14 +152,16 @@ def backward(b: MoELayerBuffers, dy, w_router, w_gate_up, w_down, stream=None,
         side.wait_event(ev)
     L.moe_route_bwd(b.x, b.topk_idx, b.topk_gate, b.d_gate, s.T, s.d, s.E, s.k, b.d_logits,
                     b.dw_router, b.ws, b.ws_bytes, side)
+    # the router's term of dx is added to the grouped rows in the dX GEMM's epilogue
     L.moe_grouped_ffn_bwd_dgrad(b.d_out_perm, b.ab, b.group_offsets, s.E, s.d, s.F, R,
-                                w_gate_up, w_down, b.d_ab, b.dx_perm, b.ws, b.ws_bytes, main)
+                                w_gate_up, w_down, b.topk_gate, b.d_gate, b.row_of_assignment,
+                                w_router, s.T, s.k, b.d_ab, b.dx_perm, b.ws, b.ws_bytes, main)
     if overlap:
         ev = torch.cuda.Event()
         ev.record(main)
         side.wait_event(ev)
-    L.moe_permute_bwd(b.dx_perm, b.row_of_assignment, b.topk_idx, b.d_logits, w_router, s.T,
-                      s.d, s.E, s.k, b.dx, b.ws, b.ws_bytes, side)
+    L.moe_permute_bwd(b.dx_perm, b.row_of_assignment, b.topk_idx, None, None, s.T, s.d, s.E,
+                      s.k, b.dx, b.ws, b.ws_bytes, side)
     if b.gather:
         L.moe_grouped_ffn_bwd_wgrad_gather(b.d_out_perm, b.x, b.token_of_row, s.T, b.h, b.d_ab,
                                            b.group_offsets, active_mask, s.E, s.d, s.F, R,

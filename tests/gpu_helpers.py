@@ -76,3 +76,12 @@ def topk_margin(z32, k):
     if z.shape[1] <= k:
         z = np.concatenate([z, np.full((z.shape[0], 1), -np.inf)], axis=1)
     return (z[:, :-1] - z[:, 1:]).min(axis=1)
+
+
+def dx_perm_ref(ref, w_router, T, k):
+    """The oracle's per-assignment rows of dx_perm [T*k, d]: dX plus the router's term
+    d_logits[t,j] * W_r[:, e_j], which the dX GEMM's epilogue adds (moe_permute_bwd then
+    sums the rows without a router term)."""
+    wr = np.asarray(w_router, np.float64)
+    rows = ref["dX"] + ref["d_logits"][:, :, None] * wr.T[ref["topk_idx"]]
+    return rows.reshape(T * k, -1)

@@ -11,8 +11,8 @@ sys.path.insert(0, os.path.dirname(HERE))
 import numpy as np  # noqa: E402
 
 from oracle import moe_oracle as O  # noqa: E402
-from gpu_helpers import (assert_close, case_inputs, oracle_inputs, run_gpu_layer,  # noqa: E402
-                         to_np, unblock_ab)
+from gpu_helpers import (assert_close, case_inputs, dx_perm_ref, oracle_inputs,  # noqa: E402
+                         run_gpu_layer, to_np, unblock_ab)
 
 
 def check(T, d, E, k, F, n_masked):
@@ -35,7 +35,7 @@ def check(T, d, E, k, F, n_masked):
     assert_close("h", to_np(b.h)[flat], nrows(ref["h"]))
     assert_close("y", to_np(b.y), ref["y"])
     assert_close("dA", to_np(b.d_ab)[flat][:, :F], nrows(ref["dA"]))
-    assert_close("dX", to_np(b.dx_perm)[flat], nrows(ref["dX"]))
+    assert_close("dX", to_np(b.dx_perm)[flat], dx_perm_ref(ref, o["w_router"], T, k))
     assert_close("dw_down", to_np(b.dw_down), ref["dw_down"])
     assert_close("dw_gate_up", to_np(b.dw_gate_up), ref["dw_gate_up"])
     assert_close("dx", to_np(b.dx), ref["dx"])

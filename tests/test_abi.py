@@ -93,8 +93,8 @@ def test_argument_validation_without_launch(lib):
                                   stream=0)
         assert e.value.status == -6
         with pytest.raises(L.MoEError) as e:
-            L.moe_grouped_ffn_bwd_dgrad(16, 16, 16, 8, 256, 256, 4096, 16, 16, 16, 16, ws,
-                                        ws_bytes, stream=0)
+            L.moe_grouped_ffn_bwd_dgrad(16, 16, 16, 8, 256, 256, 4096, 16, 16, None, None, None,
+                                        None, 0, 1, 16, 16, ws, ws_bytes, stream=0)
         assert e.value.status == -6
         with pytest.raises(L.MoEError) as e:
             L.moe_grouped_ffn_bwd_wgrad(16, 16, 16, 16, 16, None, 8, 256, 256, 4096, 16, 16, ws,
@@ -205,6 +205,18 @@ def test_new_entry_points_validate_before_launch(lib):
     with pytest.raises(L.MoEError) as e:  # combine backward with neither output
         L.moe_unpermute_combine_bwd(16, 16, 16, 16, 16, 16, 10, 128, 8, 2, None, None, stream=0)
     assert e.value.status == -1
+    with pytest.raises(L.MoEError) as e:  # router term: with tokens, every per-token input
+        L.moe_grouped_ffn_bwd_dgrad(16, 16, 16, 8, 256, 256, 4096, 16, 16, 16, None, 16, 16, 10,
+                                    2, 16, 16, 16, 1 << 20, stream=0)
+    assert e.value.status == -1
+    with pytest.raises(L.MoEError) as e:  # router term inputs without w_router
+        L.moe_grouped_ffn_bwd_dgrad(16, 16, 16, 8, 256, 256, 4096, 16, 16, 16, 16, 16, None, 10,
+                                    2, 16, 16, 16, 1 << 20, stream=0)
+    assert e.value.status == -1
+    with pytest.raises(L.MoEError) as e:  # router term: workspace for the per-row dz
+        L.moe_grouped_ffn_bwd_dgrad(16, 16, 16, 8, 256, 256, 4096, 16, 16, 16, 16, 16, 16, 10,
+                                    2, 16, 16, 16, 256, stream=0)
+    assert e.value.status == -6
     for bad in (0, 999_999, 2_000_000_001):
         with pytest.raises(L.MoEError) as e:
             L.moe_selftest_wait_timeout(bad, stream=0)

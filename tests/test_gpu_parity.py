@@ -16,8 +16,8 @@ from oracle import moe_oracle as O
 from paper_2601_14327_gb300 import _lib as L
 from paper_2601_14327_gb300 import layer
 
-from gpu_helpers import (assert_close, case_inputs, oracle_inputs, rel_err, run_gpu_layer, to_np,
-                         topk_margin, unblock_ab)
+from gpu_helpers import (assert_close, case_inputs, dx_perm_ref, oracle_inputs, rel_err,
+                         run_gpu_layer, to_np, topk_margin, unblock_ab)
 
 pytestmark = pytest.mark.gpu
 
@@ -261,7 +261,7 @@ def test_layer_fwd_bwd_against_oracle(T, d, E, k, F, bias, n_masked):
     assert_close("d_gate", b.d_gate.cpu().numpy(), ref["d_gate"])
     assert_close("dA", to_np(b.d_ab)[flat][:, :F], nrows(ref["dA"]))
     assert_close("dB", to_np(b.d_ab)[flat][:, F:], nrows(ref["dB"]))
-    assert_close("dX", to_np(b.dx_perm)[flat], nrows(ref["dX"]))
+    assert_close("dX", to_np(b.dx_perm)[flat], dx_perm_ref(ref, o["w_router"], T, k))
     assert_close("dw_down", to_np(b.dw_down), ref["dw_down"])
     assert_close("dw_gate_up", to_np(b.dw_gate_up), ref["dw_gate_up"])
     assert_close("d_logits", b.d_logits.cpu().numpy(), ref["d_logits"])
@@ -441,6 +441,44 @@ def test_one_sm_gemm_kernel_against_oracle():
     r = subprocess.run([sys.executable, script], env=env, capture_output=True, text=True,
                        timeout=900)
     assert r.returncode == 0, r.stdout[-2000:] + r.stderr[-4000:]
+
+
+@pytest.mark.parametrize("T,d,E,k,F", [(1500, 384, 12, 4, 640), (3000, 256, 256, 8, 256)])
+def test_router_term_in_dx_epilogue_equals_unpermute_sum_form(T, d, E, k, F):
+    """The router's share of dx, added per grouped row in the dX GEMM's epilogue (the
+    layer's default), against the same term added per token by moe_permute_bwd: both
+    within the bf16 rounding of their sums, and both against the oracle."""
+    inp = case_inputs(T, d, E, k, F, seed=T + 1)
+    o = oracle_inputs(inp)
+    z = O.router_logits(o["x"], o["w_router"], o["bias"])
+    ref = O.moe_layer(o["x"], o["w_router"], o["bias"], None, k, o["w_gate_up"], o["w_down"],
+                      dy=o["dy"], logits32=z)
+    b = run_gpu_layer(inp, E, k, logits_in=z)
+    fused_dx = to_np(b.dx)
+    # recompute dX rows without the router term and sum them with moe_permute_bwd's
+    R = b.shape.rows_cap
+    g = {n: v.cuda() for n, v in inp.items()}
+    L.moe_grouped_ffn_bwd_dgrad(b.d_out_perm, b.ab, b.group_offsets, E, d, F, R, g["w_gate_up"],
+                                g["w_down"], None, None, None, None, T, k, b.d_ab, b.dx_perm,
+                                b.ws, b.ws_bytes)
+    flat = b.row_of_assignment.cpu().numpy().reshape(-1)
+    assert_close("dX without the router term", to_np(b.dx_perm)[flat], ref["dX"].reshape(T * k, -1))
+    dx2 = torch.empty_like(b.dx)
+    L.moe_permute_bwd(b.dx_perm, b.row_of_assignment, b.topk_idx, b.d_logits, g["w_router"], T,
+                      d, E, k, dx2, b.ws, b.ws_bytes)
+    torch.cuda.synchronize()
+    assert L.moe_device_error(clear=True) == 0
+    unfused_dx = to_np(dx2)
+    assert_close("dx (router term in the dX epilogue)", fused_dx, ref["dx"])
+    assert_close("dx (router term in the unpermute-sum)", unfused_dx, ref["dx"])
+    # the two differ only by where the bf16 roundings (unit roundoff u = 2^-9) fall: each
+    # form rounds its k rows (dX_j + router_j, or dX_j alone) and its final sum, so
+    # |fused - unfused| <= u * (sum_j |dX_j + router_j| + sum_j |dX_j| + 2 |dx|); the
+    # oracle's rows stand in for the GPU's, with a factor 2 for their own error
+    rows = dx_perm_ref(ref, o["w_router"], T, k).reshape(T, k, -1)
+    scale = (np.abs(rows).sum(axis=1) + np.abs(ref["dX"]).sum(axis=1)
+             + 2 * np.abs(ref["dx"]))
+    assert (np.abs(fused_dx - unfused_dx) <= 2.0 ** -8 * scale + 1e-30).all()
 
 
 def test_dynamic_schedule_equals_fixed_stride(tmp_path):

@@ -889,22 +889,30 @@ def run_call(args):
     for _ in range(args.warmup):
         fn()
     torch.cuda.synchronize()
+    clocks = ClockSampler(0)
+    clocks.start()
+    clocks.wait_first()
     L.moe_timing_enable(True)
     L.moe_timing_read(reset=True)
     stream = torch.cuda.current_stream()
     a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    clocks.mark_start()
     a.record(stream)
     for _ in range(args.steps):
         fn()
     b.record(stream)
     torch.cuda.synchronize()
+    clocks.mark_end()
+    clk = clocks.stop()
     L.moe_timing_enable(False)
     per_kernel = L.moe_timing_read(reset=True)
     assert L.moe_device_error(clear=True) == 0, "device error during the timed calls"
     ms = a.elapsed_time(b)
     tflops_peak, peak_source = tensor_peak(peaks, ms / 1e3)
-    table = kernel_report(wl, per_kernel, args.steps, peaks, tflops_peak, wl.live_counts())
-    print(json.dumps({"call": args.call, "workload": wl.cfg.name,
+    table = kernel_report(wl, per_kernel, args.steps, peaks, tflops_peak, wl.live_counts(),
+                          sm_mhz=clk.get("sm_mhz"))
+    print(json.dumps({"call": args.call, "workload": wl.cfg.name, "clocks": clk,
                       "config": {"T": wl.shape.T, "d_model": wl.shape.d, "experts": wl.shape.E,
                                  "top_k": wl.shape.k, "d_ff": wl.shape.F},
                       "calls": args.steps, "ms_per_call": round(ms / args.steps, 4),

@@ -49,6 +49,7 @@ constexpr uint64_t kRtWaitNs = 2000000000ull;
 
 struct RouteTcParams {
   int M;             // output rows: tokens (logits) or d_model (router weight gradient)
+  int MT;            // 128-row tiles per CTA (1 or 2); tile m's accumulator at TMEM column 256*m
   int kb_per_split;  // k-blocks of one split
   int nkb;           // k-blocks of the reduction (over d, or over the padded tokens)
   int NP;            // MMA N: experts rounded up to 16
@@ -60,10 +61,19 @@ struct RouteTcParams {
 
 // Experts rounded up to the MMA's N granularity, and the matching TMEM allocation.
 int route_tc_np(int E) { return (E + 15) / 16 * 16; }
-uint32_t route_tc_tmem_cols(int NP) { return NP <= 32 ? 32u : (NP <= 64 ? 64u : (NP <= 128 ? 128u : 256u)); }
-uint32_t route_tc_stage_bytes(int NP) { return kRtABytes + 3u * uint32_t(NP) * 128u; }
-size_t route_tc_smem(int NP, int stages) {
-  return 1024 + size_t(stages) * route_tc_stage_bytes(NP) + size_t(2 * stages + 1) * 8 + 16;
+// 128-row tiles per CTA: two above 96 experts (up to 192), where the three weight terms of a
+// k-block (3 x NP x 128 bytes) outweigh the 16 KB x tile: two x tiles share each weight stage,
+// halving the L2 reads of the weight terms per FLOP; one CTA per SM either way.
+int route_tc_mt(int NP) { return (NP > 96 && NP <= 192) ? 2 : 1; }
+uint32_t route_tc_tmem_cols(int NP, int MT) {
+  if (MT == 2) return 512u;
+  return NP <= 32 ? 32u : (NP <= 64 ? 64u : (NP <= 128 ? 128u : 256u));
+}
+uint32_t route_tc_stage_bytes(int NP, int MT = 1) {
+  return uint32_t(MT) * kRtABytes + 3u * uint32_t(NP) * 128u;
+}
+size_t route_tc_smem(int NP, int stages, int MT = 1) {
+  return 1024 + size_t(stages) * route_tc_stage_bytes(NP, MT) + size_t(2 * stages + 1) * 8 + 16;
 }
 // Two CTAs per SM with a ring of at least two stages each where that fits (more
 // independent x streams per SM: measured faster than one CTA with a deeper ring), else
@@ -76,7 +86,7 @@ int route_tc_stages(int NP) {
   if (route_tc_two_per_sm(NP)) {
     while (st < 8 && 2 * (route_tc_smem(NP, st + 1) + 1024) <= size_t(kRtSmemPerSm)) ++st;
   } else {
-    st = int((kRtMaxSmem - 2048) / route_tc_stage_bytes(NP));
+    st = int((kRtMaxSmem - 2048) / route_tc_stage_bytes(NP, route_tc_mt(NP)));
   }
   return std::min(8, st);
 }
@@ -84,7 +94,8 @@ int route_tc_stages(int NP) {
 // for the logits, d_model for the weight gradient) give few tiles. A function of
 // (M, K, NP) alone, so the workspace size is too. K > 0.
 void route_tc_split(int M, int K, int NP, int *splits, int *kb_per_split) {
-  const int tiles = std::max(1, (M + kRtBM - 1) / kRtBM);
+  const int rows = kRtBM * route_tc_mt(NP);
+  const int tiles = std::max(1, (M + rows - 1) / rows);
   const int nkb = (K + kRtBK - 1) / kRtBK;
   const int target = kRtSms * (route_tc_two_per_sm(NP) ? 2 : 1);
   int s = std::max(1, std::min({target / tiles, kRtMaxSplits, nkb}));
@@ -139,7 +150,8 @@ __global__ void __launch_bounds__(kRtThreads, 1)
   const uint32_t raw = tc::smem_u32(smem_raw);
   const uint32_t pad = (1024u - (raw & 1023u)) & 1023u;
   const uint32_t b_bytes = uint32_t(p.NP) * 128u;
-  const uint32_t stage_bytes = kRtABytes + 3u * b_bytes;
+  const uint32_t a_bytes = uint32_t(p.MT) * kRtABytes;  // the CTA's x tiles of a k-block
+  const uint32_t stage_bytes = a_bytes + 3u * b_bytes;
   const int S = p.stages;
   const uint32_t s0 = raw + pad;
   uint64_t *bars = reinterpret_cast<uint64_t *>(smem_raw + pad + size_t(S) * stage_bytes);
@@ -196,15 +208,19 @@ __global__ void __launch_bounds__(kRtThreads, 1)
       tc::mbar_arrive_expect_tx(full_bar(s), stage_bytes);
       const uint32_t dst = s0 + s * stage_bytes;
       const int k0 = kb * kRtBK;
-      if (DW) {  // x^T: features mt*128 .. +127 (two 64-wide boxes) x tokens k0 .. k0+63
-        tc::tma_load_2d(dst, &tmX, full_bar(s), mt * kRtBM, k0);
-        tc::tma_load_2d(dst + 64 * 128, &tmX, full_bar(s), mt * kRtBM + 64, k0);
-      } else {
-        tc::tma_load_2d(dst, &tmX, full_bar(s), k0, mt * kRtBM);
+      for (int m = 0; m < p.MT; ++m) {
+        const int row0 = (mt * p.MT + m) * kRtBM;
+        const uint32_t am = dst + uint32_t(m) * kRtABytes;
+        if (DW) {  // x^T: features row0 .. +127 (two 64-wide boxes) x tokens k0 .. k0+63
+          tc::tma_load_2d(am, &tmX, full_bar(s), row0, k0);
+          tc::tma_load_2d(am + 64 * 128, &tmX, full_bar(s), row0 + 64, k0);
+        } else {
+          tc::tma_load_2d(am, &tmX, full_bar(s), k0, row0);
+        }
       }
 #pragma unroll
       for (int j = 0; j < 3; ++j)
-        tc::tma_load_2d(dst + kRtABytes + j * b_bytes, &tmW, full_bar(s), k0, j * p.NP);
+        tc::tma_load_2d(dst + a_bytes + j * b_bytes, &tmW, full_bar(s), k0, j * p.NP);
     }
     // every issued load lands before the CTA may exit (also after an abort)
     for (int s = 0; s < S; ++s) {
@@ -227,15 +243,19 @@ __global__ void __launch_bounds__(kRtThreads, 1)
         break;
       }
       tc::fence_after_sync();
-      const uint32_t a_s = s0 + s * stage_bytes, b_s = a_s + kRtABytes;
+      const uint32_t a_s = s0 + s * stage_bytes, b_s = a_s + a_bytes;
+      for (int m = 0; m < p.MT; ++m) {
+        const uint32_t am = a_s + uint32_t(m) * kRtABytes;
 #pragma unroll
-      for (int kk = 0; kk < kRtBK / 16; ++kk) {
-        const uint64_t ad = DW ? tc::smem_desc_sw128(a_s + kk * 2048, 8192, 1024)
-                               : tc::smem_desc_sw128(a_s + kk * 32, 16, 1024);
+        for (int kk = 0; kk < kRtBK / 16; ++kk) {
+          const uint64_t ad = DW ? tc::smem_desc_sw128(am + kk * 2048, 8192, 1024)
+                                 : tc::smem_desc_sw128(am + kk * 32, 16, 1024);
 #pragma unroll
-        for (int j = 0; j < 3; ++j) {
-          const uint64_t bd = tc::smem_desc_sw128(b_s + j * b_bytes + kk * 32, 16, 1024);
-          tc::mma_bf16(tmem_base, ad, bd, idesc, (it != 0 || kk != 0 || j != 0) ? 1u : 0u);
+          for (int j = 0; j < 3; ++j) {
+            const uint64_t bd = tc::smem_desc_sw128(b_s + j * b_bytes + kk * 32, 16, 1024);
+            tc::mma_bf16(tmem_base + uint32_t(m) * 256u, ad, bd, idesc,
+                         (it != 0 || kk != 0 || j != 0) ? 1u : 0u);
+          }
         }
       }
       tc::mma_commit(empty_bar(s));
@@ -258,16 +278,20 @@ __global__ void __launch_bounds__(kRtThreads, 1)
   ok = __shfl_sync(0xffffffffu, ok, 0);
   if (ok) {
     tc::fence_after_sync();
-    const int t = mt * kRtBM + warp * 32 + lane;
-    float *dst = p.partial + (size_t(split) * p.M + t) * p.NE;
-    for (int c0 = 0; c0 < p.NP; c0 += 32) {
-      uint32_t r[32];
-      tc::tmem_ld_32x32b_x32(tmem_base + (uint32_t(warp * 32) << 16) + uint32_t(c0), r);
-      tc::tmem_ld_wait();
-      if (t < p.M) {
+    for (int m = 0; m < p.MT; ++m) {
+      const int t = (mt * p.MT + m) * kRtBM + warp * 32 + lane;
+      float *dst = p.partial + (size_t(split) * p.M + t) * p.NE;
+      for (int c0 = 0; c0 < p.NP; c0 += 32) {
+        uint32_t r[32];
+        tc::tmem_ld_32x32b_x32(tmem_base + (uint32_t(warp * 32) << 16) + uint32_t(m) * 256u +
+                                   uint32_t(c0),
+                               r);
+        tc::tmem_ld_wait();
+        if (t < p.M) {
 #pragma unroll
-        for (int q = 0; q < 8; ++q)
-          stg_v4(dst + c0 + 4 * q, make_uint4(r[4 * q], r[4 * q + 1], r[4 * q + 2], r[4 * q + 3]));
+          for (int q = 0; q < 8; ++q)
+            stg_v4(dst + c0 + 4 * q, make_uint4(r[4 * q], r[4 * q + 1], r[4 * q + 2], r[4 * q + 3]));
+        }
       }
     }
   }
@@ -460,9 +484,9 @@ __global__ void zero_f32_kernel(float *p, int n) {
 // (token tile, split). Returns the number of partial planes written in *splits.
 int launch_route_tc(const uint16_t *x, const float *w, int T, int d, int E, int NE, uint16_t *w3,
                     float *partial, int *splits_out, cudaStream_t s) {
-  const int NP = route_tc_np(E);
+  const int NP = route_tc_np(E), MT = route_tc_mt(NP);
   const int stages = route_tc_stages(NP);
-  const size_t smem = route_tc_smem(NP, stages);
+  const size_t smem = route_tc_smem(NP, stages, MT);
   static bool attr_set = false;
   if (!attr_set) {
     cudaError_t e = cudaFuncSetAttribute(route_tc_kernel<false>,
@@ -482,14 +506,15 @@ int launch_route_tc(const uint16_t *x, const float *w, int T, int d, int E, int 
   route_tc_split(T, d, route_tc_np(E), &splits, &per);
   RouteTcParams p;
   p.M = T;
+  p.MT = MT;
   p.kb_per_split = per;
   p.nkb = (d + kRtBK - 1) / kRtBK;
   p.NP = NP;
   p.NE = NE;
   p.stages = stages;
-  p.tmem_cols = route_tc_tmem_cols(NP);
+  p.tmem_cols = route_tc_tmem_cols(NP, MT);
   p.partial = partial;
-  dim3 grid((T + kRtBM - 1) / kRtBM, splits);
+  dim3 grid((T + kRtBM * MT - 1) / (kRtBM * MT), splits);
   MOE_LAUNCH("route_logits", s, route_tc_kernel<false><<<grid, kRtThreads, smem, s>>>(mx, mw, p));
   *splits_out = splits;
   return moe::launch_status("moe_route: logits");
@@ -589,9 +614,9 @@ namespace {
 // Weight-gradient launch on the tensor cores: partial[split][i][e] over the split's tokens.
 int launch_route_dw(const uint16_t *x, const uint16_t *dz3, int T, int d, int E, float *partial,
                     int *splits_out, cudaStream_t s) {
-  const int NP = route_tc_np(E), Tp = route_tokens_padded(T);
+  const int NP = route_tc_np(E), Tp = route_tokens_padded(T), MT = route_tc_mt(NP);
   const int stages = route_tc_stages(NP);
-  const size_t smem = route_tc_smem(NP, stages);
+  const size_t smem = route_tc_smem(NP, stages, MT);
   static bool attr_set = false;
   if (!attr_set) {
     cudaError_t e = cudaFuncSetAttribute(route_tc_kernel<true>,
@@ -609,14 +634,15 @@ int launch_route_dw(const uint16_t *x, const uint16_t *dz3, int T, int d, int E,
   route_tc_split(d, Tp, NP, &splits, &per);
   RouteTcParams p;
   p.M = d;
+  p.MT = MT;
   p.kb_per_split = per;
   p.nkb = Tp / kRtBK;
   p.NP = NP;
   p.NE = route_dw_stride(E);
   p.stages = stages;
-  p.tmem_cols = route_tc_tmem_cols(NP);
+  p.tmem_cols = route_tc_tmem_cols(NP, MT);
   p.partial = partial;
-  dim3 grid((d + kRtBM - 1) / kRtBM, splits);
+  dim3 grid((d + kRtBM * MT - 1) / (kRtBM * MT), splits);
   MOE_LAUNCH("route_bwd_dw", s, route_tc_kernel<true><<<grid, kRtThreads, smem, s>>>(mx, mz, p));
   *splits_out = splits;
   return moe::launch_status("moe_route_bwd: weight gradient");

@@ -70,6 +70,9 @@ def test_route_ties_go_to_lower_index():
 
 
 @pytest.mark.parametrize("T,d,E", [(777, 512, 64), (300, 1024, 171), (129, 256, 256),
+                                   # two 128-token tiles per CTA (97..192 experts), the second
+                                   # one partly past T
+                                   (1000, 384, 100), (2500, 7168, 171),
                                    # d not a multiple of the 64-wide k-block (zero-filled tail),
                                    # few experts (MMA N = 16), one token, the smallest d
                                    (333, 200, 13), (1, 72, 256), (64, 8, 5), (50, 136, 2)])
@@ -92,6 +95,9 @@ def test_route_logits_fp32(T, d, E):
 
 
 @pytest.mark.parametrize("T,d,E,k", [(3000, 256, 64, 8), (777, 512, 171, 4), (129, 200, 256, 8),
+                                     # two 128-feature tiles per CTA, the second one partly
+                                     # past d
+                                     (1000, 384, 120, 4),
                                      # tokens not a multiple of the 64-token k-block, d not a
                                      # multiple of the 128-feature tile, MMA N = 16, one token
                                      (333, 136, 13, 2), (1, 72, 5, 1), (64, 8, 2, 2),

@@ -98,10 +98,10 @@ int64_t moe_perm_rows_max(int T, int k, int E);
 
 /* Bytes of scratch `ws` every device entry point below may use for a layer of
  * this shape (one buffer serves all calls of a step issued on one stream).
- * Its first 256 bytes hold the grouped GEMMs' tile counter: the moe_grouped_ffn_*
- * entry points need a ws of at least 256 bytes (16-byte aligned) and only use
- * those; two GEMM calls whose kernels may overlap on the GPU need separate
- * workspaces. The other calls use disjoint regions after them, so the router
+ * Its first 256 bytes hold the weight-gradient GEMMs' tile counter: the
+ * moe_grouped_ffn_* entry points need a ws of at least 256 bytes (16-byte
+ * aligned), and two weight-gradient calls whose kernels may overlap on the GPU
+ * need separate workspaces. The other calls use disjoint regions after them, so the router
  * backward and the unpermute-sum may share one workspace with GEMM calls running
  * beside them on another stream. */
 size_t moe_workspace_size(int T, int d, int E, int k, int F);
@@ -261,11 +261,14 @@ int moe_permute_noalloc(const uint16_t *x, const int32_t *topk_idx, const int32_
  * Groups of 0 rows cost nothing. ws: at least 256 bytes, 16-byte aligned (the
  * tile counter; see moe_workspace_size).
  * Schedule (all moe_grouped_ffn_* GEMMs): the tiles are listed heaviest expert
- * first, the longest-processing-time order of Algorithm 2's greedy; CTA pairs
- * that run out of work take the next tile of the list from a shared counter, so
- * the heaviest tile left always goes to the least-loaded pair (Algorithm 2 with
- * the GPU's CTA pairs as its devices, applied online). A tile's arithmetic does
- * not depend on which pair runs it: results are bitwise reproducible.
+ * first, the longest-processing-time order of Algorithm 2's greedy. In the
+ * weight-gradient GEMMs, whose tiles cost as much as their expert has rows, CTA
+ * pairs that run out of work take the next tile of the list from a counter in
+ * ws, so the heaviest tile left always goes to the least-loaded pair (Algorithm 2
+ * with the GPU's CTA pairs as its devices, applied online); the other GEMMs'
+ * tiles all cost the same and each pair takes every 76th one. A tile's
+ * arithmetic does not depend on which pair runs it: results are bitwise
+ * reproducible.
  * Limits: d % 128 == 0, F % 128 == 0, all pointers 16-byte aligned.
  */
 int moe_grouped_ffn_fwd(const uint16_t *x_perm, const int32_t *group_offsets, int E, int d,

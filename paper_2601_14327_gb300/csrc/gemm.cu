@@ -781,18 +781,27 @@ __global__ void __launch_bounds__(kThreads, 1)
     return t;
   };
 
-  // ---- tile hand-off. The even CTA's producer takes tile number n of this pair: the
-  // pair's index for n = 0, then the next unclaimed tile of the list (an atomic counter
-  // shared by all pairs; p.dynamic == 0: every nclusters-th tile), -1 once the list is
-  // exhausted. It writes the tile into slot n % kRing of both CTAs' rings and arrives on
-  // the slots' barriers before it issues the tile's loads; the odd CTA's producer and
-  // the MMA issuer wait there. The MMA issuer passes each tile on to both CTAs' epilogue
-  // warps through s_epi[buffer] and epi_bar[buffer] once that accumulator buffer is free.
+  // ---- tile numbers. The weight gradients' tiles differ in cost (K = the expert's rows):
+  // there the even CTA's producer takes tile number n of this pair, the pair's index for
+  // n = 0, then the next unclaimed tile of the list (an atomic counter shared by all
+  // pairs), -1 once the list is exhausted. It writes the tile into slot n % kRing of both
+  // CTAs' rings and arrives on the slots' barriers before it issues the tile's loads; the
+  // odd CTA's producer and the MMA issuer wait there, and the MMA issuer passes each tile
+  // on to both CTAs' epilogue warps through s_epi[buffer] and epi_bar[buffer] once that
+  // accumulator buffer is free. The activation GEMMs' tiles all cost the same (and with
+  // p.dynamic == 0 the weight gradients' too): every role of a pair then computes its tile
+  // numbers itself, cluster, cluster + nclusters, ..., with no hand-off.
+  const bool dyn = Tr::WGRAD && p.dynamic;
+  auto static_tile = [&](uint32_t n) -> int {
+    const int tile = cluster + int(n) * nclusters;
+    return tile < total ? tile : -1;
+  };
   const uint32_t ring_peer = tc::mapa(tc::smem_u32(const_cast<int *>(s_ring)), 1);
   const uint32_t ring_bar_peer = tc::mapa(ring_bar(0), 1);
   int claimed = cluster;  // even CTA's producer: the tile it publishes next
   // Returns this pair's tile number n (-1: no more), or -2 after a failed wait.
   auto next_tile = [&](uint32_t n) -> int {
+    if (!dyn) return static_tile(n);
     const int slot = int(n % kRing);
     if (leader) {
       const int v = claimed < total ? claimed : -1;
@@ -800,7 +809,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       tc::st_cluster_u32(ring_peer + 4u * slot, v);
       tc::mbar_arrive(ring_bar(slot));
       tc::mbar_arrive_cluster(ring_bar_peer + 8u * slot);
-      if (v >= 0) claimed = p.dynamic ? nclusters + atomicAdd(p.sched_ctr, 1) : claimed + nclusters;
+      if (v >= 0) claimed = nclusters + atomicAdd(p.sched_ctr, 1);
       return v;
     }
     if (!tc::mbar_wait_cluster(ring_bar(slot), (n / kRing) & 1u, kWaitLimitNs, abort_flag)) {
@@ -940,16 +949,24 @@ __global__ void __launch_bounds__(kThreads, 1)
       uint32_t it = 0;
       bool ok = true, issued = false;
       for (uint32_t n = 0; ok; ++n) {
-        const int slot = int(n % kRing);
-        if (!tc::mbar_wait(ring_bar(slot), (n / kRing) & 1u, kWaitLimitNs, abort_flag)) { fail(abort_flag); break; }
-        const int tile = s_ring[slot];
+        int tile;
+        if (dyn) {
+          const int slot = int(n % kRing);
+          if (!tc::mbar_wait(ring_bar(slot), (n / kRing) & 1u, kWaitLimitNs, abort_flag)) { fail(abort_flag); break; }
+          tile = s_ring[slot];
+        } else {
+          tile = static_tile(n);
+          if (tile < 0) break;
+        }
         const uint32_t a = n & 1u, aph = (n >> 1) & 1u;
         if (!tc::mbar_wait(tempty_bar(a), aph ^ 1u, kWaitLimitNs, abort_flag)) { fail(abort_flag); break; }
-        // the epilogue warps of both CTAs learn the tile of buffer a (-1: no more tiles)
-        s_epi[a] = tile;
-        tc::st_cluster_u32(epi_peer + 4u * a, tile);
-        tc::mbar_arrive(epi_bar(a));
-        tc::mbar_arrive_cluster(epi_bar_peer + 8u * a);
+        if (dyn) {
+          // the epilogue warps of both CTAs learn the tile of buffer a (-1: no more tiles)
+          s_epi[a] = tile;
+          tc::st_cluster_u32(epi_peer + 4u * a, tile);
+          tc::mbar_arrive(epi_bar(a));
+          tc::mbar_arrive_cluster(epi_bar_peer + 8u * a);
+        }
         if (tile < 0) break;
         tc::fence_after_sync();
         const PairTile t = decode(tile);
@@ -1008,10 +1025,16 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     for (uint32_t n = 0;; ++n) {
       const uint32_t a = n & 1u, aph = (n >> 1) & 1u;
-      bool ok = tc::mbar_wait_cluster(epi_bar(a), aph, kWaitLimitNs, abort_flag);
-      __syncwarp();
-      if (!ok) { fail(abort_flag); break; }
-      const int tile = s_epi[a];
+      bool ok = true;
+      int tile;
+      if (dyn) {
+        ok = tc::mbar_wait_cluster(epi_bar(a), aph, kWaitLimitNs, abort_flag);
+        __syncwarp();
+        if (!ok) { fail(abort_flag); break; }
+        tile = s_epi[a];
+      } else {
+        tile = static_tile(n);
+      }
       if (tile < 0) break;
       const PairTile t = decode(tile);
       const int mt = 2 * t.mp + int(rank);
@@ -1165,6 +1188,7 @@ int run_gemm_out(int N, const void *a_base, uint64_t a_rows, uint64_t a_cols, co
                  uint64_t o_cols, GemmParams p, cudaStream_t s, const char *what) {
   using Tr = Traits<MODE>;
   const bool pair = use_pair<MODE>();
+  if (!Tr::WGRAD) p.dynamic = 0;  // equal-cost tiles: fixed stride, no counter to reset
   const int BN = (MODE == kGateUp || N % 256 == 0) ? 256 : 128;
   p.n_tiles = (MODE == kGateUp) ? N / 256 : N / BN;
   const bool gather = p.token_of_row != nullptr;

@@ -260,15 +260,15 @@ int moe_permute_noalloc(const uint16_t *x, const int32_t *topk_idx, const int32_
  * out_perm [rows_cap,d] bf16. Only rows below group_offsets[E] are written.
  * Groups of 0 rows cost nothing. ws: at least 256 bytes, 16-byte aligned (the
  * tile counter; see moe_workspace_size).
- * Schedule (all moe_grouped_ffn_* GEMMs): the tiles are listed heaviest expert
- * first, the longest-processing-time order of Algorithm 2's greedy. In the
- * weight-gradient GEMMs, whose tiles cost as much as their expert has rows, CTA
- * pairs that run out of work take the next tile of the list from a counter in
+ * Schedule (all moe_grouped_ffn_* GEMMs): in the weight-gradient GEMMs, whose
+ * tiles cost as much as their expert has rows, the tiles are listed heaviest
+ * expert first (the longest-processing-time order of Algorithm 2's greedy) and
+ * CTA pairs that run out of work take the next tile of the list from a counter in
  * ws, so the heaviest tile left always goes to the least-loaded pair (Algorithm 2
  * with the GPU's CTA pairs as its devices, applied online); the other GEMMs'
- * tiles all cost the same and each pair takes every 76th one. A tile's
- * arithmetic does not depend on which pair runs it: results are bitwise
- * reproducible.
+ * tiles all cost the same, are listed in expert order and each pair takes every
+ * 76th one. A tile's arithmetic does not depend on which pair runs it: results
+ * are bitwise reproducible.
  * Limits: d % 128 == 0, F % 128 == 0, all pointers 16-byte aligned.
  */
 int moe_grouped_ffn_fwd(const uint16_t *x_perm, const int32_t *group_offsets, int E, int d,

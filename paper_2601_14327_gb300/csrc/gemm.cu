@@ -384,9 +384,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc::tmem_relinquish();
   }
   // ---- tile schedule, built from the device-resident group offsets ----
-  // Experts heaviest first (ties to the lower id); in the weight-gradient modes pruned
-  // experts (active_mask 0) come last with no tile, live experts without rows get tiles
-  // of zero k-blocks (their zero gradient).
+  // Weight gradients: experts heaviest first (ties to the lower id), pruned experts
+  // (active_mask 0) last with no tile, live experts without rows with tiles of zero
+  // k-blocks (their zero gradient). Activation GEMMs: expert order.
   for (int e = threadIdx.x; e <= E; e += kThreads) s_goff[e] = p.group_offsets[e];
   __syncthreads();
   auto sort_key = [&](int e) {
@@ -394,6 +394,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     return (Tr::WGRAD && p.active_mask != nullptr && p.active_mask[e] == 0) ? -1 : rows;
   };
   for (int e = threadIdx.x; e < E; e += kThreads) {
+    if (!Tr::WGRAD) {  // equal-cost tiles: expert order, the grouped layout's memory order
+      s_order[e] = e;
+      continue;
+    }
     const int ce = sort_key(e);
     int r = 0;
     for (int q = 0; q < E; ++q) {
@@ -698,12 +702,14 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc::tmem_relinquish_pair();
   }
   // ---- tile list: identical in both CTAs of every pair ----
-  // Experts in descending order of rows (ties to the lower id): the longest-processing-
-  // time order of Algorithm 2's greedy balancing. A pair that runs out of work claims the
-  // next tile of this list, i.e. the heaviest tile left goes to the least-loaded pair.
-  // Weight gradients: pruned experts (active_mask 0) come last and get nothing; live
-  // experts without rows come before them and get no tile either (their zero gradients
-  // are stored by the epilogue warps up front, while the first tiles' MMAs run).
+  // Weight gradients (a tile costs as much as its expert has rows): experts in descending
+  // order of rows (ties to the lower id), the longest-processing-time order of Algorithm
+  // 2's greedy balancing; a pair that runs out of work claims the next tile of this list,
+  // i.e. the heaviest tile left goes to the least-loaded pair. Pruned experts (active_mask
+  // 0) come last and get nothing; live experts without rows come before them and get no
+  // tile either (their zero gradients are stored by the epilogue warps up front, while the
+  // first tiles' MMAs run). Activation GEMMs (every tile costs the same): expert order,
+  // which follows the grouped layout in memory (measured 1-2% faster than heaviest first).
   for (int e = threadIdx.x; e <= E; e += kThreads) s_goff[e] = p.group_offsets[e];
   __syncthreads();
   auto sort_key = [&](int e) {
@@ -711,6 +717,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     return (Tr::WGRAD && p.active_mask != nullptr && p.active_mask[e] == 0) ? -1 : rows;
   };
   for (int e = threadIdx.x; e < E; e += kThreads) {
+    if (!Tr::WGRAD) {  // equal-cost tiles: expert order, the grouped layout's memory order
+      s_order[e] = e;
+      continue;
+    }
     const int ce = sort_key(e);
     int r = 0;
     for (int q = 0; q < E; ++q) {

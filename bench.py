@@ -193,7 +193,7 @@ class Workload:
     """Inputs, the one-time LAEP prune, and the buffers of one layer step."""
 
     def __init__(self, cfg_id: int, device: str, compact_override=None, tokens=None,
-                 experts=None, no_prune=False, bias=None, gather=False, overlap=True,
+                 experts=None, no_prune=False, bias=None, gather=False, overlap=False,
                  backward=None, fused_combine=False):
         c = synth.CONFIGS[cfg_id]
         if tokens or experts or no_prune or bias:  # a variant of the workload (profiling)
@@ -997,9 +997,9 @@ def main():
     ap.add_argument("--fused-combine", type=int, default=0,
                     help="combine in a separate kernel (0) or in the down GEMM's epilogue with "
                          "fp32 atomics (1; y's last bits may vary from run to run)")
-    ap.add_argument("--overlap", type=int, default=1,
+    ap.add_argument("--overlap", type=int, default=0,
                     help="router backward and unpermute-sum on a second stream beside the "
-                         "GEMMs (1) or on the main stream after them (0)")
+                         "GEMMs (1) or on the main stream after them (0, the default)")
     ap.add_argument("--flush-l2", action="store_true",
                     help="rewrite a 256 MB buffer before every timed step (time the steps only)")
     ap.add_argument("--graph", type=int, default=1,

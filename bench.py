@@ -87,11 +87,22 @@ def measured_peaks():
     if os.path.exists(path):
         with open(path) as f:
             p = json.load(f)
+        clk = (p.get("clocks_under_load") or {}).get("sm_mhz_median")
         return {"hbm_gbs": p["hbm_gbs"], "bf16_tflops": p["bf16_tflops"],
                 "bf16_tflops_sustained": p.get("bf16_tflops_sustained", p["bf16_tflops"]),
-                "source": "measured"}
+                "sustained_sm_mhz": clk, "source": "measured"}
     return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0,
-            "source": "fallback"}
+            "sustained_sm_mhz": None, "source": "fallback"}
+
+
+def per_clock_frac(tflops, sm_mhz, peaks):
+    """TFLOP/s per MHz of SM clock against the sustained cuBLAS run's TFLOP/s per MHz at its
+    own median clock: the fraction of the reference's work per clock, which clock
+    differences between the two measurements do not inflate (None without both clocks)."""
+    ref_mhz = peaks.get("sustained_sm_mhz")
+    if not sm_mhz or not ref_mhz:
+        return None
+    return round((tflops / sm_mhz) / (peaks["bf16_tflops_sustained"] / ref_mhz), 4)
 
 
 def tensor_peak(peaks, region_s):
@@ -492,6 +503,7 @@ def kernel_report(wl, per_kernel, steps, peaks, tflops_peak, counts, sm_mhz=None
                      group_bound_frac=round(bound[n] / per_launch_s, 4))
             if sm_mhz:
                 e["gflops_per_mhz"] = round(tf * 1e3 / sm_mhz, 1)
+                e["frac_per_clock"] = per_clock_frac(tf, sm_mhz, peaks)
         elif n in hbm:
             gbs = hbm[n] / per_launch_s / 1e9
             e.update(gbs=round(gbs, 1), frac=round(gbs / peaks["hbm_gbs"], 4),
@@ -754,6 +766,8 @@ def run_ours(args):
                          "gflops_per_mhz": (round(all_gemm_tflops * 1e3 / clk_eager["sm_mhz"], 1)
                                             if clk_eager.get("sm_mhz") else None),
                          "sm_mhz": clk_eager.get("sm_mhz"),
+                         "frac_per_clock": per_clock_frac(all_gemm_tflops, clk_eager.get("sm_mhz"),
+                                                          peaks),
                          "ms_per_step": round(all_gemm_ms, 4),
                          "group_bound_frac": round(gemm_bound_frac, 4),
                          "group_bound": "sum over live experts of max(FLOPs/tensor peak, "
@@ -761,6 +775,10 @@ def run_ours(args):
         "roofline": {"kernel": dom, "bound": "tensor", "achieved": round(dom_tflops, 1),
                      "peak": tflops_peak, "unit": "TFLOP/s", "frac": round(dom_tflops / tflops_peak, 4),
                      "frac_nominal": round(dom_tflops / BF16_NOMINAL_TFLOPS, 4),
+                     "frac_per_clock": per_clock_frac(dom_tflops, clk_eager.get("sm_mhz"), peaks),
+                     "frac_per_clock_note": "TFLOP/s per MHz of SM clock over the sustained cuBLAS "
+                                            "run's TFLOP/s per MHz at its median clock "
+                                            "(clocks_under_load of MEASURED_PEAKS.json)",
                      "traffic": committed_traffic(c.name, dom) if default_workload else None,
                      "peak_source": peak_source,
                      "achieved_from": f"algorithmic FLOPs of one launch / mean CUDA-event "

@@ -90,3 +90,13 @@ def test_oracle_sample_on_routed_experts_equals_the_full_layer():
     np.testing.assert_array_equal(sub["dw_down"], full["dw_down"][used])
     np.testing.assert_array_equal(sub["dw_router"], full["dw_router"][:, used])
     assert not full["dw_gate_up"][np.setdiff1d(np.arange(E), used)].any()
+
+
+def test_per_clock_fraction_discounts_the_clock_difference():
+    peaks = {"bf16_tflops_sustained": 1575.5, "sustained_sm_mhz": 1342.0}
+    # the same work per clock as the reference at a higher clock is 1.0, not above it
+    assert bench.per_clock_frac(1575.5 * 1500 / 1342, 1500.0, peaks) == 1.0
+    assert bench.per_clock_frac(1496.0, 1485.0, peaks) == round((1496 / 1485) / (1575.5 / 1342), 4)
+    assert bench.per_clock_frac(1496.0, None, peaks) is None
+    assert bench.per_clock_frac(1496.0, 1485.0, {"bf16_tflops_sustained": 1.0,
+                                                "sustained_sm_mhz": None}) is None

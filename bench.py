@@ -821,11 +821,11 @@ def layer_calls(wl):
         "combine": lambda: L.moe_unpermute_combine(b.out_perm, b.row_of_assignment, b.topk_gate,
                                                    s.T, s.d, s.k, b.y),
         "combine_bwd": lambda: L.moe_unpermute_combine_bwd(
-            i["dy"], b.out_perm, b.row_of_assignment, b.topk_gate, b.group_offsets,
-            b.group_counts, s.T, s.d, s.E, s.k, b.d_out_perm, b.d_gate),
+            i["dy"], None, b.row_of_assignment, b.topk_gate, b.group_offsets,
+            b.group_counts, s.T, s.d, s.E, s.k, b.d_out_perm, None),
         "ffn_bwd_dgrad": lambda: L.moe_grouped_ffn_bwd_dgrad(
             b.d_out_perm, b.ab, b.group_offsets, s.E, s.d, s.F, R, i["w_gate_up"], i["w_down"],
-            b.topk_gate, b.d_gate, b.row_of_assignment, i["w_router"], s.T, s.k, b.d_ab,
+            b.topk_gate, None, b.row_of_assignment, i["w_router"], s.T, s.k, b.d_gate, b.d_ab,
             b.dx_perm, b.ws, b.ws_bytes),
         "ffn_bwd_wgrad": lambda: L.moe_grouped_ffn_bwd_wgrad(
             b.d_out_perm, b.x_perm, b.h, b.d_ab, b.group_offsets, wl.mask, s.E, s.d, s.F, R,

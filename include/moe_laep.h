@@ -391,10 +391,18 @@ int moe_unpermute_combine_bwd(const uint16_t *dy, const uint16_t *out_perm,
  * forward; d_ab [rows_cap,2F] bf16 caller scratch (receives [dA|dB]);
  * outputs dx_perm [rows_cap,d] bf16, dw_gate_up [E,2F,d] bf16,
  * dw_down [E,d,F] bf16 (fp32 accumulation). ws as in moe_grouped_ffn_fwd.
- * Router term (optional, on when w_router is not NULL; topk_gate, d_gate and
- * row_of_assignment are then needed unless T == 0, and must be NULL otherwise): with
+ * Gate gradient (optional, d_gate_out [T,k] fp32 not NULL; needs topk_gate and
+ * row_of_assignment unless T == 0): the dH GEMM's epilogue recomputes
+ * H = silu(A) * B from ab_saved and sums dH * H over each grouped row; since
+ * dH = g * dy W_down, that sum is g * <dy, O>, and d_gate_out[t,j] = sum / g[t,j]
+ * (0 for a zero gate, which no selected expert has), the d_gate of
+ * moe_unpermute_combine_bwd without its read of out_perm (call that one with
+ * d_gate NULL). Sums in a fixed order: bitwise reproducible.
+ * Router term (optional, on when w_router is not NULL; topk_gate and
+ * row_of_assignment are then needed unless T == 0, and d_gate unless d_gate_out is
+ * given, whose values it then uses; d_gate is NULL whenever w_router is): with
  * topk_gate [T,k] and row_of_assignment [T,k] (moe_route, moe_permute), d_gate [T,k]
- * (moe_unpermute_combine_bwd) and w_router [d,E] fp32, the dX GEMM's epilogue adds
+ * (moe_unpermute_combine_bwd, or d_gate_out) and w_router [d,E] fp32, the dX GEMM's epilogue adds
  * the router's share of the input gradient to every grouped row before rounding:
  *   dx_perm[row(t,j), :] = dX(t,j) + dz[t,j] * w_router[:, e_j],
  *   dz[t,j] = g[t,j] * (d_gate[t,j] - sum_i g[t,i] * d_gate[t,i])
@@ -411,8 +419,9 @@ int moe_grouped_ffn_bwd(const uint16_t *d_out_perm, const uint16_t *x_perm,
                         int F, int64_t rows_cap, const uint16_t *w_gate_up,
                         const uint16_t *w_down, const float *topk_gate, const float *d_gate,
                         const int32_t *row_of_assignment, const float *w_router, int T, int k,
-                        uint16_t *d_ab, uint16_t *dx_perm, uint16_t *dw_gate_up,
-                        uint16_t *dw_down, void *ws, size_t ws_bytes, moe_stream_t stream);
+                        float *d_gate_out, uint16_t *d_ab, uint16_t *dx_perm,
+                        uint16_t *dw_gate_up, uint16_t *dw_down, void *ws, size_t ws_bytes,
+                        moe_stream_t stream);
 
 /*
  * moe_grouped_ffn_bwd_dgrad / moe_grouped_ffn_bwd_wgrad - the two halves of
@@ -430,8 +439,8 @@ int moe_grouped_ffn_bwd_dgrad(const uint16_t *d_out_perm, const uint16_t *ab_sav
                               const uint16_t *w_gate_up, const uint16_t *w_down,
                               const float *topk_gate, const float *d_gate,
                               const int32_t *row_of_assignment, const float *w_router, int T,
-                              int k, uint16_t *d_ab, uint16_t *dx_perm, void *ws, size_t ws_bytes,
-                              moe_stream_t stream);
+                              int k, float *d_gate_out, uint16_t *d_ab, uint16_t *dx_perm,
+                              void *ws, size_t ws_bytes, moe_stream_t stream);
 int moe_grouped_ffn_bwd_wgrad(const uint16_t *d_out_perm, const uint16_t *x_perm,
                               const uint16_t *h, const uint16_t *d_ab,
                               const int32_t *group_offsets, const uint8_t *active_mask, int E,

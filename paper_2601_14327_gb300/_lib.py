@@ -55,9 +55,9 @@ _SIGS = {
     "moe_unpermute_combine": (I, [P, P, P, I, I, I, P, P]),
     "moe_unpermute_combine_bwd": (I, [P, P, P, P, P, P, I, I, I, I, P, P, P]),
     "moe_grouped_ffn_bwd": (I, [P, P, P, P, P, P, I, I, I, I64, P, P, P, P, P, P, I, I, P, P, P,
-                                P, P, SZ, P]),
-    "moe_grouped_ffn_bwd_dgrad": (I, [P, P, P, I, I, I, I64, P, P, P, P, P, P, I, I, P, P, P, SZ,
-                                      P]),
+                                P, P, P, SZ, P]),
+    "moe_grouped_ffn_bwd_dgrad": (I, [P, P, P, I, I, I, I64, P, P, P, P, P, P, I, I, P, P, P, P,
+                                      SZ, P]),
     "moe_grouped_ffn_bwd_wgrad": (I, [P, P, P, P, P, P, I, I, I, I64, P, P, P, SZ, P]),
     "moe_route_bwd": (I, [P, P, P, P, I, I, I, I, P, P, P, SZ, P]),
     "moe_permute_bwd": (I, [P, P, P, P, P, I, I, I, I, P, P, SZ, P]),
@@ -247,22 +247,24 @@ def moe_unpermute_combine_bwd(dy, out_perm, row_of_assignment, topk_gate, group_
 
 def moe_grouped_ffn_bwd(d_out_perm, x_perm, ab_saved, h, group_offsets, active_mask, E, d, F,
                         rows_cap, w_gate_up, w_down, topk_gate, d_gate, row_of_assignment,
-                        w_router, T, k, d_ab, dx_perm, dw_gate_up, dw_down, ws, ws_bytes,
-                        stream=None):
+                        w_router, T, k, d_gate_out, d_ab, dx_perm, dw_gate_up, dw_down, ws,
+                        ws_bytes, stream=None):
     _check("moe_grouped_ffn_bwd", load().moe_grouped_ffn_bwd(
         _ptr(d_out_perm), _ptr(x_perm), _ptr(ab_saved), _ptr(h), _ptr(group_offsets),
         _ptr(active_mask), E, d, F, rows_cap, _ptr(w_gate_up), _ptr(w_down), _ptr(topk_gate),
-        _ptr(d_gate), _ptr(row_of_assignment), _ptr(w_router), T, k, _ptr(d_ab), _ptr(dx_perm),
-        _ptr(dw_gate_up), _ptr(dw_down), _ptr(ws), ws_bytes, _stream(stream)))
+        _ptr(d_gate), _ptr(row_of_assignment), _ptr(w_router), T, k, _ptr(d_gate_out),
+        _ptr(d_ab), _ptr(dx_perm), _ptr(dw_gate_up), _ptr(dw_down), _ptr(ws), ws_bytes,
+        _stream(stream)))
 
 
 def moe_grouped_ffn_bwd_dgrad(d_out_perm, ab_saved, group_offsets, E, d, F, rows_cap, w_gate_up,
-                              w_down, topk_gate, d_gate, row_of_assignment, w_router, T, k, d_ab,
-                              dx_perm, ws, ws_bytes, stream=None):
+                              w_down, topk_gate, d_gate, row_of_assignment, w_router, T, k,
+                              d_gate_out, d_ab, dx_perm, ws, ws_bytes, stream=None):
     _check("moe_grouped_ffn_bwd_dgrad", load().moe_grouped_ffn_bwd_dgrad(
         _ptr(d_out_perm), _ptr(ab_saved), _ptr(group_offsets), E, d, F, rows_cap,
         _ptr(w_gate_up), _ptr(w_down), _ptr(topk_gate), _ptr(d_gate), _ptr(row_of_assignment),
-        _ptr(w_router), T, k, _ptr(d_ab), _ptr(dx_perm), _ptr(ws), ws_bytes, _stream(stream)))
+        _ptr(w_router), T, k, _ptr(d_gate_out), _ptr(d_ab), _ptr(dx_perm), _ptr(ws), ws_bytes,
+        _stream(stream)))
 
 
 def moe_grouped_ffn_bwd_wgrad(d_out_perm, x_perm, h, d_ab, group_offsets, active_mask, E, d, F,

@@ -118,6 +118,8 @@ WsLayout ws_layout(int T, int d, int E, int k, int F) {
   off += align256(size_t(moe_perm_rows_max(T, k, E)) * 8);
   w.row_dz = off;
   off += align256(size_t(moe_perm_rows_max(T, k, E)) * 4);
+  w.gate_partial = off;
+  off += align256(size_t(moe_perm_rows_max(T, k, E)) * size_t(std::max(F, 0) / 64) * 4);
   w.route_partial = off;
   off += align256(route_partial_bytes(T, d, E));
   w.route_w3 = off;

@@ -39,6 +39,7 @@ struct WsLayout {
   size_t w_router_t;    // fp32  [E, d]            moe_permute_bwd transposed router
   size_t combine_rows;  // int32 + fp32 [rows_cap] moe_grouped_ffn_fwd_combine token and gate of each row
   size_t row_dz;        // fp32  [rows_cap]        moe_grouped_ffn_bwd_dgrad router logit gradient per grouped row
+  size_t gate_partial;  // fp32  [rows_cap, F/64]  moe_grouped_ffn_bwd_dgrad per-row dH * H sums (gate gradient)
   size_t route_partial; // fp32  [splits, T, NE]   moe_route split-reduction partial logits
   size_t route_w3;      // bf16  [3, NP, d]        moe_route router weight as three bf16 terms
   size_t total;

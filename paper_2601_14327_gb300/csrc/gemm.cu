@@ -97,6 +97,12 @@ struct GemmParams {
   // and w_router [d, E] fp32.
   const float *row_dz;
   const float *w_router;
+  // kDgradDown with the gate gradient (nullptr: without): for every grouped row r,
+  // gate_partial[r * gate_stride + nt * 2 + half] = sum over the tile's column half of
+  // dH[r, f] * H[r, f], H = silu(A) * B recomputed from the saved pre-activations; the
+  // row's sum over its partials is g * <dy, O> (dH = g * dy W_down).
+  float *gate_partial;
+  int gate_stride;
   // Weight-gradient modes: experts with active_mask[e] == 0 (pruned by LAEP) get no tile
   // and no store; their gradient buffers are left as they are (nullptr: all experts live).
   const uint8_t *active_mask;
@@ -209,6 +215,7 @@ __device__ __forceinline__ void epilogue_tile(const GemmParams &p, const CUtenso
     const int F = p.F;
     const int f0 = nt * BN;
     const int trow = int(row) - lane;
+    float gsum = 0.f;  // this row's sum of dH * H over the warp's columns
 #pragma unroll 1
     for (int c = half * (BN / 2); c < (half + 1) * (BN / 2); c += 32) {
       uint4 va[4], vb[4];
@@ -232,6 +239,7 @@ __device__ __forceinline__ void epilogue_tile(const GemmParams &p, const CUtenso
           const float sg = sigmoid_f(fa[i]);
           da[i] = dh * fb[i] * (sg * (1.f + fa[i] * (1.f - sg)));
           db[i] = dh * fa[i] * sg;
+          gsum = fmaf(db[i], fb[i], gsum);  // dh * silu(a) * b = dH * H
         }
         vda[v] = pack8(da);
         vdb[v] = pack8(db);
@@ -239,6 +247,7 @@ __device__ __forceinline__ void epilogue_tile(const GemmParams &p, const CUtenso
       stage_and_store(tmO, stage, lane, vda, f0 + c, trow);
       stage_and_store(tmO, stage, lane, vdb, F + f0 + c, trow);
     }
+    if (p.gate_partial != nullptr) p.gate_partial[row * p.gate_stride + nt * 2 + half] = gsum;
   } else {
     int trow;
     if (Tr::WGRAD) {
@@ -1312,6 +1321,26 @@ __global__ void router_row_dz_kernel(const float *__restrict__ topk_gate,
     }
   }
 }
+// d_gate[t, j] = <dy[t], O[row(t, j)]> from the dH GEMM's per-row partial sums of dH * H
+// (summed in a fixed order), which equal g[t, j] * <dy[t], O[row]>; divided by the gate
+// (positive for every selected expert; 0 is written for a zero gate).
+__global__ void gate_from_rows_kernel(const float *__restrict__ partial, int stride,
+                                      const float *__restrict__ topk_gate,
+                                      const int32_t *__restrict__ row_of_assignment, int64_t A,
+                                      int64_t R, float *__restrict__ d_gate) {
+  for (int64_t a = blockIdx.x * int64_t(blockDim.x) + threadIdx.x; a < A;
+       a += int64_t(gridDim.x) * blockDim.x) {
+    const int32_t r = row_of_assignment[a];
+    if (r < 0 || r >= R) {
+      dev_flag(&g_dev_err, MOE_DEV_ROWS_OVERFLOW);
+      continue;
+    }
+    float s = 0.f;
+    for (int i = 0; i < stride; ++i) s += partial[size_t(r) * stride + i];
+    const float g = topk_gate[a];
+    d_gate[a] = g > 0.f ? s / g : 0.f;
+  }
+}
 __global__ void zero_f32x4_kernel(float4 *__restrict__ p, int64_t n4) {
   for (int64_t i = blockIdx.x * int64_t(blockDim.x) + threadIdx.x; i < n4;
        i += int64_t(gridDim.x) * blockDim.x)
@@ -1494,8 +1523,8 @@ int moe_grouped_ffn_bwd_dgrad(const uint16_t *d_out_perm, const uint16_t *ab_sav
                               const uint16_t *w_gate_up, const uint16_t *w_down,
                               const float *topk_gate, const float *d_gate,
                               const int32_t *row_of_assignment, const float *w_router, int T,
-                              int k, uint16_t *d_ab, uint16_t *dx_perm, void *ws, size_t ws_bytes,
-                              moe_stream_t stream) {
+                              int k, float *d_gate_out, uint16_t *d_ab, uint16_t *dx_perm,
+                              void *ws, size_t ws_bytes, moe_stream_t stream) {
   const char *fn = "moe_grouped_ffn_bwd_dgrad";
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   if (int st = check_common(E, d, F, rows_cap, fn)) return st;
@@ -1506,39 +1535,63 @@ int moe_grouped_ffn_bwd_dgrad(const uint16_t *d_out_perm, const uint16_t *ab_sav
   int st;
   GemmParams p{};
   if ((st = use_sched_ws(p, ws, ws_bytes, fn))) return st;
-  // the router's term of the input gradient, added in the dX GEMM's epilogue
-  const bool router = w_router != nullptr;
-  if (!router && (topk_gate || d_gate || row_of_assignment))
-    return moe::set_error(MOE_ERR_ARG, "%s: router term arguments without w_router", fn);
-  if (router) {
+  // d_gate_out: the gate gradient from the dH GEMM's epilogue; w_router: the router's term
+  // of the input gradient, added in the dX GEMM's epilogue (from d_gate_out, or d_gate)
+  const bool router = w_router != nullptr, gate = d_gate_out != nullptr;
+  if (!router && d_gate)
+    return moe::set_error(MOE_ERR_ARG, "%s: d_gate without w_router", fn);
+  if (d_gate && gate)
+    return moe::set_error(MOE_ERR_ARG, "%s: d_gate is either an input or computed here", fn);
+  if (!router && !gate && (topk_gate || row_of_assignment))
+    return moe::set_error(MOE_ERR_ARG, "%s: routing arguments without a router term or d_gate_out", fn);
+  int64_t Rr = 0;
+  moe::WsLayout L{};
+  if (router || gate) {
     if (T < 0 || k < 1 || k > 8 || k > E) return moe::set_error(MOE_ERR_ARG, "%s: T=%d k=%d", fn, T, k);
-    if (T > 0 && (!topk_gate || !d_gate || !row_of_assignment))
-      return moe::set_error(MOE_ERR_ARG, "%s: the router term needs topk_gate, d_gate and "
+    if (T > 0 && (!topk_gate || !row_of_assignment || (router && !gate && !d_gate)))
+      return moe::set_error(MOE_ERR_ARG, "%s: the router term needs topk_gate, d_gate (or "
+                            "d_gate_out) and row_of_assignment; d_gate_out needs topk_gate and "
                             "row_of_assignment", fn);
-    const int64_t Rr = moe_perm_rows_max(T, k, E);
+    Rr = moe_perm_rows_max(T, k, E);
     if (rows_cap < Rr) return moe::set_error(MOE_ERR_ARG, "%s: rows_cap too small", fn);
-    const moe::WsLayout L = moe::ws_layout(T, d, E, k, F);
+    L = moe::ws_layout(T, d, E, k, F);
     if (ws_bytes < L.total) return moe::set_error(MOE_ERR_WORKSPACE, "%s: workspace", fn);
+  }
+  p.group_offsets = group_offsets;
+  p.E = E; p.d = d; p.F = F;
+  // dH = dO W_down, fused SwiGLU backward -> [dA | dB] (and the rows' dH * H sums)
+  p.nkb = d / BK;
+  p.out = d_ab;
+  p.aux = ab_saved;
+  if (gate) {
+    p.gate_partial = reinterpret_cast<float *>(static_cast<char *>(ws) + L.gate_partial);
+    p.gate_stride = 2 * (F / (F % 256 == 0 ? 256 : 128));  // column halves of the N tiles
+  }
+  if ((st = run_gemm<kDgradDown>(F, d_out_perm, R, d, w_down, uint64_t(E) * d, F, R, 2 * F, p,
+                                 s, "moe_grouped_ffn_bwd: dH GEMM")))
+    return st;
+  p.gate_partial = nullptr;
+  const int64_t A = int64_t(T) * k;
+  if (gate && A > 0) {
+    MOE_LAUNCH("gate_from_rows", s, gate_from_rows_kernel<<<grid_for(A), 256, 0, s>>>(
+                                        reinterpret_cast<const float *>(static_cast<char *>(ws) + L.gate_partial),
+                                        2 * (F / (F % 256 == 0 ? 256 : 128)), topk_gate,
+                                        row_of_assignment, A, Rr, d_gate_out));
+    if ((st = moe::launch_status("moe_grouped_ffn_bwd_dgrad: gate gradient"))) return st;
+  }
+  if (router) {
     float *row_dz = reinterpret_cast<float *>(static_cast<char *>(ws) + L.row_dz);
     cudaError_t e = cudaMemsetAsync(row_dz, 0, size_t(Rr) * 4, s);
     if (e != cudaSuccess) return moe::cuda_status(e, "moe_grouped_ffn_bwd_dgrad: zero row_dz");
     if (T > 0) {
       MOE_LAUNCH("router_row_dz", s, router_row_dz_kernel<<<grid_for(T), 256, 0, s>>>(
-                                         topk_gate, d_gate, row_of_assignment, T, k, Rr, row_dz));
+                                         topk_gate, gate ? d_gate_out : d_gate, row_of_assignment,
+                                         T, k, Rr, row_dz));
       if ((st = moe::launch_status("moe_grouped_ffn_bwd_dgrad: router rows"))) return st;
     }
     p.row_dz = row_dz;
     p.w_router = w_router;
   }
-  p.group_offsets = group_offsets;
-  p.E = E; p.d = d; p.F = F;
-  // dH = dO W_down, fused SwiGLU backward -> [dA | dB]
-  p.nkb = d / BK;
-  p.out = d_ab;
-  p.aux = ab_saved;
-  if ((st = run_gemm<kDgradDown>(F, d_out_perm, R, d, w_down, uint64_t(E) * d, F, R, 2 * F, p,
-                                 s, "moe_grouped_ffn_bwd: dH GEMM")))
-    return st;
   // dX = [dA | dB] W_gate_up
   p.nkb = 2 * F / BK;
   p.out = dx_perm;
@@ -1621,11 +1674,13 @@ int moe_grouped_ffn_bwd(const uint16_t *d_out_perm, const uint16_t *x_perm,
                         const uint16_t *w_gate_up, const uint16_t *w_down,
                         const float *topk_gate, const float *d_gate,
                         const int32_t *row_of_assignment, const float *w_router, int T, int k,
-                        uint16_t *d_ab, uint16_t *dx_perm, uint16_t *dw_gate_up,
-                        uint16_t *dw_down, void *ws, size_t ws_bytes, moe_stream_t stream) {
+                        float *d_gate_out, uint16_t *d_ab, uint16_t *dx_perm,
+                        uint16_t *dw_gate_up, uint16_t *dw_down, void *ws, size_t ws_bytes,
+                        moe_stream_t stream) {
   if (int st = moe_grouped_ffn_bwd_dgrad(d_out_perm, ab_saved, group_offsets, E, d, F, rows_cap,
                                          w_gate_up, w_down, topk_gate, d_gate, row_of_assignment,
-                                         w_router, T, k, d_ab, dx_perm, ws, ws_bytes, stream))
+                                         w_router, T, k, d_gate_out, d_ab, dx_perm, ws, ws_bytes,
+                                         stream))
     return st;
   return moe_grouped_ffn_bwd_wgrad(d_out_perm, x_perm, h, d_ab, group_offsets, active_mask, E, d,
                                    F, rows_cap, dw_gate_up, dw_down, ws, ws_bytes, stream);

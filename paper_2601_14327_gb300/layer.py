@@ -129,15 +129,16 @@ def forward(b: MoELayerBuffers, x, w_router, bias, w_gate_up, w_down, active_mas
 
 def backward(b: MoELayerBuffers, dy, w_router, w_gate_up, w_down, stream=None,
              overlap: bool = False, active_mask=None):
-    """combine bwd -> grouped FFN bwd (dgrad, then wgrad) -> router bwd -> permute bwd.
+    """combine bwd -> grouped FFN dgrad (with the gate gradient and the router's term of dx)
+    -> router bwd -> permute bwd -> grouped FFN wgrad.
 
     active_mask: the LAEP mask the forward routed with (None: all experts live). Pruned
     experts' weight gradients are not written (their buffers keep what they held); live
     experts without tokens get exact zeros.
 
-    With overlap, the router backward (after the combine backward) and the
-    unpermute-sum (after the dX GEMM) run on a second stream while the main stream
-    computes the weight gradients; the main stream waits for them at the end. The
+    With overlap, the router backward and the unpermute-sum (after the dgrad GEMMs) run on
+    a second stream while the main stream computes the weight gradients; the main stream
+    waits for them at the end. The
     default is one stream: on GB300 at T=65536, d_model=7168 the step is power-capped,
     and running those memory-bound kernels beside the GEMMs slowed the GEMMs by more
     than it hid (96.1-96.7 against 97.0-97.3 ms per step).
@@ -146,23 +147,23 @@ def backward(b: MoELayerBuffers, dy, w_router, w_gate_up, w_down, stream=None,
     R = s.rows_cap
     main = torch.cuda.current_stream() if stream is None else stream
     side = b.side if overlap else main
-    L.moe_unpermute_combine_bwd(dy, b.out_perm, b.row_of_assignment, b.topk_gate,
+    # d_out_perm = g * dy; the gate gradient comes from the dH GEMM (below), so the combine
+    # backward does not read out_perm
+    L.moe_unpermute_combine_bwd(dy, None, b.row_of_assignment, b.topk_gate,
                                 b.group_offsets, b.group_counts, s.T, s.d, s.E, s.k,
-                                b.d_out_perm, b.d_gate, main)
+                                b.d_out_perm, None, main)
+    # dH (+ the gate gradient into b.d_gate), dX with the router's term of dx added to the
+    # grouped rows in its epilogue
+    L.moe_grouped_ffn_bwd_dgrad(b.d_out_perm, b.ab, b.group_offsets, s.E, s.d, s.F, R,
+                                w_gate_up, w_down, b.topk_gate, None, b.row_of_assignment,
+                                w_router, s.T, s.k, b.d_gate, b.d_ab, b.dx_perm, b.ws,
+                                b.ws_bytes, main)
     if overlap:
         ev = torch.cuda.Event()
         ev.record(main)
         side.wait_event(ev)
     L.moe_route_bwd(b.x, b.topk_idx, b.topk_gate, b.d_gate, s.T, s.d, s.E, s.k, b.d_logits,
                     b.dw_router, b.ws, b.ws_bytes, side)
-    # the router's term of dx is added to the grouped rows in the dX GEMM's epilogue
-    L.moe_grouped_ffn_bwd_dgrad(b.d_out_perm, b.ab, b.group_offsets, s.E, s.d, s.F, R,
-                                w_gate_up, w_down, b.topk_gate, b.d_gate, b.row_of_assignment,
-                                w_router, s.T, s.k, b.d_ab, b.dx_perm, b.ws, b.ws_bytes, main)
-    if overlap:
-        ev = torch.cuda.Event()
-        ev.record(main)
-        side.wait_event(ev)
     L.moe_permute_bwd(b.dx_perm, b.row_of_assignment, b.topk_idx, None, None, s.T, s.d, s.E,
                       s.k, b.dx, b.ws, b.ws_bytes, side)
     if b.gather:

@@ -94,7 +94,7 @@ def test_argument_validation_without_launch(lib):
         assert e.value.status == -6
         with pytest.raises(L.MoEError) as e:
             L.moe_grouped_ffn_bwd_dgrad(16, 16, 16, 8, 256, 256, 4096, 16, 16, None, None, None,
-                                        None, 0, 1, 16, 16, ws, ws_bytes, stream=0)
+                                        None, 0, 1, None, 16, 16, ws, ws_bytes, stream=0)
         assert e.value.status == -6
         with pytest.raises(L.MoEError) as e:
             L.moe_grouped_ffn_bwd_wgrad(16, 16, 16, 16, 16, None, 8, 256, 256, 4096, 16, 16, ws,
@@ -207,15 +207,23 @@ def test_new_entry_points_validate_before_launch(lib):
     assert e.value.status == -1
     with pytest.raises(L.MoEError) as e:  # router term: with tokens, every per-token input
         L.moe_grouped_ffn_bwd_dgrad(16, 16, 16, 8, 256, 256, 4096, 16, 16, 16, None, 16, 16, 10,
-                                    2, 16, 16, 16, 1 << 20, stream=0)
+                                    2, None, 16, 16, 16, 1 << 20, stream=0)
     assert e.value.status == -1
-    with pytest.raises(L.MoEError) as e:  # router term inputs without w_router
+    with pytest.raises(L.MoEError) as e:  # d_gate input without w_router
         L.moe_grouped_ffn_bwd_dgrad(16, 16, 16, 8, 256, 256, 4096, 16, 16, 16, 16, 16, None, 10,
-                                    2, 16, 16, 16, 1 << 20, stream=0)
+                                    2, None, 16, 16, 16, 1 << 20, stream=0)
+    assert e.value.status == -1
+    with pytest.raises(L.MoEError) as e:  # d_gate both given and asked for
+        L.moe_grouped_ffn_bwd_dgrad(16, 16, 16, 8, 256, 256, 4096, 16, 16, 16, 16, 16, 16, 10,
+                                    2, 16, 16, 16, 16, 1 << 20, stream=0)
+    assert e.value.status == -1
+    with pytest.raises(L.MoEError) as e:  # gate gradient without row_of_assignment
+        L.moe_grouped_ffn_bwd_dgrad(16, 16, 16, 8, 256, 256, 4096, 16, 16, 16, None, None, None,
+                                    10, 2, 16, 16, 16, 16, 1 << 20, stream=0)
     assert e.value.status == -1
     with pytest.raises(L.MoEError) as e:  # router term: workspace for the per-row dz
         L.moe_grouped_ffn_bwd_dgrad(16, 16, 16, 8, 256, 256, 4096, 16, 16, 16, 16, 16, 16, 10,
-                                    2, 16, 16, 16, 256, stream=0)
+                                    2, None, 16, 16, 16, 256, stream=0)
     assert e.value.status == -6
     for bad in (0, 999_999, 2_000_000_001):
         with pytest.raises(L.MoEError) as e:

@@ -465,8 +465,8 @@ def test_router_term_in_dx_epilogue_equals_unpermute_sum_form(T, d, E, k, F):
     R = b.shape.rows_cap
     g = {n: v.cuda() for n, v in inp.items()}
     L.moe_grouped_ffn_bwd_dgrad(b.d_out_perm, b.ab, b.group_offsets, E, d, F, R, g["w_gate_up"],
-                                g["w_down"], None, None, None, None, T, k, b.d_ab, b.dx_perm,
-                                b.ws, b.ws_bytes)
+                                g["w_down"], None, None, None, None, T, k, None, b.d_ab,
+                                b.dx_perm, b.ws, b.ws_bytes)
     flat = b.row_of_assignment.cpu().numpy().reshape(-1)
     assert_close("dX without the router term", to_np(b.dx_perm)[flat], ref["dX"].reshape(T * k, -1))
     dx2 = torch.empty_like(b.dx)
@@ -485,6 +485,35 @@ def test_router_term_in_dx_epilogue_equals_unpermute_sum_form(T, d, E, k, F):
     scale = (np.abs(rows).sum(axis=1) + np.abs(ref["dX"]).sum(axis=1)
              + 2 * np.abs(ref["dx"]))
     assert (np.abs(fused_dx - unfused_dx) <= 2.0 ** -8 * scale + 1e-30).all()
+
+
+@pytest.mark.parametrize("T,d,E,k,F", [(1500, 384, 12, 4, 640), (3000, 256, 256, 8, 256),
+                                       (700, 512, 8, 8, 256)])
+def test_gate_gradient_from_dh_epilogue(T, d, E, k, F):
+    """d_gate from the dH GEMM's epilogue (the layer's default: sum over each grouped row of
+    dH * H, H recomputed from the saved pre-activations, divided by the gate) against the
+    oracle's <dy, o> and against moe_unpermute_combine_bwd's dot product with the stored O.
+    Both carry the bf16 roundings of their inputs (O, or g*dy and W_down); they must agree
+    within those, and the layer's routing gradient with them."""
+    inp = case_inputs(T, d, E, k, F, seed=T + 3)
+    o = oracle_inputs(inp)
+    z = O.router_logits(o["x"], o["w_router"], o["bias"])
+    ref = O.moe_layer(o["x"], o["w_router"], o["bias"], None, k, o["w_gate_up"], o["w_down"],
+                      dy=o["dy"], logits32=z)
+    b = run_gpu_layer(inp, E, k, logits_in=z)
+    fused = b.d_gate.cpu().numpy().astype(np.float64)
+    assert_close("d_gate (dH epilogue)", fused, ref["d_gate"])
+    dg2 = torch.empty_like(b.d_gate)
+    L.moe_unpermute_combine_bwd(inp["dy"].cuda(), b.out_perm, b.row_of_assignment, b.topk_gate,
+                                b.group_offsets, b.group_counts, T, d, E, k, None, dg2)
+    torch.cuda.synchronize()
+    assert L.moe_device_error(clear=True) == 0
+    direct = dg2.cpu().numpy().astype(np.float64)
+    assert_close("d_gate (combine backward)", direct, ref["d_gate"])
+    # |difference| within a few bf16 roundings of the terms of the dot product
+    scale = np.einsum("td,tjd->tj", np.abs(o["dy"]), np.abs(ref["o"]))
+    assert (np.abs(fused - direct) <= 2.0 ** -6 * scale + 1e-30).all()
+    assert_close("d_logits", b.d_logits.cpu().numpy(), ref["d_logits"])
 
 
 def test_dynamic_schedule_equals_fixed_stride(tmp_path):

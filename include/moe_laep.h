@@ -395,7 +395,8 @@ int moe_unpermute_combine_bwd(const uint16_t *dy, const uint16_t *out_perm,
  * row_of_assignment unless T == 0): the dH GEMM's epilogue recomputes
  * H = silu(A) * B from ab_saved and sums dH * H over each grouped row; since
  * dH = g * dy W_down, that sum is g * <dy, O>, and d_gate_out[t,j] = sum / g[t,j]
- * (0 for a zero gate, which no selected expert has), the d_gate of
+ * (0 where the gate is 0, an fp32 softmax that underflowed: the routing backward
+ * multiplies d_gate by its gate, so no gradient changes), the d_gate of
  * moe_unpermute_combine_bwd without its read of out_perm (call that one with
  * d_gate NULL). Sums in a fixed order: bitwise reproducible.
  * Router term (optional, on when w_router is not NULL; topk_gate and

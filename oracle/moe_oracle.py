@@ -25,6 +25,8 @@ its reason in the design notes):
   R8  count mode: prune the P smallest counts (Eq. 2's largest=False top-K).
   R9  at least k experts are always kept (the paper does not say; routing
       needs k live experts).
+  R10 bias fixed, not trained (no bias gradient); masked experts get a zero
+      router gradient.
   R11 Algorithm 1 over ITER iterations: the running load sum restarts for every
       (iteration, layer); Marker counts how often each expert (by id, not by
       sorted position) is flagged; the number pruned per layer is the mean
@@ -37,6 +39,11 @@ its reason in the design notes):
       in argmin to the lower group; when the expert count is not a multiple of
       the group count the per-group capacity is rounded up (the listing would
       otherwise never place the remainder).
+  R14 an expert without assignments gets a zero weight gradient here; this
+      stands for a live expert (the kernels leave a pruned expert's dW alone).
+  R15 d_gate is <dy, o> for every slot; the kernels report 0 where the fp32
+      gate underflowed to 0, which no gradient downstream can see (the routing
+      backward multiplies d_gate by its gate).
 """
 from __future__ import annotations
 

@@ -763,12 +763,16 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t tmem_base = static_cast<uint32_t>(misc[0]);
   const int total = s_prefix[E];
 
+  // Every role of a pair sees the pair's tiles in increasing order (a fixed stride, or
+  // claims from a counter that only grows), so the expert of the next tile is found by
+  // walking forward from the previous one: a step or two of shared-memory reads per
+  // tile instead of a binary search over all experts (measured ~1,100 cycles per tile,
+  // which one-k-block tiles of light experts could not hide).
+  int cursor = 0;
   auto decode = [&](int tile) {
-    int lo = 0, hi = E - 1;
-    while (lo < hi) {
-      const int mid = (lo + hi + 1) >> 1;
-      if (s_prefix[mid] <= tile) lo = mid; else hi = mid - 1;
-    }
+    int lo = s_prefix[cursor] <= tile ? cursor : 0;
+    while (lo + 1 < E && s_prefix[lo + 1] <= tile) ++lo;
+    cursor = lo;
     PairTile t;
     const int local = tile - s_prefix[lo];
     t.e = s_order[lo];
@@ -922,31 +926,31 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (leader) tc::mbar_arrive_expect_tx(full_bar(s), 2 * Sh::STAGE_BYTES);
           const uint32_t a_dst = sA0 + s * Sh::A_BYTES, b_dst = sB0 + s * Sh::B_BYTES;
           const uint32_t fb = full_leader + 8u * s;
+          const int k0 = kb * KB;
+          // K-major operands: one box per 64-deep K half (the 128-byte swizzle row), half h
+          // at h * rows * 128 bytes. MN-major operands: one box of 64 columns x KB k-rows per
+          // 64 columns, column block i at i * KB * 128 bytes (half as many loads).
+          if (Tr::A_MN) {  // weight gradients: [dA|dB] or dO of the group, K = group rows
 #pragma unroll
-          for (int h = 0; h < KB / 64; ++h) {  // the stage's 64-deep K halves
-            const int k0 = kb * KB + h * 64;
-            const uint32_t ad = a_dst + uint32_t(h) * (BM * 128), bd = b_dst + uint32_t(h) * (BNH * 128);
-            if (MODE == kGateUp) {  // even CTA: gate rows, odd CTA: up rows
-              tc::tma_load_2d_pair(ad, &tmA, fb, k0, t.goff + mt * BM);
-              tc::tma_load_2d_pair(bd, &tmB, fb, k0, t.e * 2 * p.F + int(rank) * p.F + t.nt * 128);
-            } else if (MODE == kDown) {
-              tc::tma_load_2d_pair(ad, &tmA, fb, k0, t.goff + mt * BM);
-              tc::tma_load_2d_pair(bd, &tmB, fb, k0, t.e * p.d + t.nt * BN + int(rank) * BNH);
-            } else if (MODE == kDgradDown || MODE == kDgradGateUp) {
-              tc::tma_load_2d_pair(ad, &tmA, fb, k0, t.goff + mt * BM);
-              const int krow = (MODE == kDgradDown ? t.e * p.d : t.e * 2 * p.F) + k0;
+            for (int i = 0; i < BM / 64; ++i)
+              tc::tma_load_2d_pair(a_dst + i * (KB * 128), &tmA, fb, mt * BM + i * 64, t.goff + k0);
+          } else {
 #pragma unroll
-              for (int i = 0; i < BNH / 64; ++i)
-                tc::tma_load_2d_pair(bd + i * 64 * 128, &tmB, fb, t.nt * BN + int(rank) * BNH + i * 64, krow);
-            } else {  // weight gradients: both operands MN-major, K = group rows
-              const int krow = t.goff + k0;
+            for (int h = 0; h < KB / 64; ++h)
+              tc::tma_load_2d_pair(a_dst + h * (BM * 128), &tmA, fb, k0 + h * 64, t.goff + mt * BM);
+          }
+          if (Tr::B_MN) {
+            const int krow = (MODE == kDgradDown ? t.e * p.d : MODE == kDgradGateUp ? t.e * 2 * p.F : t.goff) + k0;
 #pragma unroll
-              for (int i = 0; i < BM / 64; ++i)
-                tc::tma_load_2d_pair(ad + i * 64 * 128, &tmA, fb, mt * BM + i * 64, krow);
+            for (int i = 0; i < BNH / 64; ++i)
+              tc::tma_load_2d_pair(b_dst + i * (KB * 128), &tmB, fb, t.nt * BN + int(rank) * BNH + i * 64, krow);
+          } else {
+            // kGateUp: even CTA gate rows, odd CTA up rows; kDown: rows of W_down
+            const int brow = MODE == kGateUp ? t.e * 2 * p.F + int(rank) * p.F + t.nt * 128
+                                             : t.e * p.d + t.nt * BN + int(rank) * BNH;
 #pragma unroll
-              for (int i = 0; i < BNH / 64; ++i)
-                tc::tma_load_2d_pair(bd + i * 64 * 128, &tmB, fb, t.nt * BN + int(rank) * BNH + i * 64, krow);
-            }
+            for (int h = 0; h < KB / 64; ++h)
+              tc::tma_load_2d_pair(b_dst + h * (BNH * 128), &tmB, fb, k0 + h * 64, brow);
           }
         }
       }
@@ -998,12 +1002,14 @@ __global__ void __launch_bounds__(kThreads, 1)
           const uint32_t a_s = sA0 + s * Sh::A_BYTES, b_s = sB0 + s * Sh::B_BYTES;
 #pragma unroll
           for (int kk = 0; kk < KB / UMMA_K; ++kk) {
-            // K-half kk / 4 of the stage, 16-wide step kk % 4 inside it
+            // K-major: K-half kk / 4 of the stage, 16-wide step kk % 4 inside it (32 bytes
+            // along the swizzled row). MN-major: k-rows 16 kk .. 16 kk + 15 of every
+            // 64-column block (2 KB each), blocks KB * 128 bytes apart.
             const uint32_t ha = uint32_t(kk >> 2) * (BM * 128), hb = uint32_t(kk >> 2) * (BNH * 128);
             const int q = kk & 3;
-            const uint64_t ad = Tr::A_MN ? tc::smem_desc_sw128(a_s + ha + q * 2048, 8192, 1024)
+            const uint64_t ad = Tr::A_MN ? tc::smem_desc_sw128(a_s + kk * 2048, KB * 128, 1024)
                                          : tc::smem_desc_sw128(a_s + ha + q * 32, 16, 1024);
-            const uint64_t bd = Tr::B_MN ? tc::smem_desc_sw128(b_s + hb + q * 2048, 8192, 1024)
+            const uint64_t bd = Tr::B_MN ? tc::smem_desc_sw128(b_s + kk * 2048, KB * 128, 1024)
                                          : tc::smem_desc_sw128(b_s + hb + q * 32, 16, 1024);
             tc::mma_bf16_pair(d_tmem, ad, bd, IDESC, (kb | kk) != 0);
           }
@@ -1219,13 +1225,16 @@ int run_gemm_out(int N, const void *a_base, uint64_t a_rows, uint64_t a_cols, co
   const bool gather_a = gather && MODE == kGateUp, gather_b = gather && MODE == kWgradGateUp;
   CUtensorMap ma, mb;
   int st;
+  // MN-major boxes: 64 columns x one ring stage of k-rows (128 in the CTA-pair kernel
+  // without gathers, BK = 64 in the others)
+  const uint32_t mn_rows = pair && !gather ? 128u : uint32_t(BK);
   if ((st = gather_a  ? make_map(&ma, a_base, a_rows, a_cols, BK, 1, what)
-            : Tr::A_MN ? make_map(&ma, a_base, a_rows, a_cols, 64, BK, what)
+            : Tr::A_MN ? make_map(&ma, a_base, a_rows, a_cols, 64, mn_rows, what)
                        : make_map(&ma, a_base, a_rows, a_cols, BK, BM, what)))
     return st;
   const uint32_t b_box_rows = pair ? uint32_t(BN / 2) : 128u;
   if ((st = gather_b  ? make_map(&mb, b_base, b_rows, b_cols, 64, 1, what)
-            : Tr::B_MN ? make_map(&mb, b_base, b_rows, b_cols, 64, BK, what)
+            : Tr::B_MN ? make_map(&mb, b_base, b_rows, b_cols, 64, mn_rows, what)
                        : make_map(&mb, b_base, b_rows, b_cols, BK, b_box_rows, what)))
     return st;
   CUtensorMap mo;  // the epilogue's output, in 32 x 32 chunks

@@ -628,6 +628,21 @@ struct PairTile {
   int e, goff, mp, nt, nkb, mtiles;
 };
 
+// A claim unit: tiles lt0 .. lt0 + cnt - 1 (in the expert's tile order) of expert e.
+struct PairUnit {
+  int e, goff, nkb, mtiles, lt0, cnt;
+};
+
+// Tiles of one claim unit of the dynamic weight-gradient schedule, from the expert's
+// k-blocks per tile: light experts' tiles (one to seven 128-row k-blocks) are claimed,
+// published to the pair and handed to the epilogue warps several at a time, about eight
+// k-blocks of work per claim. Each hand-off costs the single producer and MMA-issuer
+// threads ~2,000 cycles (a cluster-scope release and arrive), which one tile of one
+// k-block (~1,000 cycles of MMA) could not hide.
+__host__ __device__ constexpr int unit_tiles(int nkb) {
+  return nkb >= 8 ? 1 : nkb >= 4 ? 2 : nkb >= 2 ? 4 : 8;
+}
+
 __device__ __forceinline__ int4 ld_rows4(const int32_t *p) {
   return __ldg(reinterpret_cast<const int4 *>(p));
 }
@@ -739,7 +754,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     s_order[r] = e;
   }
   __syncthreads();
+  const bool dyn = Tr::WGRAD && p.dynamic;
   if (threadIdx.x == 0) {
+    // s_prefix counts claim units: tiles, or groups of light experts' tiles (dyn)
     int acc = 0, n_empty = 0, n_pruned = 0;
     for (int i = 0; i < E; ++i) {
       s_prefix[i] = acc;
@@ -750,7 +767,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         continue;
       }
       const int mt = Tr::WGRAD ? p.m_tiles_w : key / BM;
-      acc += ((mt + 1) / 2) * p.n_tiles;
+      const int tiles = ((mt + 1) / 2) * p.n_tiles;
+      const int g = dyn ? unit_tiles(key / KB) : 1;
+      acc += (tiles + g - 1) / g;
     }
     s_prefix[E] = acc;
     misc[2] = n_empty;
@@ -769,14 +788,29 @@ __global__ void __launch_bounds__(kThreads, 1)
   // tile instead of a binary search over all experts (measured ~1,100 cycles per tile,
   // which one-k-block tiles of light experts could not hide).
   int cursor = 0;
-  auto decode = [&](int tile) {
-    int lo = s_prefix[cursor] <= tile ? cursor : 0;
-    while (lo + 1 < E && s_prefix[lo + 1] <= tile) ++lo;
+  auto decode_unit = [&](int unit) {
+    int lo = s_prefix[cursor] <= unit ? cursor : 0;
+    while (lo + 1 < E && s_prefix[lo + 1] <= unit) ++lo;
     cursor = lo;
+    PairUnit u;
+    u.e = s_order[lo];
+    u.goff = s_goff[u.e];
+    const int rows = s_goff[u.e + 1] - u.goff;
+    u.nkb = Tr::WGRAD ? rows / KB : p.nkb / (KB / BK);
+    u.mtiles = Tr::WGRAD ? p.m_tiles_w : rows / BM;
+    const int g = dyn ? unit_tiles(u.nkb) : 1;
+    u.lt0 = (unit - s_prefix[lo]) * g;
+    u.cnt = min(g, ((u.mtiles + 1) / 2) * p.n_tiles - u.lt0);
+    return u;
+  };
+  // Tile j of a unit: the expert's tile lt0 + j as (row pair, column tile).
+  auto tile_in = [&](const PairUnit &u, int j) {
     PairTile t;
-    const int local = tile - s_prefix[lo];
-    t.e = s_order[lo];
-    t.goff = s_goff[t.e];
+    const int local = u.lt0 + j;
+    t.e = u.e;
+    t.goff = u.goff;
+    t.nkb = u.nkb;
+    t.mtiles = u.mtiles;
     if (Tr::WGRAD && p.n_tiles > kWgradBlock) {
       // Weight gradients with many column tiles: an expert's (row pair, column) tiles in
       // blocks of kWgradBlock row pairs, column by column inside a block, so that the
@@ -798,33 +832,30 @@ __global__ void __launch_bounds__(kThreads, 1)
       t.mp = local / p.n_tiles;
       t.nt = local - t.mp * p.n_tiles;
     }
-    const int rows = s_goff[t.e + 1] - t.goff;
-    t.nkb = Tr::WGRAD ? rows / KB : p.nkb / (KB / BK);
-    t.mtiles = Tr::WGRAD ? p.m_tiles_w : rows / BM;
     return t;
   };
 
-  // ---- tile numbers. The weight gradients' tiles differ in cost (K = the expert's rows):
-  // there the even CTA's producer takes tile number n of this pair, the pair's index for
-  // n = 0, then the next unclaimed tile of the list (an atomic counter shared by all
-  // pairs), -1 once the list is exhausted. It writes the tile into slot n % kRing of both
-  // CTAs' rings and arrives on the slots' barriers before it issues the tile's loads; the
-  // odd CTA's producer and the MMA issuer wait there, and the MMA issuer passes each tile
-  // on to both CTAs' epilogue warps through s_epi[buffer] and epi_bar[buffer] once that
-  // accumulator buffer is free. The activation GEMMs' tiles all cost the same (and with
-  // p.dynamic == 0 the weight gradients' too): every role of a pair then computes its tile
-  // numbers itself, cluster, cluster + nclusters, ..., with no hand-off.
-  const bool dyn = Tr::WGRAD && p.dynamic;
-  auto static_tile = [&](uint32_t n) -> int {
-    const int tile = cluster + int(n) * nclusters;
-    return tile < total ? tile : -1;
+  // ---- claim units. The weight gradients' tiles differ in cost (K = the expert's rows):
+  // there the even CTA's producer takes unit number n of this pair, the pair's index for
+  // n = 0, then the next unclaimed unit of the list (an atomic counter shared by all
+  // pairs), -1 once the list is exhausted. It writes the unit into slot n % kRing of both
+  // CTAs' rings and arrives on the slots' barriers before it issues the unit's loads; the
+  // odd CTA's producer and the MMA issuer wait there, and the MMA issuer passes each unit
+  // on to both CTAs' epilogue warps through s_epi[n % 2] and epi_bar[n % 2] once the
+  // accumulator buffer of the unit's first tile is free. The activation GEMMs' tiles all
+  // cost the same (and with p.dynamic == 0 the weight gradients' too): a unit is one tile,
+  // and every role of a pair computes its unit numbers itself, cluster, cluster +
+  // nclusters, ..., with no hand-off.
+  auto static_unit = [&](uint32_t n) -> int {
+    const int unit = cluster + int(n) * nclusters;
+    return unit < total ? unit : -1;
   };
   const uint32_t ring_peer = tc::mapa(tc::smem_u32(const_cast<int *>(s_ring)), 1);
   const uint32_t ring_bar_peer = tc::mapa(ring_bar(0), 1);
-  int claimed = cluster;  // even CTA's producer: the tile it publishes next
-  // Returns this pair's tile number n (-1: no more), or -2 after a failed wait.
-  auto next_tile = [&](uint32_t n) -> int {
-    if (!dyn) return static_tile(n);
+  int claimed = cluster;  // even CTA's producer: the unit it publishes next
+  // Returns this pair's unit number n (-1: no more), or -2 after a failed wait.
+  auto next_unit = [&](uint32_t n) -> int {
+    if (!dyn) return static_unit(n);
     const int slot = int(n % kRing);
     if (leader) {
       const int v = claimed < total ? claimed : -1;
@@ -849,53 +880,56 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint32_t it = 0;
     bool ok = true;
     for (uint32_t n = 0; ok; ++n) {
-      int tile = 0;
-      if (lane == 0) tile = next_tile(n);
-      tile = __shfl_sync(0xffffffffu, tile, 0);
-      if (tile < 0) break;
-      const PairTile t = decode(tile);
-      const int mt = 2 * t.mp + int(rank);
-      int4 rows4 = make_int4(0, 0, 0, 0), nxt = make_int4(0, 0, 0, 0);
-      // kGateUp: this lane's 4 rows of the tile (token 0 for the row block past an
-      // odd group end, which is computed but not stored)
-      if (MODE == kGateUp && mt < t.mtiles) rows4 = ld_rows4(p.token_of_row + t.goff + mt * BM + 4 * lane);
-      if (MODE == kWgradGateUp && t.nkb > 0) nxt = ld_rows4(p.token_of_row + t.goff + 4 * grp);
-      for (int kb = 0; kb < t.nkb; ++kb, ++it) {
-        const int s = it % STAGES;
-        const uint32_t ph = (it / STAGES) & 1u;
-        if (MODE == kWgradGateUp) {
-          rows4 = nxt;
-          if (kb + 1 < t.nkb) nxt = ld_rows4(p.token_of_row + t.goff + (kb + 1) * BK + 4 * grp);
-        }
-        int w_ok = 1;
-        if (lane == 0) w_ok = tc::mbar_wait(empty_bar(s), ph ^ 1u, kWaitLimitNs, abort_flag) ? 1 : 0;
-        w_ok = __shfl_sync(0xffffffffu, w_ok, 0);
-        if (!w_ok) {
-          if (lane == 0) fail(abort_flag);
-          ok = false;
-          break;
-        }
-        const uint32_t a_dst = sA0 + s * Sh::A_BYTES, b_dst = sB0 + s * Sh::B_BYTES;
-        const uint32_t fb = full_leader + 8u * s;
-        const int k0 = kb * BK;
-        if (lane == 0) {
-          if (leader) tc::mbar_arrive_expect_tx(full_bar(s), 2 * Sh::STAGE_BYTES);
-          if (MODE == kGateUp) {  // even CTA: gate rows, odd CTA: up rows
-            tc::tma_load_2d_pair(b_dst, &tmB, fb, k0, t.e * 2 * p.F + int(rank) * p.F + t.nt * 128);
-          } else {  // A = [dA | dB] of the group, MN-major
-            const int krow = t.goff + k0;
-#pragma unroll
-            for (int i = 0; i < BM / 64; ++i)
-              tc::tma_load_2d_pair(a_dst + i * 64 * 128, &tmA, fb, mt * BM + i * 64, krow);
+      int unit = 0;
+      if (lane == 0) unit = next_unit(n);
+      unit = __shfl_sync(0xffffffffu, unit, 0);
+      if (unit < 0) break;
+      const PairUnit u = decode_unit(unit);
+      for (int j = 0; j < u.cnt && ok; ++j) {
+        const PairTile t = tile_in(u, j);
+        const int mt = 2 * t.mp + int(rank);
+        int4 rows4 = make_int4(0, 0, 0, 0), nxt = make_int4(0, 0, 0, 0);
+        // kGateUp: this lane's 4 rows of the tile (token 0 for the row block past an
+        // odd group end, which is computed but not stored)
+        if (MODE == kGateUp && mt < t.mtiles) rows4 = ld_rows4(p.token_of_row + t.goff + mt * BM + 4 * lane);
+        if (MODE == kWgradGateUp && t.nkb > 0) nxt = ld_rows4(p.token_of_row + t.goff + 4 * grp);
+        for (int kb = 0; kb < t.nkb; ++kb, ++it) {
+          const int s = it % STAGES;
+          const uint32_t ph = (it / STAGES) & 1u;
+          if (MODE == kWgradGateUp) {
+            rows4 = nxt;
+            if (kb + 1 < t.nkb) nxt = ld_rows4(p.token_of_row + t.goff + (kb + 1) * BK + 4 * grp);
           }
-        }
-        if (MODE == kGateUp) {
-          tc::tma_gather4_pair(a_dst + uint32_t(lane) * 512u, &tmA, fb, k0, rows4.x, rows4.y,
-                               rows4.z, rows4.w);
-        } else if (box < BNH / 64) {
-          tc::tma_gather4_pair(b_dst + uint32_t(box) * 64u * 128u + uint32_t(grp) * 512u, &tmB, fb,
-                               t.nt * BN + int(rank) * BNH + box * 64, rows4.x, rows4.y, rows4.z,
-                               rows4.w);
+          int w_ok = 1;
+          if (lane == 0) w_ok = tc::mbar_wait(empty_bar(s), ph ^ 1u, kWaitLimitNs, abort_flag) ? 1 : 0;
+          w_ok = __shfl_sync(0xffffffffu, w_ok, 0);
+          if (!w_ok) {
+            if (lane == 0) fail(abort_flag);
+            ok = false;
+            break;
+          }
+          const uint32_t a_dst = sA0 + s * Sh::A_BYTES, b_dst = sB0 + s * Sh::B_BYTES;
+          const uint32_t fb = full_leader + 8u * s;
+          const int k0 = kb * BK;
+          if (lane == 0) {
+            if (leader) tc::mbar_arrive_expect_tx(full_bar(s), 2 * Sh::STAGE_BYTES);
+            if (MODE == kGateUp) {  // even CTA: gate rows, odd CTA: up rows
+              tc::tma_load_2d_pair(b_dst, &tmB, fb, k0, t.e * 2 * p.F + int(rank) * p.F + t.nt * 128);
+            } else {  // A = [dA | dB] of the group, MN-major
+              const int krow = t.goff + k0;
+#pragma unroll
+              for (int i = 0; i < BM / 64; ++i)
+                tc::tma_load_2d_pair(a_dst + i * 64 * 128, &tmA, fb, mt * BM + i * 64, krow);
+            }
+          }
+          if (MODE == kGateUp) {
+            tc::tma_gather4_pair(a_dst + uint32_t(lane) * 512u, &tmA, fb, k0, rows4.x, rows4.y,
+                                 rows4.z, rows4.w);
+          } else if (box < BNH / 64) {
+            tc::tma_gather4_pair(b_dst + uint32_t(box) * 64u * 128u + uint32_t(grp) * 512u, &tmB, fb,
+                                 t.nt * BN + int(rank) * BNH + box * 64, rows4.x, rows4.y, rows4.z,
+                                 rows4.w);
+          }
         }
       }
     }
@@ -915,42 +949,45 @@ __global__ void __launch_bounds__(kThreads, 1)
       uint32_t it = 0;
       bool ok = true;
       for (uint32_t n = 0; ok; ++n) {
-        const int tile = next_tile(n);
-        if (tile < 0) break;
-        const PairTile t = decode(tile);
-        const int mt = 2 * t.mp + int(rank);  // this CTA's 128-row block
-        for (int kb = 0; kb < t.nkb; ++kb, ++it) {
-          const int s = it % STAGES;
-          const uint32_t ph = (it / STAGES) & 1u;
-          if (!tc::mbar_wait(empty_bar(s), ph ^ 1u, kWaitLimitNs, abort_flag)) { fail(abort_flag); ok = false; break; }
-          if (leader) tc::mbar_arrive_expect_tx(full_bar(s), 2 * Sh::STAGE_BYTES);
-          const uint32_t a_dst = sA0 + s * Sh::A_BYTES, b_dst = sB0 + s * Sh::B_BYTES;
-          const uint32_t fb = full_leader + 8u * s;
-          const int k0 = kb * KB;
-          // K-major operands: one box per 64-deep K half (the 128-byte swizzle row), half h
-          // at h * rows * 128 bytes. MN-major operands: one box of 64 columns x KB k-rows per
-          // 64 columns, column block i at i * KB * 128 bytes (half as many loads).
-          if (Tr::A_MN) {  // weight gradients: [dA|dB] or dO of the group, K = group rows
+        const int unit = next_unit(n);
+        if (unit < 0) break;
+        const PairUnit u = decode_unit(unit);
+        for (int j = 0; j < u.cnt && ok; ++j) {
+          const PairTile t = tile_in(u, j);
+          const int mt = 2 * t.mp + int(rank);  // this CTA's 128-row block
+          for (int kb = 0; kb < t.nkb; ++kb, ++it) {
+            const int s = it % STAGES;
+            const uint32_t ph = (it / STAGES) & 1u;
+            if (!tc::mbar_wait(empty_bar(s), ph ^ 1u, kWaitLimitNs, abort_flag)) { fail(abort_flag); ok = false; break; }
+            if (leader) tc::mbar_arrive_expect_tx(full_bar(s), 2 * Sh::STAGE_BYTES);
+            const uint32_t a_dst = sA0 + s * Sh::A_BYTES, b_dst = sB0 + s * Sh::B_BYTES;
+            const uint32_t fb = full_leader + 8u * s;
+            const int k0 = kb * KB;
+            // K-major operands: one box per 64-deep K half (the 128-byte swizzle row), half h
+            // at h * rows * 128 bytes. MN-major operands: one box of 64 columns x KB k-rows per
+            // 64 columns, column block i at i * KB * 128 bytes (half as many loads).
+            if (Tr::A_MN) {  // weight gradients: [dA|dB] or dO of the group, K = group rows
 #pragma unroll
-            for (int i = 0; i < BM / 64; ++i)
-              tc::tma_load_2d_pair(a_dst + i * (KB * 128), &tmA, fb, mt * BM + i * 64, t.goff + k0);
-          } else {
+              for (int i = 0; i < BM / 64; ++i)
+                tc::tma_load_2d_pair(a_dst + i * (KB * 128), &tmA, fb, mt * BM + i * 64, t.goff + k0);
+            } else {
 #pragma unroll
-            for (int h = 0; h < KB / 64; ++h)
-              tc::tma_load_2d_pair(a_dst + h * (BM * 128), &tmA, fb, k0 + h * 64, t.goff + mt * BM);
-          }
-          if (Tr::B_MN) {
-            const int krow = (MODE == kDgradDown ? t.e * p.d : MODE == kDgradGateUp ? t.e * 2 * p.F : t.goff) + k0;
+              for (int h = 0; h < KB / 64; ++h)
+                tc::tma_load_2d_pair(a_dst + h * (BM * 128), &tmA, fb, k0 + h * 64, t.goff + mt * BM);
+            }
+            if (Tr::B_MN) {
+              const int krow = (MODE == kDgradDown ? t.e * p.d : MODE == kDgradGateUp ? t.e * 2 * p.F : t.goff) + k0;
 #pragma unroll
-            for (int i = 0; i < BNH / 64; ++i)
-              tc::tma_load_2d_pair(b_dst + i * (KB * 128), &tmB, fb, t.nt * BN + int(rank) * BNH + i * 64, krow);
-          } else {
-            // kGateUp: even CTA gate rows, odd CTA up rows; kDown: rows of W_down
-            const int brow = MODE == kGateUp ? t.e * 2 * p.F + int(rank) * p.F + t.nt * 128
-                                             : t.e * p.d + t.nt * BN + int(rank) * BNH;
+              for (int i = 0; i < BNH / 64; ++i)
+                tc::tma_load_2d_pair(b_dst + i * (KB * 128), &tmB, fb, t.nt * BN + int(rank) * BNH + i * 64, krow);
+            } else {
+              // kGateUp: even CTA gate rows, odd CTA up rows; kDown: rows of W_down
+              const int brow = MODE == kGateUp ? t.e * 2 * p.F + int(rank) * p.F + t.nt * 128
+                                               : t.e * p.d + t.nt * BN + int(rank) * BNH;
 #pragma unroll
-            for (int h = 0; h < KB / 64; ++h)
-              tc::tma_load_2d_pair(b_dst + h * (BNH * 128), &tmB, fb, k0 + h * 64, brow);
+              for (int h = 0; h < KB / 64; ++h)
+                tc::tma_load_2d_pair(b_dst + h * (BNH * 128), &tmB, fb, k0 + h * 64, brow);
+            }
           }
         }
       }
@@ -971,53 +1008,67 @@ __global__ void __launch_bounds__(kThreads, 1)
       const uint32_t epi_bar_peer = tc::mapa(epi_bar(0), 1);
       uint32_t it = 0;
       bool ok = true, issued = false;
+      uint32_t nt_done = 0;  // tiles issued: tile i accumulates in buffer i % 2
       for (uint32_t n = 0; ok; ++n) {
-        int tile;
+        int unit;
         if (dyn) {
           const int slot = int(n % kRing);
           if (!tc::mbar_wait(ring_bar(slot), (n / kRing) & 1u, kWaitLimitNs, abort_flag)) { fail(abort_flag); break; }
-          tile = s_ring[slot];
+          unit = s_ring[slot];
         } else {
-          tile = static_tile(n);
-          if (tile < 0) break;
+          unit = static_unit(n);
+          if (unit < 0) break;
         }
-        const uint32_t a = n & 1u, aph = (n >> 1) & 1u;
-        if (!tc::mbar_wait(tempty_bar(a), aph ^ 1u, kWaitLimitNs, abort_flag)) { fail(abort_flag); break; }
+        // The buffer of the unit's first tile is free: the epilogue warps are done with
+        // tile nt_done - 2, hence have read the unit that slot n % 2 held before.
+        {
+          const uint32_t a = nt_done & 1u, aph = (nt_done >> 1) & 1u;
+          if (!tc::mbar_wait(tempty_bar(a), aph ^ 1u, kWaitLimitNs, abort_flag)) { fail(abort_flag); break; }
+        }
         if (dyn) {
-          // the epilogue warps of both CTAs learn the tile of buffer a (-1: no more tiles)
-          s_epi[a] = tile;
-          tc::st_cluster_u32(epi_peer + 4u * a, tile);
-          tc::mbar_arrive(epi_bar(a));
-          tc::mbar_arrive_cluster(epi_bar_peer + 8u * a);
+          // the epilogue warps of both CTAs learn the unit (-1: no more units)
+          const uint32_t e_slot = n & 1u;
+          s_epi[e_slot] = unit;
+          tc::st_cluster_u32(epi_peer + 4u * e_slot, unit);
+          tc::mbar_arrive(epi_bar(e_slot));
+          tc::mbar_arrive_cluster(epi_bar_peer + 8u * e_slot);
         }
-        if (tile < 0) break;
+        if (unit < 0) break;
         tc::fence_after_sync();
-        const PairTile t = decode(tile);
-        const uint32_t d_tmem = tmem_base + a * BN;
-        for (int kb = 0; kb < t.nkb; ++kb, ++it) {
-          const int s = it % STAGES;
-          const uint32_t ph = (it / STAGES) & 1u;
-          if (!tc::mbar_wait(full_bar(s), ph, kWaitLimitNs, abort_flag)) { fail(abort_flag); ok = false; break; }
-          tc::fence_after_sync();
-          const uint32_t a_s = sA0 + s * Sh::A_BYTES, b_s = sB0 + s * Sh::B_BYTES;
-#pragma unroll
-          for (int kk = 0; kk < KB / UMMA_K; ++kk) {
-            // K-major: K-half kk / 4 of the stage, 16-wide step kk % 4 inside it (32 bytes
-            // along the swizzled row). MN-major: k-rows 16 kk .. 16 kk + 15 of every
-            // 64-column block (2 KB each), blocks KB * 128 bytes apart.
-            const uint32_t ha = uint32_t(kk >> 2) * (BM * 128), hb = uint32_t(kk >> 2) * (BNH * 128);
-            const int q = kk & 3;
-            const uint64_t ad = Tr::A_MN ? tc::smem_desc_sw128(a_s + kk * 2048, KB * 128, 1024)
-                                         : tc::smem_desc_sw128(a_s + ha + q * 32, 16, 1024);
-            const uint64_t bd = Tr::B_MN ? tc::smem_desc_sw128(b_s + kk * 2048, KB * 128, 1024)
-                                         : tc::smem_desc_sw128(b_s + hb + q * 32, 16, 1024);
-            tc::mma_bf16_pair(d_tmem, ad, bd, IDESC, (kb | kk) != 0);
+        const PairUnit u = decode_unit(unit);
+        for (int j = 0; j < u.cnt && ok; ++j, ++nt_done) {
+          const uint32_t a = nt_done & 1u, aph = (nt_done >> 1) & 1u;
+          if (j > 0) {
+            if (!tc::mbar_wait(tempty_bar(a), aph ^ 1u, kWaitLimitNs, abort_flag)) { fail(abort_flag); ok = false; break; }
+            tc::fence_after_sync();
           }
-          tc::mma_commit_pair_mc(empty_bar(s), 0x3);  // frees the stage in both CTAs
-          issued = true;
+          const PairTile t = tile_in(u, j);
+          const uint32_t d_tmem = tmem_base + a * BN;
+          for (int kb = 0; kb < t.nkb; ++kb, ++it) {
+            const int s = it % STAGES;
+            const uint32_t ph = (it / STAGES) & 1u;
+            if (!tc::mbar_wait(full_bar(s), ph, kWaitLimitNs, abort_flag)) { fail(abort_flag); ok = false; break; }
+            tc::fence_after_sync();
+            const uint32_t a_s = sA0 + s * Sh::A_BYTES, b_s = sB0 + s * Sh::B_BYTES;
+#pragma unroll
+            for (int kk = 0; kk < KB / UMMA_K; ++kk) {
+              // K-major: K-half kk / 4 of the stage, 16-wide step kk % 4 inside it (32 bytes
+              // along the swizzled row). MN-major: k-rows 16 kk .. 16 kk + 15 of every
+              // 64-column block (2 KB each), blocks KB * 128 bytes apart.
+              const uint32_t ha = uint32_t(kk >> 2) * (BM * 128), hb = uint32_t(kk >> 2) * (BNH * 128);
+              const int q = kk & 3;
+              const uint64_t ad = Tr::A_MN ? tc::smem_desc_sw128(a_s + kk * 2048, KB * 128, 1024)
+                                           : tc::smem_desc_sw128(a_s + ha + q * 32, 16, 1024);
+              const uint64_t bd = Tr::B_MN ? tc::smem_desc_sw128(b_s + kk * 2048, KB * 128, 1024)
+                                           : tc::smem_desc_sw128(b_s + hb + q * 32, 16, 1024);
+              tc::mma_bf16_pair(d_tmem, ad, bd, IDESC, (kb | kk) != 0);
+            }
+            tc::mma_commit_pair_mc(empty_bar(s), 0x3);  // frees the stage in both CTAs
+            issued = true;
+          }
+          if (!ok) break;
+          tc::mma_commit_pair_mc(tfull_bar(a), 0x3);  // both halves of the accumulator ready
         }
-        if (!ok) break;
-        tc::mma_commit_pair_mc(tfull_bar(a), 0x3);  // both halves of the accumulator ready
       }
       if (issued) {
         tc::mma_commit_pair(drain_bar);
@@ -1048,35 +1099,66 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       }
     }
-    for (uint32_t n = 0;; ++n) {
-      const uint32_t a = n & 1u, aph = (n >> 1) & 1u;
-      bool ok = true;
-      int tile;
+    uint32_t nt_done = 0;  // tiles finished: tile i is in accumulator buffer i % 2
+    bool ok = true;
+    for (uint32_t n = 0; ok; ++n) {
+      int unit;
       if (dyn) {
-        ok = tc::mbar_wait_cluster(epi_bar(a), aph, kWaitLimitNs, abort_flag);
+        const uint32_t e_slot = n & 1u;
+        ok = tc::mbar_wait_cluster(epi_bar(e_slot), (n >> 1) & 1u, kWaitLimitNs, abort_flag);
         __syncwarp();
         if (!ok) { fail(abort_flag); break; }
-        tile = s_epi[a];
+        unit = s_epi[e_slot];
       } else {
-        tile = static_tile(n);
+        unit = static_unit(n);
       }
-      if (tile < 0) break;
-      const PairTile t = decode(tile);
-      const int mt = 2 * t.mp + int(rank);
-      const bool mine = mt < t.mtiles;  // this CTA's row block exists
-      ok = tc::mbar_wait(tfull_bar(a), aph, kWaitLimitNs, abort_flag);
-      __syncwarp();
-      if (!ok) { fail(abort_flag); break; }
-      tc::fence_after_sync();
-      if (mine) {
+      if (unit < 0) break;
+      const PairUnit u = decode_unit(unit);
+      for (int j = 0; j < u.cnt; ++j, ++nt_done) {
+        const uint32_t a = nt_done & 1u, aph = (nt_done >> 1) & 1u;
+        const PairTile t = tile_in(u, j);
+        const int mt = 2 * t.mp + int(rank);
+        const bool mine = mt < t.mtiles;  // this CTA's row block exists
+        ok = tc::mbar_wait(tfull_bar(a), aph, kWaitLimitNs, abort_flag);
+        __syncwarp();
+        if (!ok) { fail(abort_flag); break; }
+        tc::fence_after_sync();
         const uint32_t tb = tmem_base + (uint32_t(q * 32) << 16) + a * BN;
-        epilogue_tile<MODE, BN>(p, &tmO, stage, lane, tb,
-                                size_t(t.goff) + size_t(mt) * BM + r_in_tile,
-                                mt * BM + r_in_tile, t.e, t.nt, half);
+        if (Tr::WGRAD) {
+          // Weight gradients: the whole column half into registers with one wait, the
+          // accumulator back to the MMA issuer, then the stores. A light expert's tile
+          // (one or two k-blocks) takes less MMA time than its epilogue, which sets the pace
+          // there: measured ~4,600 cycles per tile with a load and a wait per 32 columns.
+          uint32_t r[BN / 2];
+          if (mine) {
+#pragma unroll
+            for (int c = 0; c < BN / 2; c += 32)
+              tc::tmem_ld_32x32b_x32(tb + half * (BN / 2) + c, *reinterpret_cast<uint32_t(*)[32]>(&r[c]));
+            tc::tmem_ld_wait();
+          }
+          tc::fence_before_sync();
+          __syncwarp();
+          if (lane == 0) tc::mbar_arrive_cluster(tempty_leader + 8u * a);
+          if (mine) {
+            const int trow = t.e * (p.m_tiles_w * BM) + mt * BM + q * 32;
+#pragma unroll
+            for (int c = 0; c < BN / 2; c += 32) {
+              uint4 v[4];
+              pack32(*reinterpret_cast<const uint32_t(*)[32]>(&r[c]), v);
+              stage_and_store(&tmO, stage, lane, v, t.nt * BN + half * (BN / 2) + c, trow);
+            }
+          }
+          continue;
+        }
+        if (mine) {
+          epilogue_tile<MODE, BN>(p, &tmO, stage, lane, tb,
+                                  size_t(t.goff) + size_t(mt) * BM + r_in_tile,
+                                  mt * BM + r_in_tile, t.e, t.nt, half);
+        }
+        tc::fence_before_sync();
+        __syncwarp();
+        if (lane == 0) tc::mbar_arrive_cluster(tempty_leader + 8u * a);
       }
-      tc::fence_before_sync();
-      __syncwarp();
-      if (lane == 0) tc::mbar_arrive_cluster(tempty_leader + 8u * a);
     }
     if (lane == 0) tc::bulk_wait0();  // this warp's output stores are complete
     __syncwarp();

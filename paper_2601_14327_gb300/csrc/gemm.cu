@@ -971,9 +971,13 @@ __global__ void __launch_bounds__(kThreads, 1)
               for (int i = 0; i < BM / 64; ++i)
                 tc::tma_load_2d_pair(a_dst + i * (KB * 128), &tmA, fb, mt * BM + i * 64, t.goff + k0);
             } else {
+              // A row block past the expert's last one (the odd CTA of a pair tile over an
+              // odd number of blocks): a box wholly above the tensor, which TMA fills with
+              // zeros without reading memory, instead of the next expert's rows
+              const int arow = mt < t.mtiles ? t.goff + mt * BM : -2 * BM;
 #pragma unroll
               for (int h = 0; h < KB / 64; ++h)
-                tc::tma_load_2d_pair(a_dst + h * (BM * 128), &tmA, fb, k0 + h * 64, t.goff + mt * BM);
+                tc::tma_load_2d_pair(a_dst + h * (BM * 128), &tmA, fb, k0 + h * 64, arow);
             }
             if (Tr::B_MN) {
               const int krow = (MODE == kDgradDown ? t.e * p.d : MODE == kDgradGateUp ? t.e * 2 * p.F : t.goff) + k0;

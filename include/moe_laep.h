@@ -265,7 +265,8 @@ int moe_permute_noalloc(const uint16_t *x, const int32_t *topk_idx, const int32_
  * expert first (the longest-processing-time order of Algorithm 2's greedy) and
  * CTA pairs that run out of work take the next tile of the list from a counter in
  * ws, so the heaviest tile left always goes to the least-loaded pair (Algorithm 2
- * with the GPU's CTA pairs as its devices, applied online); the other GEMMs'
+ * with the GPU's CTA pairs as its devices, applied online; a light expert's tiles
+ * of 1-7 k-blocks of 128 rows are claimed 8, 4 or 2 at a time); the other GEMMs'
  * tiles all cost the same, are listed in expert order and each pair takes every
  * 76th one. A tile's arithmetic does not depend on which pair runs it: results
  * are bitwise reproducible.

@@ -110,6 +110,10 @@ struct GemmParams {
   // caller's workspace); dynamic = 0 walks the list with a fixed stride instead.
   int *sched_ctr;
   int dynamic;
+  // Activation GEMMs split between two launches (0: no split): 1 = the CTA-pair kernel
+  // takes each group's whole pairs of 128-row blocks only, 2 = the one-SM kernel takes the
+  // last block of each group with an odd number of blocks only.
+  int rows_split;
 };
 
 struct Tile {
@@ -422,7 +426,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       s_prefix[i] = acc;
       const int key = sort_key(s_order[i]);
       if (key < 0) continue;  // pruned
-      acc += Tr::WGRAD ? p.m_tiles_w * p.n_tiles : (key / BM) * p.n_tiles;
+      const int mt = p.rows_split == 2 ? (key / BM) & 1 : key / BM;  // odd last block only
+      acc += Tr::WGRAD ? p.m_tiles_w * p.n_tiles : mt * p.n_tiles;
     }
     s_prefix[E] = acc;
   }
@@ -442,8 +447,13 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int local = tile - s_prefix[lo];
     t.e = s_order[lo];
     t.goff = s_goff[t.e];
-    t.mt = local / p.n_tiles;
-    t.nt = local - t.mt * p.n_tiles;
+    if (!Tr::WGRAD && p.rows_split == 2) {  // the group's last (odd) block, every N tile
+      t.mt = (s_goff[t.e + 1] - t.goff) / BM - 1;
+      t.nt = local;
+    } else {
+      t.mt = local / p.n_tiles;
+      t.nt = local - t.mt * p.n_tiles;
+    }
     t.nkb = Tr::WGRAD ? (s_goff[t.e + 1] - t.goff) / BK : p.nkb;
     return t;
   };
@@ -767,7 +777,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         continue;
       }
       const int mt = Tr::WGRAD ? p.m_tiles_w : key / BM;
-      const int tiles = ((mt + 1) / 2) * p.n_tiles;
+      // pairs of row blocks; with rows_split == 1 a last odd block is left to the one-SM kernel
+      const int tiles = ((p.rows_split == 1 ? mt : mt + 1) / 2) * p.n_tiles;
       const int g = dyn ? unit_tiles(key / KB) : 1;
       acc += (tiles + g - 1) / g;
     }
@@ -800,7 +811,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     u.mtiles = Tr::WGRAD ? p.m_tiles_w : rows / BM;
     const int g = dyn ? unit_tiles(u.nkb) : 1;
     u.lt0 = (unit - s_prefix[lo]) * g;
-    u.cnt = min(g, ((u.mtiles + 1) / 2) * p.n_tiles - u.lt0);
+    u.cnt = min(g, ((p.rows_split == 1 ? u.mtiles : u.mtiles + 1) / 2) * p.n_tiles - u.lt0);
     return u;
   };
   // Tile j of a unit: the expert's tile lt0 + j as (row pair, column tile).
@@ -1275,6 +1286,20 @@ int launch_pair(const CUtensorMap &a, const CUtensorMap &b, const CUtensorMap &o
   return moe::launch_status(what);
 }
 
+// Row-block split of the activation GEMMs (see run_gemm_out): on when the grouped layout
+// has at least 2^18 rows. Measured on GB300 (same box, split on / off): T=65536,
+// d_model=7168, 171 live experts 94.5-95.0 / 95.2-95.4 ms per layer step; T=32768 and
+// T=16384 at d_model=4096 unchanged (the second launch costs what the half tiles save).
+// MOE_GEMM_SPLIT=0 turns it off (A/B runs).
+bool split_rows(uint64_t rows) {
+  static int on = -1;
+  if (on < 0) {
+    const char *e = getenv("MOE_GEMM_SPLIT");
+    on = (e != nullptr && e[0] == '0') ? 0 : 1;
+  }
+  return on && rows >= (uint64_t(1) << 18);
+}
+
 // Builds the tensor maps for one GEMM and launches it. A: [a_rows, a_cols] row-major
 // bf16; B likewise. N = output columns (for kGateUp: 2F, in tiles of 128 gate + 128 up).
 // The output p.out is [o_rows, o_cols] row-major bf16.
@@ -1331,8 +1356,24 @@ int run_gemm_out(int N, const void *a_base, uint64_t a_rows, uint64_t a_cols, co
         return BN == 256 ? launch_pair<MODE, 256, true>(ma, mb, mo, p, s, what)
                          : launch_pair<MODE, 128, true>(ma, mb, mo, p, s, what);
     }
-    return BN == 256 ? launch_pair<MODE, 256, false>(ma, mb, mo, p, s, what)
-                     : launch_pair<MODE, 128, false>(ma, mb, mo, p, s, what);
+    if (Tr::WGRAD || !split_rows(a_rows))
+      return BN == 256 ? launch_pair<MODE, 256, false>(ma, mb, mo, p, s, what)
+                       : launch_pair<MODE, 128, false>(ma, mb, mo, p, s, what);
+    // Activation GEMMs on many rows: a group's last block of an odd number of 128-row
+    // blocks would be half of a 256-row pair tile whose other half is computed and dropped;
+    // the one-SM kernel (128-row tiles) takes those blocks in a second launch.
+    GemmParams q = p;
+    q.rows_split = 1;
+    if ((st = BN == 256 ? launch_pair<MODE, 256, false>(ma, mb, mo, q, s, what)
+                        : launch_pair<MODE, 128, false>(ma, mb, mo, q, s, what)))
+      return st;
+    CUtensorMap mb1;  // the one-SM kernel's B boxes
+    if ((st = Tr::B_MN ? make_map(&mb1, b_base, b_rows, b_cols, 64, BK, what)
+                       : make_map(&mb1, b_base, b_rows, b_cols, BK, 128, what)))
+      return st;
+    q.rows_split = 2;
+    return BN == 256 ? launch_one<MODE, 256>(ma, mb1, mo, q, s, what)
+                     : launch_one<MODE, 128>(ma, mb1, mo, q, s, what);
   }
   return BN == 256 ? launch_one<MODE, 256>(ma, mb, mo, p, s, what)
                    : launch_one<MODE, 128>(ma, mb, mo, p, s, what);

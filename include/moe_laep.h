@@ -268,7 +268,8 @@ int moe_permute_noalloc(const uint16_t *x, const int32_t *topk_idx, const int32_
  * with the GPU's CTA pairs as its devices, applied online; a light expert's tiles
  * of 1-7 k-blocks of 128 rows are claimed 8, 4 or 2 at a time); the other GEMMs'
  * tiles all cost the same, are listed in expert order and each pair takes every
- * 76th one. A tile's arithmetic does not depend on which pair runs it: results
+ * 76th one (with rows_cap >= 2^18, a group's odd last 128-row block is computed
+ * by a second, one-SM launch on the same stream). A tile's arithmetic does not depend on which pair runs it: results
  * are bitwise reproducible.
  * Limits: d % 128 == 0, F % 128 == 0, all pointers 16-byte aligned.
  */

@@ -534,6 +534,26 @@ def test_dynamic_schedule_equals_fixed_stride(tmp_path):
             assert torch.equal(dyn[n], static[i][n]), (G.SCHEDULE_CASES[i], n)
 
 
+def test_row_block_split_equals_single_launch(tmp_path):
+    """On 2^18 or more grouped rows the activation GEMMs are two launches: the CTA-pair
+    kernel over whole pairs of 128-row blocks, then the one-SM kernel over each group's odd
+    last block. Every output and gradient equals, bit for bit, the single CTA-pair launch
+    (MOE_GEMM_SPLIT=0, read once per process, so that half runs in a child process): both
+    kernels add the same products in the same order."""
+    import gpu_split_check as G
+    path = str(tmp_path / "single.pt")
+    env = dict(os.environ, MOE_GEMM_SPLIT="0")
+    script = os.path.join(os.path.dirname(os.path.abspath(__file__)), "gpu_split_check.py")
+    r = subprocess.run([sys.executable, script, path], env=env, capture_output=True, text=True,
+                       timeout=900)
+    assert r.returncode == 0, r.stdout[-2000:] + r.stderr[-4000:]
+    single = torch.load(path)
+    for i, split in enumerate(G.run_cases()):
+        assert split["odd_groups"] > 0, G.SPLIT_CASES[i]
+        for n in G.NAMES:
+            assert torch.equal(split[n], single[i][n]), (G.SPLIT_CASES[i], n)
+
+
 def test_pruned_experts_weight_gradients_untouched():
     """Pruned experts (LAEP mask 0) get no tile and no store in the weight-gradient GEMMs:
     their gradient buffers keep what the caller left there. A live expert that received no

@@ -62,6 +62,28 @@ template <int MODE> struct Traits {
   static constexpr bool WGRAD = (MODE == kWgradDown || MODE == kWgradGateUp);
 };
 
+// In-place scan by one warp of s[1..n] (n <= 256): afterwards s[i] = s[1] + ... + s[i] and
+// s[0] = 0. With the count of list position j stored at s[j + 1], s[i] is then the first
+// tile (or unit) of position i and s[n] the total.
+__device__ __forceinline__ void warp_prefix_counts(int *s, int n, int lane) {
+  const int c = (n + 31) >> 5;
+  const int lo = lane * c + 1, hi = min(n, lo + c - 1);
+  int sum = 0;
+  for (int i = lo; i <= hi; ++i) {
+    sum += s[i];
+    s[i] = sum;
+  }
+  int incl = sum;
+#pragma unroll
+  for (int off = 1; off < 32; off <<= 1) {
+    const int v = __shfl_up_sync(0xffffffffu, incl, off);
+    if (lane >= off) incl += v;
+  }
+  const int excl = incl - sum;
+  for (int i = lo; i <= hi; ++i) s[i] += excl;
+  if (lane == 0) s[0] = 0;
+}
+
 template <int BN> struct Shape {
   static constexpr int STAGES = BN == 256 ? 4 : 6;
   static constexpr uint32_t A_BYTES = BM * BK * 2;
@@ -69,7 +91,7 @@ template <int BN> struct Shape {
   static constexpr uint32_t STAGE_BYTES = A_BYTES + B_BYTES;
   static constexpr int NBARS = 2 * STAGES + 5;
   static constexpr size_t SMEM = 1024 + size_t(STAGES) * STAGE_BYTES + NBARS * 8 +
-                                 (4 + 257 + 256 + 257) * 4 + 1024 + kEpiWarps * 2048;
+                                 (4 + 257 + 256 + 257 + 256) * 4 + 1024 + kEpiWarps * 2048;
   static constexpr uint32_t TMEM_COLS = 2 * BN;
 };
 
@@ -359,8 +381,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   int *s_goff = misc + 4;          // [E+1]
   int *s_order = s_goff + 257;     // [E]   experts in schedule order
   int *s_prefix = s_order + 256;   // [E+1] first tile of each scheduled expert
+  int *s_key = s_prefix + 257;     // [E]   rows of each expert, -1 when pruned
   const uint32_t stage_base =
-      (tc::smem_u32(s_prefix + 257) + 1023u) & ~1023u;  // epilogue staging, 2 KB per warp
+      (tc::smem_u32(s_key + 256) + 1023u) & ~1023u;  // epilogue staging, 2 KB per warp
   volatile int *abort_flag = misc + 1;
   volatile int no_abort = 0;
 
@@ -402,35 +425,32 @@ __global__ void __launch_bounds__(kThreads, 1)
   // k-blocks (their zero gradient). Activation GEMMs: expert order.
   for (int e = threadIdx.x; e <= E; e += kThreads) s_goff[e] = p.group_offsets[e];
   __syncthreads();
-  auto sort_key = [&](int e) {
+  for (int e = threadIdx.x; e < E; e += kThreads) {
     const int rows = s_goff[e + 1] - s_goff[e];
-    return (Tr::WGRAD && p.active_mask != nullptr && p.active_mask[e] == 0) ? -1 : rows;
-  };
+    s_key[e] = (Tr::WGRAD && p.active_mask != nullptr && p.active_mask[e] == 0) ? -1 : rows;
+  }
+  __syncthreads();
   for (int e = threadIdx.x; e < E; e += kThreads) {
     if (!Tr::WGRAD) {  // equal-cost tiles: expert order, the grouped layout's memory order
       s_order[e] = e;
       continue;
     }
-    const int ce = sort_key(e);
+    const int ce = s_key[e];
     int r = 0;
     for (int q = 0; q < E; ++q) {
-      const int cq = sort_key(q);
+      const int cq = s_key[q];
       r += (cq > ce) || (cq == ce && q < e);
     }
     s_order[r] = e;
   }
   __syncthreads();
-  if (threadIdx.x == 0) {
-    int acc = 0;
-    for (int i = 0; i < E; ++i) {
-      s_prefix[i] = acc;
-      const int key = sort_key(s_order[i]);
-      if (key < 0) continue;  // pruned
-      const int mt = p.rows_split == 2 ? (key / BM) & 1 : key / BM;  // odd last block only
-      acc += Tr::WGRAD ? p.m_tiles_w * p.n_tiles : mt * p.n_tiles;
-    }
-    s_prefix[E] = acc;
+  for (int i = threadIdx.x; i < E; i += kThreads) {  // tiles of list position i
+    const int key = s_key[s_order[i]];
+    const int mt = p.rows_split == 2 ? (key / BM) & 1 : key / BM;  // odd last block only
+    s_prefix[i + 1] = key < 0 ? 0 : Tr::WGRAD ? p.m_tiles_w * p.n_tiles : mt * p.n_tiles;
   }
+  __syncthreads();
+  if (warp == 0) warp_prefix_counts(s_prefix, E, lane);
   tc::fence_before_sync();
   __syncthreads();
   tc::fence_after_sync();
@@ -630,7 +650,7 @@ template <int BN, int KB> struct PairShape {
   // full/empty per stage, tfull/tempty per accumulator, drain, tile ring, epilogue tile
   static constexpr int NBARS = 2 * STAGES + 5 + kRing + 2;
   static constexpr size_t SMEM = 1024 + size_t(STAGES) * STAGE_BYTES + NBARS * 8 +
-                                 (4 + 257 + 256 + 257 + kRing + 2) * 4 + 1024 + kEpiWarps * 2048;
+                                 (4 + 257 + 256 + 257 + 256 + kRing + 2) * 4 + 1024 + kEpiWarps * 2048;
   static constexpr uint32_t TMEM_COLS = 2 * BN;
 };
 
@@ -688,7 +708,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   int *s_goff = misc + 4;
   int *s_order = s_goff + 257;
   int *s_prefix = s_order + 256;
-  volatile int *s_ring = s_prefix + 257;  // [kRing] tile hand-off (see kRing)
+  int *s_key = s_prefix + 257;            // [E] rows of each expert, -1 when pruned (wgrad)
+  volatile int *s_ring = s_key + 256;     // [kRing] tile hand-off (see kRing)
   volatile int *s_epi = s_ring + kRing;   // [2] tile of each accumulator buffer, for the epilogue
   const uint32_t stage_base =
       (tc::smem_u32(const_cast<int *>(s_epi + 2)) + 1023u) & ~1023u;  // epilogue staging, 2 KB per warp
@@ -725,6 +746,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc::mbar_init(drain_bar, 1);
     tc::fence_mbar_init();
     misc[1] = 0;
+    misc[2] = 0;  // live experts without rows (weight gradients)
+    misc[3] = 0;  // pruned experts
   }
   if (warp == 0 && lane == 0) {
     tc::tma_prefetch_desc(&tmA);
@@ -746,46 +769,46 @@ __global__ void __launch_bounds__(kThreads, 1)
   // which follows the grouped layout in memory (measured 1-2% faster than heaviest first).
   for (int e = threadIdx.x; e <= E; e += kThreads) s_goff[e] = p.group_offsets[e];
   __syncthreads();
-  auto sort_key = [&](int e) {
+  for (int e = threadIdx.x; e < E; e += kThreads) {
     const int rows = s_goff[e + 1] - s_goff[e];
-    return (Tr::WGRAD && p.active_mask != nullptr && p.active_mask[e] == 0) ? -1 : rows;
-  };
+    s_key[e] = (Tr::WGRAD && p.active_mask != nullptr && p.active_mask[e] == 0) ? -1 : rows;
+  }
+  __syncthreads();
   for (int e = threadIdx.x; e < E; e += kThreads) {
     if (!Tr::WGRAD) {  // equal-cost tiles: expert order, the grouped layout's memory order
       s_order[e] = e;
       continue;
     }
-    const int ce = sort_key(e);
+    const int ce = s_key[e];
     int r = 0;
     for (int q = 0; q < E; ++q) {
-      const int cq = sort_key(q);
+      const int cq = s_key[q];
       r += (cq > ce) || (cq == ce && q < e);
     }
     s_order[r] = e;
   }
   __syncthreads();
   const bool dyn = Tr::WGRAD && p.dynamic;
-  if (threadIdx.x == 0) {
-    // s_prefix counts claim units: tiles, or groups of light experts' tiles (dyn)
-    int acc = 0, n_empty = 0, n_pruned = 0;
-    for (int i = 0; i < E; ++i) {
-      s_prefix[i] = acc;
-      const int e = s_order[i];
-      const int key = sort_key(e);
-      if (Tr::WGRAD && key <= 0) {
-        if (key < 0) ++n_pruned; else ++n_empty;
-        continue;
-      }
+  // claim units of list position i (tiles, or groups of light experts' tiles when dyn) at
+  // s_prefix[i + 1], then one warp's scan; measured before as a loop of one thread over the
+  // experts, ~9.5 us per launch (36 us in the weight gradients, with the mask read from
+  // global memory by the sort)
+  for (int i = threadIdx.x; i < E; i += kThreads) {
+    const int key = s_key[s_order[i]];
+    int units = 0;
+    if (Tr::WGRAD && key <= 0) {
+      atomicAdd(&misc[key < 0 ? 3 : 2], 1);  // pruned / live without rows: no tile
+    } else {
       const int mt = Tr::WGRAD ? p.m_tiles_w : key / BM;
       // pairs of row blocks; with rows_split == 1 a last odd block is left to the one-SM kernel
       const int tiles = ((p.rows_split == 1 ? mt : mt + 1) / 2) * p.n_tiles;
       const int g = dyn ? unit_tiles(key / KB) : 1;
-      acc += (tiles + g - 1) / g;
+      units = (tiles + g - 1) / g;
     }
-    s_prefix[E] = acc;
-    misc[2] = n_empty;
-    misc[3] = n_pruned;
+    s_prefix[i + 1] = units;
   }
+  __syncthreads();
+  if (warp == 0) warp_prefix_counts(s_prefix, E, lane);
   tc::fence_before_sync();
   __syncthreads();
   tc::cluster_sync();  // barriers of both CTAs initialized before any remote use

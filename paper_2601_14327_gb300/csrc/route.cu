@@ -338,7 +338,9 @@ __global__ void __launch_bounds__(kRouteThreads, 4) route_topk_kernel(
     // Order-preserving unsigned keys of the logits (a larger float gives a larger key,
     // -0 is taken as +0 so that equal logits tie; 0 marks an expert that cannot be
     // selected). Each round takes the warp maximum of the keys with one redux and the
-    // lowest expert holding it with one ballot per slot.
+    // lowest expert holding it with a second: a lane offers expert 32 j + lane for its
+    // lowest slot j holding its own maximum, when that equals the warp's. (One ballot per
+    // slot and round before: ~1,200 warp instructions per token at 192 experts, top-8.)
     unsigned key[TK];
 #pragma unroll
     for (int j = 0; j < TK; ++j) {
@@ -351,15 +353,15 @@ __global__ void __launch_bounds__(kRouteThreads, 4) route_topk_kernel(
     for (int s = 0; s < 8; ++s) {
       if (s >= k) break;
       unsigned best = 0;
+      int bj = 0;
 #pragma unroll
-      for (int j = 0; j < TK; ++j) best = max(best, key[j]);
+      for (int j = 0; j < TK; ++j)
+        if (key[j] > best) {  // strict: the lowest slot keeps a tie
+          best = key[j];
+          bj = j;
+        }
       const unsigned m = __reduce_max_sync(0xffffffffu, best);
-      int be = -1;
-#pragma unroll
-      for (int j = TK - 1; j >= 0; --j) {  // the lowest slot j wins, then the lowest lane
-        const unsigned bal = __ballot_sync(0xffffffffu, key[j] == m);
-        if (bal) be = 32 * j + __ffs(bal) - 1;
-      }
+      const int be = int(__reduce_min_sync(0xffffffffu, best == m ? unsigned(32 * bj + lane) : ~0u));
 #pragma unroll
       for (int j = 0; j < TK; ++j)
         if (32 * j + lane == be) key[j] = 0u;
@@ -527,7 +529,12 @@ int launch_route(const uint16_t *x, const float *w, const float *b, const uint8_
   int splits = 0;
   if (lin == nullptr)
     if (int st = launch_route_tc(x, w, T, d, E, NE, w3, partial, &splits, s)) return st;
-  const int grid2 = (T + kRouteThreads / 32 - 1) / (kRouteThreads / 32);
+  // one warp per token, grid-stride over the tokens; four blocks per SM, so that each
+  // block's shared histogram sums ~100 tokens' assignments before its global atomics (one
+  // block per 8 tokens sent 512k atomics to the counters at T=65536, top-8; the heaviest
+  // expert's counter took ~60k of them one after another)
+  const int grid2 = int(std::min<int64_t>((int64_t(T) + kRouteThreads / 32 - 1) / (kRouteThreads / 32),
+                                          int64_t(moe::num_sms()) * 4));
   MOE_LAUNCH("route_topk", s, route_topk_kernel<NE><<<grid2, kRouteThreads, 0, s>>>(
                                   partial, splits, lin, b, mask, T, E, k, lout, idx, gate, counts));
   return moe::launch_status("moe_route: top-k");

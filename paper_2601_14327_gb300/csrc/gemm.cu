@@ -625,19 +625,22 @@ __global__ void __launch_bounds__(kThreads, 1)
 // (it expects both CTAs' bytes); the MMA commit arrives on the `empty` and
 // `tfull` barriers of both CTAs; both CTAs' epilogue warps arrive on the even
 // CTA's `tempty` barrier. Tiles whose odd row block lies past the group (a group
-// with an odd number of 128-row blocks) are computed but not stored.
+// with an odd number of 128-row blocks) are computed on a zero-filled A box and not
+// stored; on 2^18 or more grouped rows the activation GEMMs leave those blocks to the
+// one-SM kernel (see run_gemm_out).
 // ============================================================================
 // KB = k-block depth of one ring stage: 128 (two 64-wide swizzle blocks of each
 // operand, K-half h at h * 16 KB of A and h * BNH * 128 bytes of B), or 64 for the
 // gathered-operand variant. Deeper stages halve the barrier waits, descriptor setup and
 // commits per FLOP (measured -2.5% to -4.4% cycles per k-block) at the same bytes in flight.
-// Tile hand-off ring of the CTA-pair kernel: the even CTA's producer claims tiles and
-// publishes each one in a slot of both CTAs' rings; the odd CTA's producer and the MMA
-// issuer read it there. A slot is rewritten kRing tiles later, which the load ring's
-// STAGES (< kRing) bound: a producer can run at most STAGES k-blocks, hence STAGES tiles,
-// ahead of the MMAs that need the other readers' progress.
+// Claim hand-off ring of the CTA-pair kernel: the even CTA's producer claims units (a
+// tile, or several tiles of a light expert) and publishes each one in a slot of both
+// CTAs' rings; the odd CTA's producer and the MMA issuer read it there. A slot is
+// rewritten kRing units later, which the load ring's STAGES (< kRing) bound: a producer
+// can run at most STAGES k-blocks, hence STAGES units, ahead of the MMAs that need the
+// other readers' progress.
 constexpr int kRing = 16;
-// Row pairs per block of the weight-gradient tile order (see decode).
+// Row pairs per block of the weight-gradient tile order (see tile_in).
 constexpr int kWgradBlock = 8;
 
 template <int BN, int KB> struct PairShape {
@@ -709,8 +712,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   int *s_order = s_goff + 257;
   int *s_prefix = s_order + 256;
   int *s_key = s_prefix + 257;            // [E] rows of each expert, -1 when pruned (wgrad)
-  volatile int *s_ring = s_key + 256;     // [kRing] tile hand-off (see kRing)
-  volatile int *s_epi = s_ring + kRing;   // [2] tile of each accumulator buffer, for the epilogue
+  volatile int *s_ring = s_key + 256;     // [kRing] unit hand-off (see kRing)
+  volatile int *s_epi = s_ring + kRing;   // [2] unit of each parity of the unit count, for the epilogue
   const uint32_t stage_base =
       (tc::smem_u32(const_cast<int *>(s_epi + 2)) + 1023u) & ~1023u;  // epilogue staging, 2 KB per warp
   volatile int *abort_flag = misc + 1;
